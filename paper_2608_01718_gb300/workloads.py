@@ -1,0 +1,230 @@
+"""Seeded synthetic workloads for the two-stage lookahead lookup.
+
+This module only draws inputs: cache entries (key embedding, lookahead-prefix embedding, prefix token ids) and
+query batches (query embedding, the query's own k-token prefix embedding and ids). It holds none of the lookup's
+arithmetic and is shared by the CUDA path's harness and by the oracle's tests.
+
+The inputs stand in for what the paper's embedding model and draft LLM produce on its datasets (BGE-large 1024-d
+or MiniLM 384-d embeddings, greedy k-token prefixes; §4.1 "LLMs and Embedding Models"). Those datasets are not
+used here. The recipe:
+
+* cluster centres: uniform random unit vectors;
+* entry i: cluster a_i uniform; key = normalise(centre[a_i] + noise), where noise is Gaussian with expected norm
+  ``cluster_sigma`` (per-component std ``cluster_sigma / sqrt(d)``); prefix embedding = an independent uniform unit
+  vector; prefix ids uniform over the vocabulary;
+* queries, shuffled within the batch:
+  - near-duplicate (benign paraphrase): normalise(key_t + noise of norm ``near_sigma``), carrying entry t's exact
+    prefix embedding and ids (same greedy response prefix);
+  - random: a uniform unit vector with a fresh prefix;
+  - collision (the threat model's key collision): normalise(key_t + noise of norm ``coll_sigma``) with a fresh
+    prefix embedding and fresh ids (a semantically distinct response);
+* targets t are uniform over the entries present at generation time, or Zipf(s) over a seeded permutation of them.
+
+Noise is read as a vector whose expected norm is sigma. Read per component instead, a near-duplicate at d=384 and
+sigma=0.05 would have cosine ~0.71 to its target and would never clear a 0.85 key threshold.
+
+Everything is generated in fixed row chunks from counter-derived seeds, so that any chunk of the store can be
+regenerated on its own (the oracle reads the store chunk by chunk for caches too large for host memory).
+"""
+from __future__ import annotations
+
+import dataclasses
+import hashlib
+import math
+from typing import Iterator
+
+import torch
+
+NEAR, RANDOM, COLLISION = 0, 1, 2
+CLASS_NAMES = {NEAR: "near-duplicate", RANDOM: "random", COLLISION: "collision"}
+
+# rows per generated store chunk; fixed so that chunk i is always the same rows
+CHUNK_ROWS = 1 << 18
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    n: int                      # entries in the cache (initial entries for the serve loop)
+    d: int                      # embedding dimension (keys and prefix embeddings)
+    k: int                      # lookahead window: prefix token ids per entry
+    vocab: int
+    clusters: int
+    batch: int                  # queries per lookup
+    mix: tuple                  # (near-duplicate, random, collision) fractions
+    tau_c: float                # key (query) threshold
+    tau_a: float                # lookahead (prefix) threshold
+    top_c: int
+    cluster_sigma: float = 0.15
+    near_sigma: float = 0.05
+    coll_sigma: float = 0.02
+    key_dtype: str = "bf16"     # dtype the keys and prefix embeddings are handed to insert in
+    zipf: float | None = None   # Zipf exponent over targets, None = uniform
+    steps: int = 1              # serve-loop steps (batches); 1 = a single lookup
+    seed: int = 20260801
+
+    def scaled(self, **kw) -> "Workload":
+        return dataclasses.replace(self, **kw)
+
+    @property
+    def store_bytes(self) -> int:
+        return self.n * (4 * self.d + 4 * self.k)
+
+
+WORKLOADS = {
+    # Tiny reference cache (fp32 keys rounded to bf16 at insert).
+    "tiny-4k": Workload("tiny-4k", n=4096, d=384, k=8, vocab=32000, clusters=64, batch=64,
+                        mix=(0.4, 0.3, 0.3), tau_c=0.85, tau_a=0.80, top_c=4, key_dtype="f32"),
+    # Mid cache, bandwidth-bound scan (the headline benchmark workload).
+    "mid-1m": Workload("mid-1m", n=1 << 20, d=768, k=16, vocab=128256, clusters=4096, batch=32,
+                       mix=(0.5, 0.3, 0.2), tau_c=0.90, tau_a=0.80, top_c=8),
+    # Large cache near HBM capacity, Zipf(1.1) popularity of near-duplicate targets.
+    "large-16m": Workload("large-16m", n=1 << 24, d=1024, k=16, vocab=128256, clusters=4096, batch=128,
+                          mix=(0.5, 0.3, 0.2), tau_c=0.90, tau_a=0.80, top_c=8, zipf=1.1),
+    # Large query batch: a dense contraction on the tensor cores.
+    "batch-4m": Workload("batch-4m", n=1 << 22, d=768, k=16, vocab=128256, clusters=4096, batch=8192,
+                         mix=(0.6, 0.25, 0.15), tau_c=0.88, tau_a=0.80, top_c=16),
+    # Streaming serve loop: 1000 batches, every miss appended.
+    "serve-2m": Workload("serve-2m", n=1 << 21, d=768, k=32, vocab=128256, clusters=4096, batch=256,
+                         mix=(0.45, 0.35, 0.2), tau_c=0.90, tau_a=0.80, top_c=8, steps=1000),
+}
+
+
+def sub_seed(master: int, tag: str, index: int = 0) -> int:
+    h = hashlib.sha256(f"{master}/{tag}/{index}".encode()).digest()
+    return int.from_bytes(h[:8], "little") >> 2
+
+
+def _gen(w: Workload, tag: str, index: int, device) -> torch.Generator:
+    g = torch.Generator(device=device)
+    g.manual_seed(sub_seed(w.seed, tag, index))
+    return g
+
+
+def _unit(x: torch.Tensor) -> torch.Tensor:
+    return x / x.norm(dim=1, keepdim=True)
+
+
+def centres(w: Workload, device="cpu") -> torch.Tensor:
+    g = _gen(w, "centres", 0, device)
+    return _unit(torch.randn((w.clusters, w.d), generator=g, device=device, dtype=torch.float32))
+
+
+def _emb_dtype(w: Workload) -> torch.dtype:
+    return torch.float32 if w.key_dtype == "f32" else torch.bfloat16
+
+
+def store_chunk(w: Workload, index: int, device="cpu", cent: torch.Tensor | None = None) -> dict:
+    """Rows [index*CHUNK_ROWS, min(n, (index+1)*CHUNK_ROWS)) of the initial store."""
+    j0 = index * CHUNK_ROWS
+    rows = min(w.n, j0 + CHUNK_ROWS) - j0
+    if rows <= 0:
+        raise IndexError(f"chunk {index} is past the {w.n}-row store")
+    if cent is None:
+        cent = centres(w, device)
+    g = _gen(w, "store", index, device)
+    cluster = torch.randint(0, w.clusters, (rows,), generator=g, device=device)
+    noise = torch.randn((rows, w.d), generator=g, device=device) * (w.cluster_sigma / math.sqrt(w.d))
+    key = _unit(cent[cluster] + noise)
+    del noise
+    prefix = _unit(torch.randn((rows, w.d), generator=g, device=device))
+    ids = torch.randint(0, w.vocab, (rows, w.k), generator=g, device=device, dtype=torch.int32)
+    dt = _emb_dtype(w)
+    return {"j0": j0, "key": key.to(dt), "prefix": prefix.to(dt), "ids": ids, "cluster": cluster}
+
+
+def iter_store(w: Workload, device="cpu") -> Iterator[dict]:
+    cent = centres(w, device)
+    for index in range((w.n + CHUNK_ROWS - 1) // CHUNK_ROWS):
+        yield store_chunk(w, index, device, cent)
+
+
+def store_rows(w: Workload, rows: torch.Tensor, device="cpu") -> dict:
+    """Regenerate selected rows of the initial store (chunk by chunk)."""
+    rows = rows.to("cpu", torch.int64)
+    out_key = torch.empty((len(rows), w.d), dtype=_emb_dtype(w), device=device)
+    out_pre = torch.empty((len(rows), w.d), dtype=_emb_dtype(w), device=device)
+    out_ids = torch.empty((len(rows), w.k), dtype=torch.int32, device=device)
+    if len(rows) == 0:
+        return {"key": out_key, "prefix": out_pre, "ids": out_ids}
+    cent = centres(w, device)
+    chunk_of = rows // CHUNK_ROWS
+    for index in torch.unique(chunk_of).tolist():
+        sel = torch.nonzero(chunk_of == index).flatten()
+        ch = store_chunk(w, index, device, cent)
+        local = (rows[sel] - ch["j0"]).to(device)
+        sel_d = sel.to(device)
+        out_key[sel_d] = ch["key"][local]
+        out_pre[sel_d] = ch["prefix"][local]
+        out_ids[sel_d] = ch["ids"][local]
+    return {"key": out_key, "prefix": out_pre, "ids": out_ids}
+
+
+def class_counts(w: Workload) -> tuple:
+    near = int(round(w.batch * w.mix[0]))
+    coll = int(round(w.batch * w.mix[2]))
+    near = min(near, w.batch)
+    coll = min(coll, w.batch - near)
+    return near, w.batch - near - coll, coll
+
+
+def query_plan(w: Workload, step: int = 0, n_entries: int | None = None) -> dict:
+    """Class and target entry of every query of batch ``step`` (drawn on the CPU: small)."""
+    n_entries = w.n if n_entries is None else n_entries
+    g = _gen(w, "plan", step, "cpu")
+    near, rand, coll = class_counts(w)
+    classes = torch.tensor([NEAR] * near + [RANDOM] * rand + [COLLISION] * coll, dtype=torch.int64)
+    classes = classes[torch.randperm(w.batch, generator=g)]
+    if w.zipf is None:
+        target = torch.randint(0, max(n_entries, 1), (w.batch,), generator=g)
+    else:
+        # Zipf(s) over ranks 1..n, mapped to entries by a seeded affine permutation of [0, n)
+        ranks = torch.arange(1, n_entries + 1, dtype=torch.float64)
+        cdf = torch.cumsum(ranks.pow(-w.zipf), 0)
+        cdf /= cdf[-1].clone()
+        u = torch.rand((w.batch,), generator=g, dtype=torch.float64)
+        r = torch.searchsorted(cdf, u).clamp_(max=n_entries - 1)
+        a = int(torch.randint(1, 1 << 30, (1,), generator=g)) | 1
+        while math.gcd(a, n_entries) != 1:
+            a += 2
+        b = int(torch.randint(0, n_entries, (1,), generator=g))
+        target = (r * a + b) % n_entries
+    target = torch.where(classes == RANDOM, torch.full_like(target, -1), target)
+    return {"class": classes, "target": target}
+
+
+def make_queries(w: Workload, plan: dict, step: int = 0, device="cpu", target_rows: dict | None = None) -> dict:
+    """Query embeddings, prefix embeddings (bf16) and prefix ids (int32) for one batch."""
+    B = w.batch
+    cls = plan["class"].to(device)
+    tgt = plan["target"].clone()
+    if target_rows is None:
+        target_rows = store_rows(w, tgt.clamp(min=0), device)
+    g = _gen(w, "queries", step, device)
+    base = target_rows["key"].to(torch.float32)
+    noise = torch.randn((B, w.d), generator=g, device=device)
+    rnd = torch.randn((B, w.d), generator=g, device=device)
+    fresh_pre = _unit(torch.randn((B, w.d), generator=g, device=device)).to(torch.bfloat16)
+    fresh_ids = torch.randint(0, w.vocab, (B, w.k), generator=g, device=device, dtype=torch.int32)
+    scale = torch.where(cls == NEAR, w.near_sigma, w.coll_sigma).to(torch.float32)[:, None] / math.sqrt(w.d)
+    q = torch.where((cls == RANDOM)[:, None], rnd, base + noise * scale)
+    q = _unit(q).to(torch.bfloat16)
+    near = (cls == NEAR)[:, None]
+    pre = torch.where(near, target_rows["prefix"].to(torch.bfloat16), fresh_pre)
+    ids = torch.where(near, target_rows["ids"], fresh_ids)
+    return {"emb": q.contiguous(), "prefix": pre.contiguous(), "ids": ids.contiguous(),
+            "class": plan["class"].clone(), "target": plan["target"].clone()}
+
+
+def batch(w: Workload, step: int = 0, device="cpu", n_entries: int | None = None) -> dict:
+    plan = query_plan(w, step, n_entries)
+    return make_queries(w, plan, step, device)
+
+
+def bf16_bits(t: torch.Tensor):
+    """Host numpy view of a bf16 tensor's bit patterns (uint16): the exact bytes both sides read."""
+    return t.detach().to("cpu").contiguous().view(torch.int16).numpy().view("uint16")
+
+
+def f32_array(t: torch.Tensor):
+    return t.detach().to("cpu", torch.float32).contiguous().numpy()
