@@ -1,0 +1,356 @@
+#!/usr/bin/env python3
+"""Throughput of the LaCache two-stage lookahead lookup on GB300.
+
+    python bench.py [--gpus N --steps K --warmup W] [--workload mid-1m] [--stage1 auto|tensor|simt]
+    python bench.py --impl reference ...        # the fp64 oracle on the host cores, a bounded sample per step
+
+A step is one lookup: stage 1 (key check with fused threshold + top-c) and stage 2 (merge, lookahead check,
+decision) for one batch of B synthetic queries against a resident cache of N entries. The inputs are resident in
+HBM before timing starts. The key store is 1.6 GB for the default workload, larger than L2, so no L2 flush is
+needed between steps. The device time is taken with CUDA events on the launching stream, between barriers, as
+the max over ranks. With N > 1 GPUs (torchrun), every rank serves its own replica of the cache with its own
+query stream: the units are independent lookups, with no collective on the data path (weak scaling).
+
+Rank 0 prints one JSON line.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "lookups/sec at 1 GB300 (N entries, batch B, k) + % of HBM or bf16 roofline"
+UNIT = "queries/s"
+FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "simt": "stage1_simt.cu"}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="mid-1m")
+    ap.add_argument("--stage1", choices=["auto", "tensor", "simt"], default="auto")
+    ap.add_argument("--batches", type=int, default=8, help="distinct query batches cycled through")
+    ap.add_argument("--e2e-steps", type=int, default=500)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def rank_info():
+    return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
+            int(os.environ.get("WORLD_SIZE", 1)))
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            return json.load(f), "measured"
+    return dict(FALLBACK), "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clock and throttle reasons while the timed region runs."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        self.proc.wait()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(float(r[1]) for r in rows),
+                "sm_max_mhz": max(float(r[2]) for r in rows),
+                "power_w_max": max(float(r[3]) for r in rows if r[3].replace(".", "").isdigit()) if rows else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+def algorithmic(w, batch):
+    """Bytes and flops the method must move / do per lookup (keys read once, c candidate rows gathered)."""
+    stage1_bytes = w.n * w.d * 2 + batch * w.d * 2
+    stage2_bytes = batch * w.top_c * (2 * w.d + 4 * w.k) + batch * (2 * w.d + 4 * w.k)
+    flops = 2 * batch * w.n * w.d + 2 * batch * w.top_c * w.d
+    return stage1_bytes, stage2_bytes, flops
+
+
+def kernel_traffic(stage1: str, workload: str):
+    """DRAM bytes per launch of the stage-1 kernel from the committed ncu capture, if the kernel source has not
+    changed since the capture (else None)."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        rec = json.load(f).get(f"stage1_{stage1}/{workload}")
+    if not rec:
+        return None
+    src = os.path.join(ROOT, "paper_2608_01718_gb300", "csrc", STAGE1_SOURCES[stage1])
+    with open(src, "rb") as f:
+        if hashlib.sha256(f.read()).hexdigest() != rec.get("source_sha256"):
+            return None
+    return rec.get("dram_bytes_per_launch")
+
+
+def cpu_threads() -> int:
+    for var in ("OPENBLAS_NUM_THREADS", "OMP_NUM_THREADS"):
+        if os.environ.get(var, "").isdigit():
+            return int(os.environ[var])
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def oracle_sample(w, rows: int, offset: int = 0, device="cpu"):
+    """Host bytes of store rows [offset, offset + rows) (regenerated chunk by chunk) and of query batch 0."""
+    import numpy as np
+
+    import oracle
+    from paper_2608_01718_gb300 import workloads as wl
+    keys, pres, ids = [], [], []
+    got = 0
+    index = offset // wl.CHUNK_ROWS
+    start = offset - index * wl.CHUNK_ROWS
+    while got < rows:
+        ch = wl.store_chunk(w, index, device)
+        take = min(rows - got, ch["key"].shape[0] - start)
+        sl = slice(start, start + take)
+        if w.key_dtype == "f32":
+            keys.append(oracle.round_to_bf16(wl.f32_array(ch["key"][sl])))
+            pres.append(oracle.round_to_bf16(wl.f32_array(ch["prefix"][sl])))
+        else:
+            keys.append(wl.bf16_bits(ch["key"][sl]))
+            pres.append(wl.bf16_bits(ch["prefix"][sl]))
+        ids.append(ch["ids"][sl].cpu().numpy())
+        got += take
+        index += 1
+        start = 0
+    store = oracle.Store.of(np.concatenate(keys), np.concatenate(pres), np.concatenate(ids))
+    q = wl.batch(w, 0, device)
+    oq = {"emb": wl.bf16_bits(q["emb"]), "prefix": wl.bf16_bits(q["prefix"]), "ids": q["ids"].cpu().numpy()}
+    return store, oq
+
+
+def time_oracle(store, oq, w) -> float:
+    """Seconds the oracle takes to look up the whole batch against the given store rows."""
+    import oracle
+    p = oracle.Params(w.tau_c, w.tau_a, w.top_c)
+    t0 = time.perf_counter()
+    oracle.lookup(store, oq, p)
+    return time.perf_counter() - t0
+
+
+def gen_device():
+    import torch
+    return "cuda" if torch.cuda.is_available() else "cpu"
+
+
+def run_reference(args, w):
+    rank, _, world = rank_info()
+    if rank != 0:
+        return 0
+    dev = gen_device()
+    # size the per-step sample so that warm-up + timed steps take about two minutes in all
+    probe_rows = min(w.n, 16384)
+    store, oq = oracle_sample(w, probe_rows, 0, dev)
+    per_row = time_oracle(store, oq, w) / probe_rows
+    budget = 120.0 / max(1, args.steps + args.warmup)
+    rows = int(min(w.n, max(2048, budget / per_row)))
+    store, oq = oracle_sample(w, rows, 0, dev)
+    total = 0.0
+    for i in range(args.warmup + args.steps):
+        t = time_oracle(store, oq, w)
+        if i >= args.warmup:
+            total += t
+    sec_per_batch_full = total / args.steps * (w.n / rows)
+    value = w.batch / sec_per_batch_full
+    cores = cpu_threads()
+    sample = (f"each step: oracle lookup of the {w.batch}-query batch against the first {rows} of the {w.n} "
+              f"store rows; value scaled to the full store by N/rows (the oracle's work is linear in N)")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": workload_config(w) | {"parallelism": "single"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(w):
+    return {"workload": w.name, "entries": w.n, "d": w.d, "k": w.k, "batch": w.batch, "top_c": w.top_c,
+            "tau_c": w.tau_c, "tau_a": w.tau_a, "mix_near_random_collision": list(w.mix),
+            "store_bytes": w.store_bytes,
+            "l2": f"no flush: the keys read per step ({w.n * w.d * 2 / 1e9:.2f} GB) exceed the 129 MB L2"}
+
+
+def run_ours(args, w):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_01718_gb300 import build
+    from paper_2608_01718_gb300 import lacache as L
+    from paper_2608_01718_gb300 import workloads as wl
+
+    rank, local_rank, world = rank_info()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    build.build()
+    stage1 = {"auto": L.LACACHE_STAGE1_AUTO, "tensor": L.LACACHE_STAGE1_TENSOR, "simt": L.LACACHE_STAGE1_SIMT}
+    cache = L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch, device=local_rank,
+                      stage1=stage1[args.stage1])
+    dtype = L.LACACHE_F32 if w.key_dtype == "f32" else L.LACACHE_BF16
+    for ch in wl.iter_store(w, "cuda"):
+        cache.insert(ch["key"], ch["prefix"], ch["ids"], dtype)
+        del ch
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    nb = args.batches
+    batches = [wl.batch(w, step=(rank * nb + i), device="cuda") for i in range(nb)]
+    outs = [L.alloc_result(w.batch, w.top_c, "cuda", candidates=False) for _ in range(nb)]
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        q = batches[i % nb]
+        L.lacache_lookup(cache.h, q["emb"], q["prefix"], q["ids"], outs[i % nb], stream)
+
+    for i in range(max(3, args.warmup)):
+        step(i)
+    torch.cuda.synchronize()
+    cache.sync()
+    kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_SIMT: "simt"}[cache.last_launch()[1]]
+    L.lacache_stage_timing(cache.h, args.steps)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(torch.cuda.current_device())
+    clocks.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clock = clocks.stop()
+    cache.sync()
+    elapsed_ms = ev0.elapsed_time(ev1)
+    t1_ms, t2_ms, timed = L.lacache_stage_times(cache.h)
+    L.lacache_stage_timing(cache.h, 0)
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+
+    # end to end through the host-buffer entry point: H2D of the batch and D2H of the decisions every step
+    hq = [{k: batches[i][k].cpu().pin_memory() for k in ("emb", "prefix", "ids")} for i in range(nb)]
+    hout = [L.alloc_result(w.batch, w.top_c, "cpu", candidates=False, pinned=True) for _ in range(nb)]
+    for i in range(max(3, args.warmup)):
+        L.lacache_lookup_host(cache.h, hq[i % nb]["emb"], hq[i % nb]["prefix"], hq[i % nb]["ids"], hout[i % nb])
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for i in range(args.e2e_steps):
+        L.lacache_lookup_host(cache.h, hq[i % nb]["emb"], hq[i % nb]["prefix"], hq[i % nb]["ids"], hout[i % nb])
+    e2e_s = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([e2e_s], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+    h2d = w.batch * (2 * w.d * 2 + w.k * 4)
+    d2h = w.batch * (4 + 1 + 4 + 4 + 4 + 4)
+
+    peaks, peak_src = load_peaks()
+    s1_bytes, s2_bytes, flops = algorithmic(w, w.batch)
+    t1_avg_s = t1_ms / max(1, timed) / 1e3
+    achieved = s1_bytes / t1_avg_s / 1e9
+    traffic = kernel_traffic(kernel_name, w.name)
+    value = world * args.steps * w.batch / (elapsed_ms / 1e3)
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": workload_config(w) | {"parallelism": f"replicas{world}" if world > 1 else "single"},
+        "stage1_kernel": kernel_name,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / peaks["hbm_gbs"], "traffic": traffic, "kernel": f"stage1_{kernel_name}",
+                     "peak_source": f"{peak_src} (copy bandwidth)",
+                     "algorithmic_bytes_per_launch": s1_bytes, "avg_launch_ms": t1_avg_s * 1e3},
+        "tensor": {"achieved_tflops": flops / (elapsed_ms / args.steps / 1e3) / 1e12,
+                   "peak_tflops": peaks["bf16_tflops"],
+                   "frac": flops / (elapsed_ms / args.steps / 1e3) / 1e12 / peaks["bf16_tflops"]},
+        "stage_ms": {"stage1": t1_ms / max(1, timed), "stage2": t2_ms / max(1, timed), "timed_lookups": timed},
+        "e2e": {"value": world * args.e2e_steps * w.batch / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
+                "api": "lacache_lookup_host (pinned host buffers, synchronous)"},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clock,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rows = min(w.n, 1 << 20)
+        store, oq = oracle_sample(w, rows, 0, "cuda")
+        t = time_oracle(store, oq, w)
+        line["cpu_baseline"] = {
+            "value": w.batch / (t * w.n / rows), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
+            "sample": f"oracle lookup of the {w.batch}-query batch against the first {rows} of the {w.n} store rows "
+                      f"({t:.1f} s), scaled to the full store by N/rows (the oracle is linear in N)"}
+    cache.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main():
+    args = parse_args()
+    from paper_2608_01718_gb300 import workloads as wl
+    w = wl.WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, w)
+    return run_ours(args, w)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,170 @@
+/*
+ * lacache.h -- C ABI of the GB300 (sm_103a) LaCache lookup library, liblacache.so.
+ *
+ * LaCache ("LaCache: Robust Semantic Caching for LLM Serving") stores each cache entry as
+ * <h(x), [h(f_k(x)), f(x)]> (section 3.2, "Cache Structure"): the key embedding of query x, the embedding of the
+ * first k tokens of its response f_k(x), and the response. A query x is served from entry x' only if both checks
+ * pass (Algorithm 1; section 4.1, "Metrics"):
+ *     stage 1, key check:        sim(x, x')           >= tau_c
+ *     stage 2, lookahead check:  sim(f_k(x), f_k(x')) >= tau_a
+ * Otherwise x is decoded from scratch and its entry is appended to the cache (Algorithm 1, last two steps).
+ *
+ * This library is that lookup, batched, on one GPU. The response f(x) is the caller's: the library returns the
+ * entry id, which stands for it. sim is the inner product of unit-norm embeddings (their cosine).
+ *
+ * Conventions for every call
+ *  - Embeddings are bf16 (IEEE binary32 upper halves) in row-major [rows x d] layout. Token ids are int32 in
+ *    row-major [rows x k] layout. All rows are dense (row stride d or k elements).
+ *  - Pointers named *_dev are CUDA device pointers (cudaMalloc or equivalent) on the handle's device. Pointers
+ *    named *_host are host pointers (page-locked memory is fastest). The caller owns every input and output
+ *    buffer; the handle owns the device store and its scratch.
+ *  - Embedding pointers must be 16-byte aligned (TMA reads them).
+ *  - `cuda_stream` is a cudaStream_t (NULL = the legacy default stream). Device calls are asynchronous on it;
+ *    argument errors are reported synchronously and leave the cache unchanged.
+ *  - Device-side faults of the library's own kernels (a bounded wait that ran out) do not abort the process:
+ *    they set a status word that lacache_sync() reports as LACACHE_ERR_DEVICE_TIMEOUT.
+ *  - A handle is not thread-safe. Lookups see every insert issued before them on the same stream.
+ */
+#ifndef LACACHE_H_
+#define LACACHE_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct lacache lacache_t; /* opaque */
+
+typedef enum {
+  LACACHE_OK = 0,
+  LACACHE_ERR_INVALID_ARG = 1,    /* bad pointer, size, alignment or parameter */
+  LACACHE_ERR_CAPACITY = 2,       /* an insert would exceed the capacity; nothing was inserted */
+  LACACHE_ERR_OOM = 3,            /* device allocation failed at create */
+  LACACHE_ERR_CUDA = 4,           /* a CUDA runtime call failed */
+  LACACHE_ERR_DEVICE_TIMEOUT = 5, /* a kernel's bounded wait ran out (reported by lacache_sync) */
+  LACACHE_ERR_UNSUPPORTED = 6     /* valid but unsupported configuration (e.g. top_c > 32, d % 8 != 0) */
+} lacache_status;
+
+/* How stage 2 decides that candidate x' passes the lookahead check (Algorithm 1; section 4.1). */
+typedef enum {
+  LACACHE_CHECK_EMB = 0,    /* sim(f_k(x), f_k(x')) >= tau_a, the form the paper evaluates */
+  LACACHE_CHECK_TOKENS = 1, /* >= token_match_min of the k prefix token ids equal position by position;
+                               token_match_min = k is Algorithm 1's h(f_k(x')) = h(f_k(x)) on ids */
+  LACACHE_CHECK_BOTH = 2    /* both of the above */
+} lacache_check_mode;
+
+typedef enum { LACACHE_BF16 = 0, LACACHE_F32 = 1 } lacache_dtype;
+
+/* Which stage-1 kernel lookups run. AUTO picks by batch size. */
+typedef enum {
+  LACACHE_STAGE1_AUTO = 0,
+  LACACHE_STAGE1_TENSOR = 1, /* tcgen05 tensor-core scan (TMA-fed, TMEM accumulators) */
+  LACACHE_STAGE1_SIMT = 2    /* CUDA-core FFMA scan */
+} lacache_stage1;
+
+/* Per-query status codes written to lacache_result.status. */
+enum { LACACHE_MISS_KEY = 0, LACACHE_HIT = 1, LACACHE_REJECT = 2 };
+
+typedef struct {
+  int32_t d;               /* embedding dimension of keys and prefix embeddings; multiple of 8, <= 8192 */
+  int32_t k;               /* lookahead window: token ids per entry, 1..256 */
+  int64_t capacity;        /* maximum number of entries (device store is allocated once, at create) */
+  float tau_c;             /* key threshold */
+  float tau_a;             /* lookahead threshold */
+  int32_t top_c;           /* candidates kept from stage 1 per query, 1..32 */
+  int32_t token_match_min; /* LACACHE_CHECK_TOKENS/BOTH: positions that must match; <= 0 means k */
+  int32_t check_mode;      /* lacache_check_mode */
+  int32_t max_batch;       /* largest B passed to lookup; sizes the scratch and host-staging buffers */
+  int32_t device;          /* CUDA device ordinal */
+  int32_t stage1;          /* lacache_stage1 */
+} lacache_config;
+
+/* Per-query outputs of a lookup, each [B] (or [B x top_c] for the optional cand_* arrays). All device pointers
+ * for lacache_lookup, host pointers for lacache_lookup_host. The cand_* arrays may be NULL (not written). */
+typedef struct {
+  int32_t* entry_id;          /* served entry j* on HIT, else -1 */
+  uint8_t* status;            /* LACACHE_MISS_KEY / LACACHE_HIT / LACACHE_REJECT */
+  float* key_score;           /* sim(x, x') of j* on HIT; otherwise the best key score over all entries
+                                 (-inf for an empty cache) */
+  float* prefix_score;        /* sim(f_k(x), f_k(x')) of j* on HIT, of the first candidate on REJECT; NaN on
+                                 MISS_KEY */
+  int32_t* token_matches;     /* equal token ids (positionwise) for the same candidate as prefix_score; -1 on
+                                 MISS_KEY */
+  int32_t* n_cand;            /* number of candidates |C_q| <= top_c */
+  int32_t* cand_id;           /* optional [B x top_c]: C_q by (key score desc, id asc), -1 padded */
+  float* cand_score;          /* optional [B x top_c]: their key scores, NaN padded */
+  float* cand_prefix_score;   /* optional [B x top_c]: their lookahead scores, NaN padded */
+  int32_t* cand_matches;      /* optional [B x top_c]: their token matches, -1 padded */
+} lacache_result;
+
+/* Create a cache on cfg->device with an empty store of cfg->capacity entries. Allocates the store
+ * (capacity * (4d + 4k) bytes), the stage-1 scratch (about SMs * max_batch * top_c * 12 bytes) and host staging.
+ * On success *out is a new handle; on failure *out is NULL and nothing stays allocated. */
+lacache_status lacache_create(const lacache_config* cfg, lacache_t** out);
+
+/* Free the handle and everything it owns. Synchronizes the device first. NULL is accepted. */
+lacache_status lacache_destroy(lacache_t* h);
+
+/* Append n entries (Algorithm 1, "add <h(x), [h(f_k(x)), f(x)]> to cache"). key_dev and prefix_dev are
+ * [n x d] in `dtype` (LACACHE_F32 rows are rounded to bf16, to nearest even, on the device); ids_dev is
+ * [n x k] int32. All-or-nothing: if size + n > capacity, returns LACACHE_ERR_CAPACITY and inserts nothing. The new
+ * entries get ids first_id .. first_id + n - 1 (first_id may be NULL). Asynchronous on cuda_stream. */
+lacache_status lacache_insert(lacache_t* h, int64_t n, const void* key_dev, const void* prefix_dev,
+                              const int32_t* ids_dev, int32_t dtype, int64_t* first_id, void* cuda_stream);
+
+/* Batched two-stage lookup of B queries (1 <= B <= max_batch): q_emb_dev [B x d] bf16 key embeddings of the
+ * queries, q_prefix_dev [B x d] bf16 embeddings of their speculatively decoded k-token prefixes f_k(x),
+ * q_ids_dev [B x k] int32 those token ids. Stage 1 keeps per query the top_c entries with key score >= tau_c by
+ * (score desc, id asc); stage 2 checks them in that order and serves the first that passes. Writes every
+ * non-NULL field of *out (device pointers). Asynchronous on cuda_stream; no host synchronization. */
+lacache_status lacache_lookup(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
+                              const int32_t* q_ids_dev, const lacache_result* out, void* cuda_stream);
+
+/* lacache_lookup for host-resident queries and results: copies the inputs into the handle's device staging,
+ * runs the same kernels, copies the results back into *out_host (host pointers) and synchronizes cuda_stream
+ * before returning. */
+lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_host, const void* q_prefix_host,
+                                   const int32_t* q_ids_host, const lacache_result* out_host, void* cuda_stream);
+
+/* The cache update of the serve loop: append, in query order, every query of a looked-up batch whose status is
+ * not LACACHE_HIT (a key miss or a lookahead rejection is decoded from scratch and added; Algorithm 1). The
+ * inputs are those of the lookup (device pointers) and its status_dev output. The rows are gathered on the
+ * device; the count is read back, so this call synchronizes cuda_stream. All-or-nothing on capacity. Writes the
+ * first new id and the number appended (either pointer may be NULL). */
+lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
+                                     const int32_t* q_ids_dev, const uint8_t* status_dev, int64_t* first_id,
+                                     int64_t* n_appended, void* cuda_stream);
+
+/* Copy entries [first, first + n) of the store into caller device buffers (key_dev/prefix_dev [n x d] bf16,
+ * ids_dev [n x k]); any of the three may be NULL. For checkpoints and checks. Asynchronous on cuda_stream. */
+lacache_status lacache_read_rows(const lacache_t* h, int64_t first, int64_t n, void* key_dev, void* prefix_dev,
+                                 int32_t* ids_dev, void* cuda_stream);
+
+/* Number of valid entries (as of the calls issued so far). */
+lacache_status lacache_size(const lacache_t* h, int64_t* n);
+
+/* Synchronize the handle's device and report any device-side status set by the library's kernels since the
+ * previous lacache_sync (the status word is then cleared). */
+lacache_status lacache_sync(lacache_t* h);
+
+/* Number of stage-1 partial lists the last lookup used, and which stage-1 kernel it ran (lacache_stage1). */
+lacache_status lacache_last_launch(const lacache_t* h, int32_t* n_splits, int32_t* stage1_kernel);
+
+/* Stage timing (measurement). lacache_stage_timing(h, m) with m > 0 makes the next m lookups record CUDA events
+ * around their stage-1 and stage-2 kernels on the lookup's own stream (three cudaEventRecord calls per lookup;
+ * the events are created here, not in the lookups). m = 0 turns it off and frees the events.
+ * lacache_stage_times synchronizes on the last recorded event and returns, over the lookups timed since the
+ * previous call, the summed device time of stage 1 (the key-check kernel) and of stage 2 (merge, lookahead
+ * check and decision), and how many lookups were timed; it then restarts the count. */
+lacache_status lacache_stage_timing(lacache_t* h, int32_t max_lookups);
+lacache_status lacache_stage_times(lacache_t* h, double* stage1_ms, double* stage2_ms, int64_t* lookups);
+
+/* Static description of a status code. */
+const char* lacache_status_string(lacache_status s);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LACACHE_H_ */

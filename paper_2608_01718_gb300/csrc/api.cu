@@ -1,0 +1,531 @@
+// C-ABI entry points of liblacache.so (declared in include/lacache.h): the device store, insert and the cache
+// update of the serve loop, and the dispatch of a lookup to the stage-1 and stage-2 kernels.
+#include <cuda.h>
+#include <math.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include <new>
+
+#include "internal.cuh"
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+struct lacache {
+  lacache_config cfg;
+  int num_sms;
+  int max_splits;
+  int64_t n;                 // valid entries, as of the calls issued so far
+  __nv_bfloat16* key;        // [capacity x d]
+  __nv_bfloat16* prefix;     // [capacity x d]
+  int32_t* ids;              // [capacity x k]
+  uint64_t* part_cand;       // [max_splits x max_batch x top_c]
+  float* part_best;          // [max_splits x max_batch]
+  unsigned int* dev_status;  // device status word
+  int32_t* append_dst;       // [max_batch] destination rank of each appended query
+  int32_t* append_count;     // device count of appended rows
+  int32_t* append_count_host;  // pinned
+  unsigned char* stage_in;   // device staging for lookup_host inputs
+  unsigned char* stage_out;  // device staging for lookup_host results
+  int last_splits;
+  int last_kernel;
+  EncodeTiledFn encode;
+  cudaEvent_t* events;       // [3 x event_cap] stage-timing events, or NULL
+  int event_cap;
+  int event_used;
+};
+
+namespace {
+
+using lc::Stage1Args;
+using lc::Stage2Args;
+
+class DeviceGuard {
+ public:
+  explicit DeviceGuard(int dev) {
+    ok_ = cudaGetDevice(&prev_) == cudaSuccess;
+    if (ok_ && prev_ != dev) ok_ = cudaSetDevice(dev) == cudaSuccess;
+    dev_ = dev;
+  }
+  ~DeviceGuard() {
+    if (ok_ && prev_ != dev_) cudaSetDevice(prev_);
+  }
+  bool ok() const { return ok_; }
+
+ private:
+  int prev_ = 0, dev_ = 0;
+  bool ok_ = false;
+};
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+lacache_status from_cuda(cudaError_t e) { return e == cudaSuccess ? LACACHE_OK : LACACHE_ERR_CUDA; }
+
+// f32 -> bf16 (round to nearest even) of n*d elements of two arrays, into the store.
+__global__ void convert_rows_kernel(const float* __restrict__ a, const float* __restrict__ b,
+                                    __nv_bfloat16* __restrict__ da, __nv_bfloat16* __restrict__ db, int64_t count) {
+  for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < count; i += (int64_t)gridDim.x * blockDim.x) {
+    da[i] = __float2bfloat16_rn(a[i]);
+    db[i] = __float2bfloat16_rn(b[i]);
+  }
+}
+
+// Rank of every non-HIT query among the non-HIT queries of the batch (query order), and their count.
+__global__ void append_rank_kernel(const uint8_t* __restrict__ status, int B, int32_t* __restrict__ dst,
+                                   int32_t* __restrict__ count) {
+  __shared__ int warp_tot[32];
+  __shared__ int carry;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  for (int base = 0; base < B; base += blockDim.x) {
+    const int q = base + threadIdx.x;
+    const int flag = (q < B && status[q] != LACACHE_HIT) ? 1 : 0;
+    const unsigned ballot = __ballot_sync(0xffffffffu, flag);
+    const int in_warp = __popc(ballot & ((1u << lane) - 1u));
+    if (lane == 0) warp_tot[warp] = __popc(ballot);
+    __syncthreads();
+    int before = carry;
+    for (int w = 0; w < warp; ++w) before += warp_tot[w];
+    if (q < B) dst[q] = flag ? before + in_warp : -1;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int t = 0;
+      for (int w = 0; w < nw; ++w) t += warp_tot[w];
+      carry += t;
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0) *count = carry;
+}
+
+// Copy the rows of the ranked queries into the store at n0 + rank, unless the batch would overflow capacity.
+__global__ void append_rows_kernel(const uint4* __restrict__ q_emb, const uint4* __restrict__ q_pre,
+                                   const int32_t* __restrict__ q_ids, const int32_t* __restrict__ dst,
+                                   const int32_t* __restrict__ count, int B, int d, int k, int64_t n0,
+                                   int64_t capacity, uint4* __restrict__ key, uint4* __restrict__ pre,
+                                   int32_t* __restrict__ ids) {
+  if (n0 + *count > capacity) return;
+  const int v_per_row = d / 8;
+  const int q = blockIdx.x;
+  if (q >= B) return;
+  const int r = dst[q];
+  if (r < 0) return;
+  const int64_t row = n0 + r;
+  for (int i = threadIdx.x; i < v_per_row; i += blockDim.x) {
+    key[row * v_per_row + i] = q_emb[(int64_t)q * v_per_row + i];
+    pre[row * v_per_row + i] = q_pre[(int64_t)q * v_per_row + i];
+  }
+  for (int i = threadIdx.x; i < k; i += blockDim.x) ids[row * k + i] = q_ids[(int64_t)q * k + i];
+}
+
+size_t stage_in_bytes(const lacache_config& c) {
+  return (size_t)c.max_batch * ((size_t)4 * c.d + (size_t)4 * c.k);
+}
+size_t stage_out_bytes(const lacache_config& c) {
+  // five [B] 4-byte arrays, four [B x top_c] 4-byte arrays, one [B] byte array, each rounded up to 16 bytes
+  return (size_t)c.max_batch * (21 + (size_t)c.top_c * 16) + 10 * 16;
+}
+
+// Device staging layout of the results of lookup_host (each array 16-byte aligned).
+lacache_result staged_result(lacache* h, int B) {
+  unsigned char* p = h->stage_out;
+  const size_t mb = (size_t)h->cfg.max_batch, tc = (size_t)h->cfg.top_c;
+  auto take = [&](size_t bytes) {
+    unsigned char* r = p;
+    p += (bytes + 15) & ~(size_t)15;
+    return r;
+  };
+  (void)B;
+  lacache_result r;
+  r.entry_id = (int32_t*)take(mb * 4);
+  r.key_score = (float*)take(mb * 4);
+  r.prefix_score = (float*)take(mb * 4);
+  r.token_matches = (int32_t*)take(mb * 4);
+  r.n_cand = (int32_t*)take(mb * 4);
+  r.cand_id = (int32_t*)take(mb * tc * 4);
+  r.cand_score = (float*)take(mb * tc * 4);
+  r.cand_prefix_score = (float*)take(mb * tc * 4);
+  r.cand_matches = (int32_t*)take(mb * tc * 4);
+  r.status = (uint8_t*)take(mb);
+  return r;
+}
+
+void free_events(lacache* h) {
+  if (!h->events) return;
+  for (int i = 0; i < 3 * h->event_cap; ++i)
+    if (h->events[i]) cudaEventDestroy(h->events[i]);
+  free(h->events);
+  h->events = nullptr;
+  h->event_cap = h->event_used = 0;
+}
+
+void free_all(lacache* h) {
+  free_events(h);
+  cudaFree(h->key);
+  cudaFree(h->prefix);
+  cudaFree(h->ids);
+  cudaFree(h->part_cand);
+  cudaFree(h->part_best);
+  cudaFree(h->dev_status);
+  cudaFree(h->append_dst);
+  cudaFree(h->append_count);
+  cudaFree(h->stage_in);
+  cudaFree(h->stage_out);
+  if (h->append_count_host) cudaFreeHost(h->append_count_host);
+}
+
+bool encode_2d(lacache* h, CUtensorMap* m, const void* base, int64_t inner, int64_t outer, uint32_t box_inner,
+               uint32_t box_outer) {
+  const cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)outer};
+  const cuuint64_t strides[1] = {(cuuint64_t)inner * 2};
+  const cuuint32_t box[2] = {box_inner, box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  return h->encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* q_prefix, const int32_t* q_ids,
+                          const lacache_result& out, cudaStream_t st) {
+  const lacache_config& c = h->cfg;
+  int splits = 0;
+  int kernel = 0;
+  cudaEvent_t* ev = nullptr;
+  if (h->events && h->event_used < h->event_cap) ev = h->events + 3 * h->event_used++;
+  if (ev && cudaEventRecord(ev[0], st) != cudaSuccess) return LACACHE_ERR_CUDA;
+  if (h->n > 0) {
+    Stage1Args a;
+    a.keys = h->key;
+    a.n = h->n;
+    a.d = c.d;
+    a.q = reinterpret_cast<const __nv_bfloat16*>(q_emb);
+    a.B = B;
+    a.tau_c = c.tau_c;
+    a.top_c = c.top_c;
+    a.part_cand = h->part_cand;
+    a.part_best = h->part_best;
+    a.dev_status = h->dev_status;
+    kernel = c.stage1 == LACACHE_STAGE1_AUTO ? LACACHE_STAGE1_TENSOR : c.stage1;
+    cudaError_t e;
+    if (kernel == LACACHE_STAGE1_TENSOR) {
+      if (!h->encode) return LACACHE_ERR_CUDA;
+      CUtensorMap tq, tk;
+      if (!encode_2d(h, &tq, q_emb, c.d, B, 64, 128) || !encode_2d(h, &tk, h->key, c.d, h->n, 64, 256))
+        return LACACHE_ERR_CUDA;
+      e = lc::launch_stage1_tensor(a, &tq, &tk, h->num_sms, h->max_splits, st, &splits);
+    } else {
+      e = lc::launch_stage1_simt(a, h->num_sms, h->max_splits, st, &splits);
+    }
+    if (e != cudaSuccess) return LACACHE_ERR_CUDA;
+  }
+  Stage2Args b;
+  b.n = h->n;
+  b.part_cand = h->part_cand;
+  b.part_best = h->part_best;
+  b.splits = splits;
+  b.B = B;
+  b.d = c.d;
+  b.k = c.k;
+  b.top_c = c.top_c;
+  b.tau_a = c.tau_a;
+  b.check_mode = c.check_mode;
+  b.token_match_min = c.token_match_min;
+  b.prefix = h->prefix;
+  b.ids = h->ids;
+  b.q_prefix = reinterpret_cast<const __nv_bfloat16*>(q_prefix);
+  b.q_ids = q_ids;
+  b.out = out;
+  if (ev && cudaEventRecord(ev[1], st) != cudaSuccess) return LACACHE_ERR_CUDA;
+  if (lc::launch_stage2(b, st) != cudaSuccess) return LACACHE_ERR_CUDA;
+  if (ev && cudaEventRecord(ev[2], st) != cudaSuccess) return LACACHE_ERR_CUDA;
+  h->last_splits = splits;
+  h->last_kernel = kernel;
+  return LACACHE_OK;
+}
+
+bool result_ok(const lacache_result* r) {
+  return r && r->entry_id && r->status && r->key_score && r->prefix_score && r->token_matches && r->n_cand;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* lacache_status_string(lacache_status s) {
+  switch (s) {
+    case LACACHE_OK: return "ok";
+    case LACACHE_ERR_INVALID_ARG: return "invalid argument";
+    case LACACHE_ERR_CAPACITY: return "capacity exceeded";
+    case LACACHE_ERR_OOM: return "device out of memory";
+    case LACACHE_ERR_CUDA: return "CUDA error";
+    case LACACHE_ERR_DEVICE_TIMEOUT: return "device wait timed out";
+    case LACACHE_ERR_UNSUPPORTED: return "unsupported configuration";
+  }
+  return "unknown status";
+}
+
+lacache_status lacache_create(const lacache_config* cfg, lacache_t** out) {
+  if (!out) return LACACHE_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg) return LACACHE_ERR_INVALID_ARG;
+  const lacache_config c = *cfg;
+  if (c.d <= 0 || c.k <= 0 || c.capacity <= 0 || c.top_c <= 0 || c.max_batch <= 0) return LACACHE_ERR_INVALID_ARG;
+  if (isnan(c.tau_c) || isnan(c.tau_a)) return LACACHE_ERR_INVALID_ARG;
+  if (c.check_mode < LACACHE_CHECK_EMB || c.check_mode > LACACHE_CHECK_BOTH) return LACACHE_ERR_INVALID_ARG;
+  if (c.stage1 < LACACHE_STAGE1_AUTO || c.stage1 > LACACHE_STAGE1_SIMT) return LACACHE_ERR_INVALID_ARG;
+  if (c.token_match_min > c.k) return LACACHE_ERR_INVALID_ARG;
+  if (c.d % 8 != 0 || c.d > lc::kMaxD || c.k > lc::kMaxK || c.top_c > lc::kMaxTopC) return LACACHE_ERR_UNSUPPORTED;
+  if (c.capacity > (int64_t)INT32_MAX || c.max_batch > (1 << 20)) return LACACHE_ERR_UNSUPPORTED;
+  int ndev = 0;
+  if (cudaGetDeviceCount(&ndev) != cudaSuccess) return LACACHE_ERR_CUDA;
+  if (c.device < 0 || c.device >= ndev) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(c.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+
+  lacache* h = new (std::nothrow) lacache;
+  if (!h) return LACACHE_ERR_OOM;
+  memset(h, 0, sizeof(*h));
+  h->cfg = c;
+  if (cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, c.device) != cudaSuccess) {
+    delete h;
+    return LACACHE_ERR_CUDA;
+  }
+  h->max_splits = lc::max_splits_for(h->num_sms);
+  const size_t cap = (size_t)c.capacity;
+  bool ok = cudaMalloc(&h->key, cap * c.d * 2) == cudaSuccess &&
+            cudaMalloc(&h->prefix, cap * c.d * 2) == cudaSuccess &&
+            cudaMalloc(&h->ids, cap * c.k * 4) == cudaSuccess &&
+            cudaMalloc(&h->part_cand, (size_t)h->max_splits * c.max_batch * c.top_c * 8) == cudaSuccess &&
+            cudaMalloc(&h->part_best, (size_t)h->max_splits * c.max_batch * 4) == cudaSuccess &&
+            cudaMalloc(&h->dev_status, 4) == cudaSuccess &&
+            cudaMalloc(&h->append_dst, (size_t)c.max_batch * 4) == cudaSuccess &&
+            cudaMalloc(&h->append_count, 4) == cudaSuccess &&
+            cudaMalloc(&h->stage_in, stage_in_bytes(c)) == cudaSuccess &&
+            cudaMalloc(&h->stage_out, stage_out_bytes(c)) == cudaSuccess &&
+            cudaMallocHost(&h->append_count_host, 4) == cudaSuccess &&
+            cudaMemset(h->dev_status, 0, 4) == cudaSuccess &&
+            cudaMemset(h->part_cand, 0, (size_t)h->max_splits * c.max_batch * c.top_c * 8) == cudaSuccess &&
+            cudaDeviceSynchronize() == cudaSuccess;
+  if (!ok) {
+    cudaGetLastError();
+    free_all(h);
+    delete h;
+    return LACACHE_ERR_OOM;
+  }
+  void* fn = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+          cudaSuccess &&
+      q == cudaDriverEntryPointSuccess)
+    h->encode = reinterpret_cast<EncodeTiledFn>(fn);
+  *out = h;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_destroy(lacache_t* h) {
+  if (!h) return LACACHE_OK;
+  DeviceGuard guard(h->cfg.device);
+  cudaDeviceSynchronize();
+  free_all(h);
+  delete h;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_insert(lacache_t* h, int64_t n, const void* key_dev, const void* prefix_dev,
+                              const int32_t* ids_dev, int32_t dtype, int64_t* first_id, void* cuda_stream) {
+  if (!h || n < 0) return LACACHE_ERR_INVALID_ARG;
+  if (dtype != LACACHE_BF16 && dtype != LACACHE_F32) return LACACHE_ERR_INVALID_ARG;
+  if (n > 0 && (!key_dev || !prefix_dev || !ids_dev)) return LACACHE_ERR_INVALID_ARG;
+  if (n > h->cfg.capacity - h->n) return LACACHE_ERR_CAPACITY;
+  if (first_id) *first_id = h->n;
+  if (n == 0) return LACACHE_OK;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const int d = h->cfg.d, k = h->cfg.k;
+  __nv_bfloat16* kd = h->key + h->n * d;
+  __nv_bfloat16* pd = h->prefix + h->n * d;
+  cudaError_t e;
+  if (dtype == LACACHE_BF16) {
+    e = cudaMemcpyAsync(kd, key_dev, (size_t)n * d * 2, cudaMemcpyDeviceToDevice, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(pd, prefix_dev, (size_t)n * d * 2, cudaMemcpyDeviceToDevice, st);
+  } else {
+    const int64_t count = n * d;
+    const int threads = 256;
+    const int64_t want = (count + threads - 1) / threads;
+    const int blocks = (int)(want < (int64_t)h->num_sms * 32 ? want : (int64_t)h->num_sms * 32);
+    convert_rows_kernel<<<blocks, threads, 0, st>>>((const float*)key_dev, (const float*)prefix_dev, kd, pd, count);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(h->ids + h->n * k, ids_dev, (size_t)n * k * 4, cudaMemcpyDeviceToDevice, st);
+  if (e != cudaSuccess) return LACACHE_ERR_CUDA;
+  h->n += n;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_lookup(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
+                              const int32_t* q_ids_dev, const lacache_result* out, void* cuda_stream) {
+  if (!h || B < 1 || B > h->cfg.max_batch) return LACACHE_ERR_INVALID_ARG;
+  if (!q_emb_dev || !q_prefix_dev || !q_ids_dev || !result_ok(out)) return LACACHE_ERR_INVALID_ARG;
+  if (!aligned16(q_emb_dev) || !aligned16(q_prefix_dev)) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  return run_lookup(h, B, q_emb_dev, q_prefix_dev, q_ids_dev, *out, (cudaStream_t)cuda_stream);
+}
+
+lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_host, const void* q_prefix_host,
+                                   const int32_t* q_ids_host, const lacache_result* out_host, void* cuda_stream) {
+  if (!h || B < 1 || B > h->cfg.max_batch) return LACACHE_ERR_INVALID_ARG;
+  if (!q_emb_host || !q_prefix_host || !q_ids_host || !result_ok(out_host)) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const lacache_config& c = h->cfg;
+  const size_t emb = (size_t)B * c.d * 2;
+  unsigned char* q_emb = h->stage_in;
+  unsigned char* q_pre = q_emb + (size_t)c.max_batch * c.d * 2;
+  int32_t* q_ids = reinterpret_cast<int32_t*>(q_pre + (size_t)c.max_batch * c.d * 2);
+  cudaError_t e = cudaMemcpyAsync(q_emb, q_emb_host, emb, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(q_pre, q_prefix_host, emb, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(q_ids, q_ids_host, (size_t)B * c.k * 4, cudaMemcpyHostToDevice, st);
+  if (e != cudaSuccess) return LACACHE_ERR_CUDA;
+  lacache_result dev = staged_result(h, B);
+  if (!out_host->cand_id) dev.cand_id = nullptr;
+  if (!out_host->cand_score) dev.cand_score = nullptr;
+  if (!out_host->cand_prefix_score) dev.cand_prefix_score = nullptr;
+  if (!out_host->cand_matches) dev.cand_matches = nullptr;
+  lacache_status s = run_lookup(h, B, q_emb, q_pre, q_ids, dev, st);
+  if (s != LACACHE_OK) return s;
+  const size_t b4 = (size_t)B * 4, bc4 = (size_t)B * c.top_c * 4;
+  struct Copy {
+    void* dst;
+    const void* src;
+    size_t bytes;
+  } copies[] = {
+      {out_host->entry_id, dev.entry_id, b4},         {out_host->status, dev.status, (size_t)B},
+      {out_host->key_score, dev.key_score, b4},       {out_host->prefix_score, dev.prefix_score, b4},
+      {out_host->token_matches, dev.token_matches, b4}, {out_host->n_cand, dev.n_cand, b4},
+      {out_host->cand_id, dev.cand_id, bc4},          {out_host->cand_score, dev.cand_score, bc4},
+      {out_host->cand_prefix_score, dev.cand_prefix_score, bc4}, {out_host->cand_matches, dev.cand_matches, bc4},
+  };
+  for (const Copy& cp : copies) {
+    if (!cp.dst) continue;
+    if (cudaMemcpyAsync(cp.dst, cp.src, cp.bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess) return LACACHE_ERR_CUDA;
+  }
+  return from_cuda(cudaStreamSynchronize(st));
+}
+
+lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
+                                     const int32_t* q_ids_dev, const uint8_t* status_dev, int64_t* first_id,
+                                     int64_t* n_appended, void* cuda_stream) {
+  if (!h || B < 1 || B > h->cfg.max_batch) return LACACHE_ERR_INVALID_ARG;
+  if (!q_emb_dev || !q_prefix_dev || !q_ids_dev || !status_dev) return LACACHE_ERR_INVALID_ARG;
+  if (!aligned16(q_emb_dev) || !aligned16(q_prefix_dev)) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const lacache_config& c = h->cfg;
+  append_rank_kernel<<<1, 1024, 0, st>>>(status_dev, B, h->append_dst, h->append_count);
+  append_rows_kernel<<<B, 128, 0, st>>>((const uint4*)q_emb_dev, (const uint4*)q_prefix_dev, q_ids_dev,
+                                        h->append_dst, h->append_count, B, c.d, c.k, h->n, c.capacity,
+                                        (uint4*)h->key, (uint4*)h->prefix, h->ids);
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(h->append_count_host, h->append_count, 4, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+  if (e != cudaSuccess) return LACACHE_ERR_CUDA;
+  const int64_t m = *h->append_count_host;
+  if (h->n + m > c.capacity) return LACACHE_ERR_CAPACITY;
+  if (first_id) *first_id = h->n;
+  if (n_appended) *n_appended = m;
+  h->n += m;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_read_rows(const lacache_t* h, int64_t first, int64_t n, void* key_dev, void* prefix_dev,
+                                 int32_t* ids_dev, void* cuda_stream) {
+  if (!h || first < 0 || n < 0 || first + n > h->n) return LACACHE_ERR_INVALID_ARG;
+  if (n == 0) return LACACHE_OK;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const int d = h->cfg.d, k = h->cfg.k;
+  cudaError_t e = cudaSuccess;
+  if (key_dev) e = cudaMemcpyAsync(key_dev, h->key + first * d, (size_t)n * d * 2, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess && prefix_dev)
+    e = cudaMemcpyAsync(prefix_dev, h->prefix + first * d, (size_t)n * d * 2, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess && ids_dev)
+    e = cudaMemcpyAsync(ids_dev, h->ids + first * k, (size_t)n * k * 4, cudaMemcpyDeviceToDevice, st);
+  return from_cuda(e);
+}
+
+lacache_status lacache_size(const lacache_t* h, int64_t* n) {
+  if (!h || !n) return LACACHE_ERR_INVALID_ARG;
+  *n = h->n;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_sync(lacache_t* h) {
+  if (!h) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  if (cudaDeviceSynchronize() != cudaSuccess) return LACACHE_ERR_CUDA;
+  unsigned int word = 0;
+  if (cudaMemcpy(&word, h->dev_status, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return LACACHE_ERR_CUDA;
+  if (word && cudaMemset(h->dev_status, 0, 4) != cudaSuccess) return LACACHE_ERR_CUDA;
+  return (word & lc::kDevTimeout) ? LACACHE_ERR_DEVICE_TIMEOUT : LACACHE_OK;
+}
+
+lacache_status lacache_stage_timing(lacache_t* h, int32_t max_lookups) {
+  if (!h || max_lookups < 0) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  if (h->events) cudaDeviceSynchronize();
+  free_events(h);
+  if (max_lookups == 0) return LACACHE_OK;
+  h->events = static_cast<cudaEvent_t*>(calloc((size_t)3 * max_lookups, sizeof(cudaEvent_t)));
+  if (!h->events) return LACACHE_ERR_OOM;
+  h->event_cap = max_lookups;
+  for (int i = 0; i < 3 * max_lookups; ++i) {
+    if (cudaEventCreate(&h->events[i]) != cudaSuccess) {
+      free_events(h);
+      return LACACHE_ERR_CUDA;
+    }
+  }
+  return LACACHE_OK;
+}
+
+lacache_status lacache_stage_times(lacache_t* h, double* stage1_ms, double* stage2_ms, int64_t* lookups) {
+  if (!h) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  double t1 = 0, t2 = 0;
+  const int used = h->events ? h->event_used : 0;
+  if (used && cudaEventSynchronize(h->events[3 * used - 1]) != cudaSuccess) return LACACHE_ERR_CUDA;
+  for (int i = 0; i < used; ++i) {
+    float a = 0, b = 0;
+    if (cudaEventElapsedTime(&a, h->events[3 * i], h->events[3 * i + 1]) != cudaSuccess ||
+        cudaEventElapsedTime(&b, h->events[3 * i + 1], h->events[3 * i + 2]) != cudaSuccess)
+      return LACACHE_ERR_CUDA;
+    t1 += a;
+    t2 += b;
+  }
+  if (h->events) h->event_used = 0;
+  if (stage1_ms) *stage1_ms = t1;
+  if (stage2_ms) *stage2_ms = t2;
+  if (lookups) *lookups = used;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_last_launch(const lacache_t* h, int32_t* n_splits, int32_t* stage1_kernel) {
+  if (!h) return LACACHE_ERR_INVALID_ARG;
+  if (n_splits) *n_splits = h->last_splits;
+  if (stage1_kernel) *stage1_kernel = h->last_kernel;
+  return LACACHE_OK;
+}
+
+}  // extern "C"

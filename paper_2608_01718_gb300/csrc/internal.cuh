@@ -1,0 +1,95 @@
+// Internal declarations shared by the lookup kernels and the C-ABI host code of liblacache.so.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <string.h>
+
+#include "lacache.h"
+
+namespace lc {
+
+constexpr int kMaxTopC = 32;
+constexpr int kMaxD = 8192;
+constexpr int kMaxK = 256;
+
+// Bits of the device status word.
+constexpr unsigned int kDevTimeout = 1u;
+
+// ---------------------------------------------------------------------------------------------------------------
+// Candidate keys. A stage-1 candidate (score s, entry id j) is packed into one uint64 whose unsigned order is the
+// candidate order of the lookup: higher score first, then lower entry id. The high word is the score's bits mapped
+// to an unsigned order; the low word is ~j. The value 0 is never produced by a finite score and marks "empty".
+// ---------------------------------------------------------------------------------------------------------------
+__host__ __device__ __forceinline__ uint32_t score_order(float s) {
+  uint32_t u;
+#ifdef __CUDA_ARCH__
+  u = __float_as_uint(s);
+#else
+  memcpy(&u, &s, 4);
+#endif
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+
+__host__ __device__ __forceinline__ float score_of_order(uint32_t o) {
+  uint32_t u = (o & 0x80000000u) ? (o & 0x7FFFFFFFu) : ~o;
+  float s;
+#ifdef __CUDA_ARCH__
+  s = __uint_as_float(u);
+#else
+  memcpy(&s, &u, 4);
+#endif
+  return s;
+}
+
+__host__ __device__ __forceinline__ uint64_t pack_cand(float s, uint32_t j) {
+  return ((uint64_t)score_order(s) << 32) | (uint64_t)(~j);
+}
+__host__ __device__ __forceinline__ float cand_score(uint64_t c) { return score_of_order((uint32_t)(c >> 32)); }
+__host__ __device__ __forceinline__ uint32_t cand_id(uint64_t c) { return ~(uint32_t)c; }
+
+// Stage-1 output: per split s and query q, the split's top_c candidates (sorted, 0-padded) and its best score.
+//   part_cand[(s * B + q) * top_c + i], part_best[s * B + q]
+struct Stage1Args {
+  const __nv_bfloat16* keys;  // [n x d] store keys
+  int64_t n;
+  int d;
+  const __nv_bfloat16* q;     // [B x d] query embeddings
+  int B;
+  float tau_c;
+  int top_c;
+  uint64_t* part_cand;
+  float* part_best;
+  unsigned int* dev_status;
+};
+
+struct Stage2Args {
+  int64_t n;                     // valid entries: candidate ids at or past n are dropped
+  const uint64_t* part_cand;
+  const float* part_best;
+  int splits;
+  int B;
+  int d;
+  int k;
+  int top_c;
+  float tau_a;
+  int check_mode;
+  int token_match_min;
+  const __nv_bfloat16* prefix;   // [n x d] store prefix embeddings
+  const int32_t* ids;            // [n x k] store prefix token ids
+  const __nv_bfloat16* q_prefix; // [B x d]
+  const int32_t* q_ids;          // [B x k]
+  lacache_result out;            // device pointers
+};
+
+// Launchers (host). Each returns the CUDA error of the launch. `splits` is the number of partial lists written.
+cudaError_t launch_stage1_simt(const Stage1Args& a, int num_sms, int max_splits, cudaStream_t st, int* splits);
+cudaError_t launch_stage1_tensor(const Stage1Args& a, const void* tmap_q, const void* tmap_k, int num_sms,
+                                 int max_splits, cudaStream_t st, int* splits);
+cudaError_t launch_stage2(const Stage2Args& a, cudaStream_t st);
+
+// Largest split count any stage-1 launcher uses for a given SM count (sizes the scratch).
+inline int max_splits_for(int num_sms) { return num_sms; }
+
+}  // namespace lc

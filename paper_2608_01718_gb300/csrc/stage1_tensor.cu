@@ -1,0 +1,466 @@
+// Stage 1 on the tensor cores: the key check sim(x, x') >= tau_c (Algorithm 1's cache search; section 4.1) as a
+// tcgen05 GEMM of the query tile against the key store, fused with the threshold and a per-query running
+// top_c. The B x N score matrix never leaves the SM.
+//
+//   D[m][n] = sum_k Q[qt*128 + m][k] * K[t*256 + n][k]      (bf16 operands, fp32 accumulation in TMEM)
+//
+// Layout of the work: units are (query tile of 128, split of the key tiles); a persistent grid walks them with
+// the query tile varying fastest, so the CTAs that run at the same time stream the same key range and share it
+// through L2. Each CTA:
+//   warp 0      TMA producer: per k-step, one 128x64 query box and one 256x64 key box (128-byte swizzle) into a
+//               4-stage shared-memory ring (mbarrier full/empty pairs);
+//   warp 1      MMA issuer: allocates 512 TMEM columns (two 128x256 fp32 accumulators) and issues
+//               tcgen05.mma kind::f16 (M=128, N=256, K=16) from one thread; tcgen05.commit frees ring stages
+//               and hands a finished accumulator to the epilogue;
+//   warps 2..5  epilogue: thread = query row (TMEM lane); reads its 256 scores with tcgen05.ld, keeps a sorted
+//               top_c of (score, id) in registers with the threshold max(tau_c, current c-th best), and finally
+//               writes the unit's partial list. Double-buffered accumulators overlap it with the next tile's MMAs.
+// Every mbarrier wait is bounded: on a timeout the CTA records LACACHE_ERR_DEVICE_TIMEOUT in the status word, the
+// other roles see an abort flag and stop, in-flight copies and MMAs are drained, TMEM is freed and the CTA exits.
+#include <cuda.h>
+#include <string.h>
+
+#include "internal.cuh"
+
+namespace lc {
+namespace {
+
+constexpr int BM = 128;                     // queries per tile (TMEM lanes)
+constexpr int BN = 256;                     // keys per tile (accumulator columns)
+constexpr int BK = 64;                      // bf16 per k-step = one 128-byte swizzled row
+constexpr int STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;        // 16 KB
+constexpr int B_BYTES = BN * BK * 2;        // 32 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int TMEM_COLS = 2 * BN;           // two accumulators
+constexpr int kThreads = 192;
+constexpr int kEpiWarps = 4;
+constexpr long long kWaitCycles = 2000000000LL;   // about one second of SM clock
+constexpr int kBarriers = 2 * STAGES + 5;          // full, empty, tmem_full x2, tmem_empty x2, drain
+constexpr size_t kStashBytes = 32 * 129 * 4;          // epilogue's rare-path chunk stash
+constexpr size_t kSmemBytes = 1024 + (size_t)STAGES * STAGE_BYTES + kBarriers * 8 + 16 + kStashBytes;
+
+// tcgen05 instruction descriptor, kind::f16: D f32 (bits 4-5 = 1), A bf16 (bits 7-9 = 1), B bf16 (bits 10-12 =
+// 1), A and B K-major (bits 15, 16 = 0), N >> 3 in bits 17-22, M >> 4 in bits 24-28.
+constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                            ((uint32_t)(BM >> 4) << 24);
+
+struct TcParams {
+  int64_t n;
+  int d;
+  int B;
+  float tau_c;
+  int top_c;
+  int q_tiles;
+  int splits;
+  int units;
+  int64_t n_tiles;
+  int k_steps;
+  uint64_t* part_cand;
+  float* part_best;
+  unsigned int* dev_status;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Wait for the phase of the given parity to complete; false after about a second, or when another role aborted.
+__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const volatile uint32_t* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  const long long t0 = clock64();
+  while (true) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (abort_flag && *abort_flag) return false;
+    if (clock64() - t0 > kWaitCycles) return false;
+  }
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
+  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+      ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(kIdesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+
+// Shared-memory matrix descriptor of a K-major operand tile written by TMA with 128-byte swizzle: rows of 128 B,
+// 8-row groups 1024 B apart (stride byte offset), leading byte offset unused for this layout (16 B), descriptor
+// version 1 (bits 46-47), swizzle mode 2 = 128 B (bits 61-63). The tile base is 1024-byte aligned.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t addr) {
+  uint64_t desc = (uint64_t)((addr >> 4) & 0x3FFFu);
+  desc |= (uint64_t)1 << 16;
+  desc |= (uint64_t)(1024 >> 4) << 32;
+  desc |= (uint64_t)1 << 46;
+  desc |= (uint64_t)2 << 61;
+  return desc;
+}
+
+// 32 consecutive fp32 accumulator columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+      "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+      "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Running top_c of one query: scores descending; among equal scores the earlier (lower) id first, which holds
+// because ids arrive in increasing order. Slots past top_c are kept but never read.
+template <int CPAD>
+struct TopC {
+  float s[CPAD];
+  uint32_t j[CPAD];
+  int count;
+  float thr;  // a new candidate enters iff score >= thr
+
+  __device__ __forceinline__ void init(float tau_c) {
+#pragma unroll
+    for (int i = 0; i < CPAD; ++i) {
+      s[i] = -INFINITY;
+      j[i] = 0xFFFFFFFFu;
+    }
+    count = 0;
+    thr = tau_c;
+  }
+  __device__ __forceinline__ void insert(float v, uint32_t id, int c) {
+#pragma unroll
+    for (int i = 0; i < CPAD; ++i) {
+      if (v > s[i]) {
+        const float ts = s[i];
+        const uint32_t tj = j[i];
+        s[i] = v;
+        j[i] = id;
+        v = ts;
+        id = tj;
+      }
+    }
+    if (count < c) ++count;
+    if (count >= c) {
+      // the c-th best is the minimum of the first c (sorted) slots; written as a masked min so that it stays a
+      // register computation rather than a dynamically indexed (local-memory) read of s[c - 1]
+      float w = INFINITY;
+#pragma unroll
+      for (int i = 0; i < CPAD; ++i) w = fminf(w, i < c ? s[i] : INFINITY);
+      thr = fmaxf(thr, nextafterf(w, INFINITY));   // equal scores arrive with larger ids: they lose
+    }
+  }
+};
+
+template <int CPAD>
+__global__ void __launch_bounds__(kThreads, 1)
+    stage1_tensor_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
+                         const TcParams p) {
+  extern __shared__ unsigned char smem_raw[];
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  unsigned char* gbase = smem_raw + (base - raw);
+  const uint32_t a_smem = base;
+  const uint32_t b_smem = base + STAGES * A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(gbase + (size_t)STAGES * STAGE_BYTES);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kBarriers);
+  float* stash = reinterpret_cast<float*>(tmem_slot + 4);
+  volatile uint32_t* abort_flag = tmem_slot + 1;
+  const uint32_t bar0 = smem_u32(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+  auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
+  auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull_bar(b), 1);
+      mbar_init(tempty_bar(b), kEpiWarps);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmap_q);
+    tma_prefetch_desc(&tmap_k);
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  auto fail = [&]() {
+    *abort_flag = 1u;
+    atomicOr(p.dev_status, kDevTimeout);
+  };
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ---------------- TMA producer ----------------
+      uint32_t it = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
+        const int qt = u % p.q_tiles, sp = u / p.q_tiles;
+        const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
+        for (int64_t t = t_begin; ok && t < t_end; ++t) {
+          for (int ks = 0; ks < p.k_steps; ++ks, ++it) {
+            const int s = it % STAGES;
+            const uint32_t ph = (it / STAGES) & 1u;
+            if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) {
+              fail();
+              ok = false;
+              break;
+            }
+            mbar_expect_tx(full_bar(s), STAGE_BYTES);
+            tma_load_2d(a_smem + s * A_BYTES, &tmap_q, full_bar(s), ks * BK, qt * BM);
+            tma_load_2d(b_smem + s * B_BYTES, &tmap_k, full_bar(s), ks * BK, (int)(t * BN));
+          }
+        }
+      }
+      // drain: the last load issued into each stage has landed before the CTA may exit
+      const uint32_t first = it > (uint32_t)STAGES ? it - STAGES : 0u;
+      for (uint32_t i = first; i < it; ++i)
+        if (!mbar_wait(full_bar(i % STAGES), (i / STAGES) & 1u, nullptr)) fail();
+    }
+  } else if (warp == 1) {
+    if (lane == 0) {
+      // ---------------- MMA issuer ----------------
+      uint32_t it = 0, tile_i = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
+        const int sp = u / p.q_tiles;
+        const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
+        for (int64_t t = t_begin; ok && t < t_end; ++t, ++tile_i) {
+          const int b = tile_i & 1u;
+          if (!mbar_wait(tempty_bar(b), ((tile_i >> 1) & 1u) ^ 1u, abort_flag)) {
+            fail();
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem + (uint32_t)(b * BN);
+          for (int ks = 0; ks < p.k_steps; ++ks, ++it) {
+            const int s = it % STAGES;
+            if (!mbar_wait(full_bar(s), (it / STAGES) & 1u, abort_flag)) {
+              fail();
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint64_t ad = smem_desc(a_smem + s * A_BYTES);
+            const uint64_t bd = smem_desc(b_smem + s * B_BYTES);
+#pragma unroll
+            for (int kk = 0; kk < BK / 16; ++kk)
+              mma_bf16(d_tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), (ks | kk) != 0 ? 1u : 0u);
+            mma_commit(empty_bar(s));
+          }
+          if (ok) mma_commit(tfull_bar(b));
+        }
+      }
+      // drain: every MMA issued by this thread has completed before TMEM is freed
+      mma_commit(drain_bar);
+      if (!mbar_wait(drain_bar, 0, nullptr)) fail();
+    }
+  } else {
+    // ---------------- epilogue ----------------
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    float* my_stash = stash + row;   // column-major [32][129]: conflict-free across a warp
+    const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+    uint32_t tile_i = 0;
+    bool ok = true;
+    const unsigned full = 0xffffffffu;
+    for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
+      const int qt = u % p.q_tiles, sp = u / p.q_tiles;
+      const int q = qt * BM + row;
+      const bool active = q < p.B;
+      const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
+      TopC<CPAD> top;
+      top.init(p.tau_c);
+      float best = -INFINITY;
+      for (int64_t t = t_begin; t < t_end; ++t, ++tile_i) {
+        const int b = tile_i & 1u;
+        const uint32_t par = (tile_i >> 1) & 1u;
+        // every lane waits (each needs the barrier's acquire); the warp proceeds only if all lanes saw the
+        // phase complete, so the warp-collective tcgen05.ld below is never reached by part of a warp
+        const bool got = mbar_wait(tfull_bar(b), par, abort_flag);
+        if (!__all_sync(full, got)) {
+          if (lane == 0) fail();
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int64_t j0 = t * BN;
+        const bool ragged = j0 + BN > p.n;
+#pragma unroll 1
+        for (int ch = 0; ch < BN / 32; ++ch) {
+          float v[32];
+          tmem_ld32(tmem + lane_addr + (uint32_t)(b * BN + ch * 32), v);
+          if (active) {
+            const int64_t jc = j0 + ch * 32;
+            if (ragged) {
+#pragma unroll
+              for (int e = 0; e < 32; ++e)
+                if (jc + e >= p.n) v[e] = -INFINITY;
+            }
+            float m = v[0];
+#pragma unroll
+            for (int e = 1; e < 32; ++e) m = fmaxf(m, v[e]);
+            best = fmaxf(best, m);
+            if (m >= top.thr) {
+              // rare path: stash the chunk in shared memory and insert the entries that clear the threshold
+              uint32_t mask = 0;
+#pragma unroll
+              for (int e = 0; e < 32; ++e) {
+                mask |= (v[e] >= top.thr ? 1u : 0u) << e;
+                my_stash[e * 129] = v[e];
+              }
+              while (mask) {
+                const int e = __ffs(mask) - 1;
+                mask &= mask - 1;
+                const float x = my_stash[e * 129];
+                if (x >= top.thr && jc + e < p.n) top.insert(x, (uint32_t)(jc + e), p.top_c);
+              }
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(tempty_bar(b));
+      }
+      if (!ok) break;
+      if (active) {
+        uint64_t* dst = p.part_cand + ((int64_t)sp * p.B + q) * p.top_c;
+#pragma unroll
+        for (int i = 0; i < CPAD; ++i)
+          if (i < p.top_c) dst[i] = i < top.count ? pack_cand(top.s[i], top.j[i]) : 0ull;
+        p.part_best[(int64_t)sp * p.B + q] = best;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, TMEM_COLS);
+  }
+}
+
+int gcd_int(int a, int b) {
+  while (b) {
+    const int t = a % b;
+    a = b;
+    b = t;
+  }
+  return a;
+}
+
+template <int CPAD>
+cudaError_t launch_cpad(const CUtensorMap* tq, const CUtensorMap* tk, const TcParams& p, int grid, cudaStream_t st) {
+  cudaError_t e = cudaFuncSetAttribute(stage1_tensor_kernel<CPAD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)kSmemBytes);
+  if (e != cudaSuccess) return e;
+  stage1_tensor_kernel<CPAD><<<grid, kThreads, kSmemBytes, st>>>(*tq, *tk, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_stage1_tensor(const Stage1Args& a, const void* tmap_q, const void* tmap_k, int num_sms,
+                                 int max_splits, cudaStream_t st, int* splits) {
+  TcParams p;
+  p.n = a.n;
+  p.d = a.d;
+  p.B = a.B;
+  p.tau_c = a.tau_c;
+  p.top_c = a.top_c;
+  p.q_tiles = (a.B + BM - 1) / BM;
+  p.n_tiles = (a.n + BN - 1) / BN;
+  p.k_steps = (a.d + BK - 1) / BK;
+  // splits such that q_tiles * splits is a multiple of the SM count (whole waves of units)
+  int s = num_sms / gcd_int(num_sms, p.q_tiles);
+  if ((int64_t)s > p.n_tiles) s = (int)p.n_tiles;
+  if (s > max_splits) s = max_splits;
+  if (s < 1) s = 1;
+  p.splits = s;
+  p.units = p.q_tiles * s;
+  p.part_cand = a.part_cand;
+  p.part_best = a.part_best;
+  p.dev_status = a.dev_status;
+  *splits = s;
+  const int grid = p.units < num_sms ? p.units : num_sms;
+  const CUtensorMap* tq = static_cast<const CUtensorMap*>(tmap_q);
+  const CUtensorMap* tk = static_cast<const CUtensorMap*>(tmap_k);
+  if (a.top_c <= 4) return launch_cpad<4>(tq, tk, p, grid, st);
+  if (a.top_c <= 8) return launch_cpad<8>(tq, tk, p, grid, st);
+  if (a.top_c <= 16) return launch_cpad<16>(tq, tk, p, grid, st);
+  return launch_cpad<32>(tq, tk, p, grid, st);
+}
+
+}  // namespace lc

@@ -1,0 +1,214 @@
+// Candidate merge, stage 2 (the lookahead check) and the decision, fused in one kernel.
+//
+// One CTA (8 warps) per query:
+//  1. merge the stage-1 partial lists (splits x top_c packed candidates) into C_q, the top_c candidates by
+//     (key score desc, entry id asc): every thread keeps a sorted top-c of the entries it reads (loads issued
+//     four at a time), each warp reduces its lanes' lists by top_c rounds of a warp-wide max, and warp 0 merges
+//     the eight warp lists the same way;
+//  2. the candidates are checked in parallel, one warp per candidate: r = <p_q, P_j> (the prefix-embedding cosine
+//     sim(f_k(x), f_k(x'))) in fp32, each lane's 8-element chunks in order, then a butterfly sum (every lane ends
+//     with the same bits); m = number of positions i < k with equal token ids;
+//  3. the served entry is the first candidate in C_q order that passes (Algorithm 1); status HIT / REJECT /
+//     MISS_KEY.
+#include "internal.cuh"
+
+namespace lc {
+namespace {
+
+constexpr int kWarps = 8;
+constexpr int kThreads = kWarps * 32;
+constexpr unsigned kFull = 0xffffffffu;
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  return v;
+}
+
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const uint64_t other = __shfl_xor_sync(kFull, v, o);
+    v = other > v ? other : v;
+  }
+  return v;
+}
+
+__device__ __forceinline__ float dot8(const uint4& u, const uint4& v, float acc) {
+  const __nv_bfloat162* a = reinterpret_cast<const __nv_bfloat162*>(&u);
+  const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 x = __bfloat1622float2(a[e]);
+    const float2 y = __bfloat1622float2(b[e]);
+    acc = fmaf(x.x, y.x, acc);
+    acc = fmaf(x.y, y.y, acc);
+  }
+  return acc;
+}
+
+template <int CPAD>
+__device__ __forceinline__ void keep(uint64_t (&loc)[CPAD], uint64_t x) {
+  if (x > loc[CPAD - 1]) {
+#pragma unroll
+    for (int i = 0; i < CPAD; ++i) {
+      if (x > loc[i]) {
+        const uint64_t t = loc[i];
+        loc[i] = x;
+        x = t;
+      }
+    }
+  }
+}
+
+template <int CPAD>
+__global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
+  __shared__ uint64_t warp_top[kWarps][CPAD];
+  __shared__ uint64_t cand[CPAD];
+  __shared__ float cand_r[CPAD];
+  __shared__ int cand_m[CPAD];
+  __shared__ float warp_best[kWarps];
+  __shared__ int s_ncand;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int q = blockIdx.x;
+  const int C = a.top_c;
+
+  // 1a. best key score over all entries (max over the splits' maxima)
+  float best = -INFINITY;
+  for (int s = threadIdx.x; s < a.splits; s += kThreads) best = fmaxf(best, a.part_best[(int64_t)s * a.B + q]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(kFull, best, o));
+  if (lane == 0) warp_best[warp] = best;
+
+  // 1b. thread-local top-c of the partial entries
+  uint64_t loc[CPAD];
+#pragma unroll
+  for (int i = 0; i < CPAD; ++i) loc[i] = 0;
+  const int total = a.splits * C;
+  for (int e0 = threadIdx.x; e0 < total; e0 += 4 * kThreads) {
+    uint64_t x[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int e = e0 + u * kThreads;
+      x[u] = 0;
+      if (e < total) {
+        const int s = e / C;
+        x[u] = a.part_cand[((int64_t)s * a.B + q) * C + (e - s * C)];
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (x[u] != 0 && (int64_t)cand_id(x[u]) >= a.n) x[u] = 0;   // never gather outside the store
+      keep(loc, x[u]);
+    }
+  }
+  // 1c. per-warp top-c
+  for (int r = 0; r < C; ++r) {
+    const uint64_t m = warp_max_u64(loc[0]);
+    if (loc[0] == m && m != 0) {
+#pragma unroll
+      for (int i = 0; i < CPAD - 1; ++i) loc[i] = loc[i + 1];
+      loc[CPAD - 1] = 0;
+    }
+    if (lane == 0) warp_top[warp][r] = m;
+  }
+  __syncthreads();
+  // 1d. warp 0 merges the eight warp lists: lane l < kWarps walks list l
+  if (warp == 0) {
+    int head = 0;
+    int n = 0;
+    for (int r = 0; r < C; ++r) {
+      const uint64_t h = (lane < kWarps && head < C) ? warp_top[lane][head] : 0;
+      const uint64_t m = warp_max_u64(h);
+      if (m == 0) break;
+      if (h == m) ++head;
+      if (lane == 0) cand[r] = m;
+      ++n;
+    }
+    if (lane == 0) {
+      s_ncand = n;
+      float b = warp_best[0];
+      for (int w = 1; w < kWarps; ++w) b = fmaxf(b, warp_best[w]);
+      warp_best[0] = b;
+    }
+  }
+  __syncthreads();
+  const int n_cand = s_ncand;
+
+  // 2. lookahead check of every candidate, one warp per candidate
+  const int d = a.d, k = a.k;
+  const uint4* pq = reinterpret_cast<const uint4*>(a.q_prefix + (int64_t)q * d);
+  const int32_t* tq = a.q_ids + (int64_t)q * k;
+  for (int i = warp; i < n_cand; i += kWarps) {
+    const uint32_t j = cand_id(cand[i]);
+    const uint4* pj = reinterpret_cast<const uint4*>(a.prefix + (int64_t)j * d);
+    float acc = 0.f;
+    for (int c8 = lane; c8 < d / 8; c8 += 32) acc = dot8(__ldg(pq + c8), __ldg(pj + c8), acc);
+    const float r = warp_sum(acc);
+    int eq = 0;
+    const int32_t* tj = a.ids + (int64_t)j * k;
+    for (int t = lane; t < k; t += 32) eq += (__ldg(tq + t) == __ldg(tj + t)) ? 1 : 0;
+    const int m = __reduce_add_sync(kFull, eq);
+    if (lane == 0) {
+      cand_r[i] = r;
+      cand_m[i] = m;
+    }
+  }
+  __syncthreads();
+
+  // optional per-candidate outputs
+  const float qnan = __int_as_float(0x7fc00000);
+  for (int i = threadIdx.x; i < C; i += kThreads) {
+    const int64_t o = (int64_t)q * C + i;
+    const bool v = i < n_cand;
+    if (a.out.cand_id) a.out.cand_id[o] = v ? (int32_t)cand_id(cand[i]) : -1;
+    if (a.out.cand_score) a.out.cand_score[o] = v ? cand_score(cand[i]) : qnan;
+    if (a.out.cand_prefix_score) a.out.cand_prefix_score[o] = v ? cand_r[i] : qnan;
+    if (a.out.cand_matches) a.out.cand_matches[o] = v ? cand_m[i] : -1;
+  }
+
+  // 3. decision: the first candidate, in C_q order, that passes
+  if (threadIdx.x == 0) {
+    const int tmin = a.token_match_min > 0 ? a.token_match_min : k;
+    int served = -1;
+    for (int i = 0; i < n_cand && served < 0; ++i) {
+      const bool emb_ok = cand_r[i] >= a.tau_a;
+      const bool tok_ok = cand_m[i] >= tmin;
+      const bool pass = a.check_mode == LACACHE_CHECK_EMB ? emb_ok
+                        : a.check_mode == LACACHE_CHECK_TOKENS ? tok_ok
+                                                               : (emb_ok && tok_ok);
+      if (pass) served = i;
+    }
+    if (served >= 0) {
+      a.out.status[q] = LACACHE_HIT;
+      a.out.entry_id[q] = (int32_t)cand_id(cand[served]);
+      a.out.key_score[q] = cand_score(cand[served]);
+      a.out.prefix_score[q] = cand_r[served];
+      a.out.token_matches[q] = cand_m[served];
+    } else {
+      a.out.status[q] = n_cand ? LACACHE_REJECT : LACACHE_MISS_KEY;
+      a.out.entry_id[q] = -1;
+      a.out.key_score[q] = warp_best[0];
+      a.out.prefix_score[q] = n_cand ? cand_r[0] : qnan;
+      a.out.token_matches[q] = n_cand ? cand_m[0] : -1;
+    }
+    a.out.n_cand[q] = n_cand;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_stage2(const Stage2Args& a, cudaStream_t st) {
+  if (a.top_c <= 4)
+    stage2_kernel<4><<<a.B, kThreads, 0, st>>>(a);
+  else if (a.top_c <= 8)
+    stage2_kernel<8><<<a.B, kThreads, 0, st>>>(a);
+  else if (a.top_c <= 16)
+    stage2_kernel<16><<<a.B, kThreads, 0, st>>>(a);
+  else
+    stage2_kernel<32><<<a.B, kThreads, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace lc

@@ -1,0 +1,170 @@
+"""Helpers for the GPU-vs-oracle parity tests: build a device cache from a workload, run lookups through the C ABI,
+feed the oracle the same bytes, and compare.
+
+The comparison rules follow from the arithmetic. The GPU accumulates bf16 products in fp32; the oracle sums
+them exactly in fp64. For unit vectors with d <= 8192, the fp32 error is far below TOL = 2e-3:
+  * scores (key, prefix; per candidate) agree within TOL everywhere;
+  * status, entry id, token matches and candidate count agree exactly for every query whose oracle decision
+    margin is >= TOL (the others are counted and reported; for them a HIT must still pass both checks
+    within TOL);
+  * a candidate id must agree exactly unless its score is within TOL of a neighbour in the oracle's order (a
+    near-tie), in which case it must be one of the oracle's tied entries.
+"""
+from __future__ import annotations
+
+import dataclasses
+
+import numpy as np
+import torch
+
+import oracle
+from paper_2608_01718_gb300 import lacache as L
+from paper_2608_01718_gb300 import workloads as wl
+
+TOL = 2e-3
+
+
+def new_cache(w: wl.Workload, stage1: int, device: int = 0, capacity: int | None = None, **kw) -> L.LaCache:
+    return L.LaCache(w.d, w.k, capacity or w.n, w.tau_c, w.tau_a, w.top_c, max_batch=kw.pop("max_batch", w.batch),
+                     device=device, stage1=stage1, **kw)
+
+
+def fill(cache: L.LaCache, w: wl.Workload, device="cuda") -> None:
+    dtype = L.LACACHE_F32 if w.key_dtype == "f32" else L.LACACHE_BF16
+    for ch in wl.iter_store(w, device):
+        cache.insert(ch["key"], ch["prefix"], ch["ids"], dtype)
+    torch.cuda.synchronize()
+
+
+def _bits(t: torch.Tensor, f32: bool):
+    return oracle.round_to_bf16(wl.f32_array(t)) if f32 else wl.bf16_bits(t)
+
+
+def oracle_store(w: wl.Workload, device="cuda") -> oracle.Store:
+    """The whole initial store as host bf16 bit patterns (for caches that fit host memory)."""
+    keys, pres, ids = [], [], []
+    f32 = w.key_dtype == "f32"
+    for ch in wl.iter_store(w, device):
+        keys.append(_bits(ch["key"], f32))
+        pres.append(_bits(ch["prefix"], f32))
+        ids.append(ch["ids"].cpu().numpy())
+    return oracle.Store.of(np.concatenate(keys), np.concatenate(pres), np.concatenate(ids))
+
+
+def oracle_queries(q: dict, rows=None) -> dict:
+    sel = slice(None) if rows is None else rows
+    return {"emb": wl.bf16_bits(q["emb"][sel]), "prefix": wl.bf16_bits(q["prefix"][sel]),
+            "ids": q["ids"][sel].cpu().numpy()}
+
+
+def params(w: wl.Workload, check_mode=oracle.CHECK_EMB, token_match_min=None) -> oracle.Params:
+    # the GPU compares fp32 scores with the fp32 thresholds it was given; the oracle takes the same values
+    return oracle.Params(float(np.float32(w.tau_c)), float(np.float32(w.tau_a)), w.top_c, check_mode,
+                         token_match_min)
+
+
+def gpu_lookup(cache: L.LaCache, q: dict) -> dict:
+    out = cache.lookup(q["emb"], q["prefix"], q["ids"])
+    torch.cuda.synchronize()
+    cache.sync()
+    return {k: v.cpu().numpy() for k, v in out.items()}
+
+
+@dataclasses.dataclass
+class Report:
+    queries: int = 0
+    band: int = 0
+    literal_band: int = 0
+    exact: int = 0
+    hits: int = 0
+    rejects: int = 0
+    misses: int = 0
+    near_ties: int = 0
+
+    def add(self, other: "Report") -> None:
+        for f in dataclasses.fields(self):
+            setattr(self, f.name, getattr(self, f.name) + getattr(other, f.name))
+
+
+def _close(a, b, tol=TOL) -> bool:
+    if np.isnan(a) and np.isnan(b):
+        return True
+    if np.isinf(a) or np.isinf(b):
+        return a == b
+    return abs(float(a) - float(b)) <= tol
+
+
+def compare(gpu: dict, res: oracle.Result, p: oracle.Params, rows=None, pair_scores=None) -> Report:
+    """Check a GPU lookup against the oracle's result for the same queries (``rows`` selects GPU rows).
+
+    ``pair_scores(b, j)`` -> (s, r) gives the oracle's exact scores of query b against entry j, used to validate a
+    HIT inside the margin band.
+    """
+    idx = np.arange(len(res.status)) if rows is None else np.asarray(rows)
+    rep = Report(queries=len(idx))
+    rep.literal_band = int(np.sum(res.literal_margin < TOL))
+    for b, g in enumerate(idx):
+        st = int(gpu["status"][g])
+        assert st in (oracle.MISS_KEY, oracle.HIT, oracle.REJECT), f"query {g}: status {st}"
+        in_band = res.margin[b] < TOL
+        if in_band:
+            rep.band += 1
+            if st == oracle.HIT and pair_scores is not None:
+                s, r, m, k = pair_scores(b, int(gpu["entry_id"][g]))
+                assert s >= p.tau_c - TOL, f"query {g}: in-band HIT fails the key check"
+                if p.check_mode in (oracle.CHECK_EMB, oracle.CHECK_BOTH):
+                    assert r >= p.tau_a - TOL, f"query {g}: in-band HIT fails the lookahead check"
+                if p.check_mode in (oracle.CHECK_TOKENS, oracle.CHECK_BOTH):
+                    assert m >= (p.token_match_min or k), f"query {g}: in-band HIT fails the token check"
+            continue
+        msg = f"query {g} (oracle row {b})"
+        assert st == res.status[b], f"{msg}: status {st} vs oracle {res.status[b]}"
+        assert gpu["entry_id"][g] == res.entry_id[b], f"{msg}: entry {gpu['entry_id'][g]} vs {res.entry_id[b]}"
+        assert _close(gpu["key_score"][g], res.key_score[b]), f"{msg}: key score {gpu['key_score'][g]} vs {res.key_score[b]}"
+        assert _close(gpu["prefix_score"][g], res.prefix_score[b]), f"{msg}: prefix score"
+        assert gpu["token_matches"][g] == res.token_matches[b], f"{msg}: token matches"
+        if res.list_margin[b] >= TOL:
+            assert gpu["n_cand"][g] == res.n_cand[b], f"{msg}: n_cand {gpu['n_cand'][g]} vs {res.n_cand[b]}"
+        if "cand_id" in gpu:
+            _compare_candidates(gpu, res, g, b, rep, msg)
+        rep.exact += 1
+        rep.hits += st == oracle.HIT
+        rep.rejects += st == oracle.REJECT
+        rep.misses += st == oracle.MISS_KEY
+    return rep
+
+
+def pair_scores_fn(store: oracle.Store, oq: dict):
+    """(s, r, m, k) of oracle query row b against entry j, from the host bytes through the oracle's own stages."""
+    def f(b, j):
+        kc = oracle.KeyCheck(oq["emb"][b:b + 1], -np.inf)
+        kc.add_rows(store.key[j:j + 1], j)
+        r, m = oracle.lookahead(oq["prefix"][b], oq["ids"][b], store.prefix[j:j + 1], store.ids[j:j + 1])
+        return float(kc.best[0]), float(r[0]), int(m[0]), store.ids.shape[1]
+    return f
+
+
+def _compare_candidates(gpu, res, g, b, rep, msg):
+    nc = int(res.n_cand[b])
+    c = res.cand_id.shape[1]
+    ng = int(gpu["n_cand"][g])
+    o_ids = list(res.cand_id[b, :nc])
+    o_scores = list(res.cand_score[b, :nc])
+    if res.next_id[b] >= 0:
+        o_ids.append(int(res.next_id[b]))
+        o_scores.append(float(res.next_score[b]))
+    for i in range(min(nc, ng)):
+        gid, gs = int(gpu["cand_id"][g, i]), float(gpu["cand_score"][g, i])
+        assert abs(gs - o_scores[i]) <= TOL, f"{msg}: candidate {i} score {gs} vs {o_scores[i]}"
+        tied = (i > 0 and o_scores[i - 1] - o_scores[i] < TOL) or \
+               (i + 1 < len(o_scores) and o_scores[i] - o_scores[i + 1] < TOL)
+        if not tied:
+            assert gid == o_ids[i], f"{msg}: candidate {i} id {gid} vs {o_ids[i]}"
+            assert _close(gpu["cand_prefix_score"][g, i], res.cand_prefix_score[b, i]), f"{msg}: cand r {i}"
+            assert gpu["cand_matches"][g, i] == res.cand_matches[b, i], f"{msg}: cand m {i}"
+        else:
+            rep.near_ties += 1
+            pos = [k for k, j in enumerate(o_ids) if j == gid]
+            assert pos and abs(o_scores[pos[0]] - gs) <= TOL, f"{msg}: tied candidate {gid} not in oracle order"
+    for i in range(ng, c):
+        assert gpu["cand_id"][g, i] == -1 and np.isnan(gpu["cand_score"][g, i])

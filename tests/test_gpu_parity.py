@@ -1,0 +1,206 @@
+"""GPU parity: the CUDA lookup (through the C ABI) against the fp64 oracle on the same seeded bytes.
+
+Both stage-1 kernels are covered (the tcgen05 tensor-core scan and the CUDA-core scan). Cases span several key
+tiles with a ragged tail, ragged query tiles and ragged k-steps, the empty cache, exact duplicates, inclusive
+thresholds, top_c = 1 and 32, every check mode, host-buffer lookups and the serve loop with appends.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_01718_gb300 import build
+from paper_2608_01718_gb300 import lacache as L
+from paper_2608_01718_gb300 import workloads as wl
+
+from parity import (TOL, Report, compare, fill, gpu_lookup, new_cache, oracle_queries, oracle_store, pair_scores_fn,
+                    params)
+
+pytestmark = pytest.mark.gpu
+
+PATHS = [pytest.param(L.LACACHE_STAGE1_TENSOR, id="tensor"), pytest.param(L.LACACHE_STAGE1_SIMT, id="simt")]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def library():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    build.build()
+    L.load()
+
+
+def run_parity(w, stage1, check_mode=oracle.CHECK_EMB, token_match_min=None, steps=(0,)):
+    st = oracle_store(w)
+    rep = Report()
+    with new_cache(w, stage1, check_mode=check_mode, token_match_min=token_match_min or 0) as cache:
+        fill(cache, w)
+        assert cache.size == w.n
+        for step in steps:
+            q = wl.batch(w, step, device="cuda")
+            g = gpu_lookup(cache, q)
+            splits, kernel = cache.last_launch()
+            assert kernel == stage1 and splits >= 1
+            oq = oracle_queries(q)
+            p = params(w, check_mode, token_match_min)
+            res = oracle.lookup(st, oq, p)
+            rep.add(compare(g, res, p, pair_scores=pair_scores_fn(st, oq)))
+    return rep
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+def test_tiny_reference_cache(stage1):
+    w = wl.WORKLOADS["tiny-4k"]
+    rep = run_parity(w, stage1, steps=(0, 1))
+    assert rep.band == 0 and rep.exact == 2 * w.batch
+    assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+def test_mid_cache_scaled_ragged_tail(stage1):
+    w = wl.WORKLOADS["mid-1m"].scaled(n=70_000)          # 273 full key tiles and a ragged one
+    rep = run_parity(w, stage1)
+    assert rep.exact + rep.band == w.batch and rep.band <= 1
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+def test_ragged_batch_dimension_and_k(stage1):
+    # B = 130: two query tiles, the second ragged; d = 200: the last k-step is ragged; k = 3; c = 5
+    w = wl.WORKLOADS["mid-1m"].scaled(n=5_000, d=200, k=3, batch=130, top_c=5, clusters=50, vocab=7)
+    rep = run_parity(w, stage1)
+    assert rep.exact + rep.band == w.batch and rep.band <= 2
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+@pytest.mark.parametrize("mode,tmin", [(oracle.CHECK_TOKENS, None), (oracle.CHECK_TOKENS, 2),
+                                       (oracle.CHECK_BOTH, None), (oracle.CHECK_BOTH, 3)])
+def test_check_modes(stage1, mode, tmin):
+    w = wl.WORKLOADS["tiny-4k"].scaled(n=3000, k=4, vocab=3, batch=48)   # small vocab: partial token matches
+    rep = run_parity(w, stage1, check_mode=mode, token_match_min=tmin)
+    assert rep.exact + rep.band == w.batch
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+@pytest.mark.parametrize("top_c", [1, 32])
+def test_top_c_extremes(stage1, top_c):
+    w = wl.WORKLOADS["tiny-4k"].scaled(top_c=top_c, batch=40)
+    rep = run_parity(w, stage1)
+    assert rep.exact + rep.band == w.batch
+
+
+def _dev(a, dtype=torch.bfloat16):
+    return torch.tensor(np.asarray(a, np.float32), device="cuda").to(dtype).contiguous()
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+def test_hand_built_duplicates_thresholds_and_order(stage1):
+    d = 64
+    e = np.eye(d)
+    half = np.zeros(d)
+    half[:4] = 0.5
+    keys = np.stack([e[1], e[0], e[0], half, e[0]])          # entries 1, 2, 4 share a key
+    pres = np.stack([e[5], e[6], e[7], e[8], e[7]])
+    ids = np.array([[1, 1], [2, 2], [3, 3], [4, 4], [3, 3]], np.int32)
+    qs = np.stack([e[0], e[0], half, e[9], e[0]])
+    qp = np.stack([e[7], e[6], e[8], e[9], e[5]])
+    qi = np.array([[3, 3], [2, 2], [4, 4], [0, 0], [0, 0]], np.int32)
+    # tau_c = 0.5: query 2 (= half) scores exactly 0.5 against entry 3 and entries 1, 2, 4 (inclusive)
+    with L.LaCache(d, 2, 16, 0.5, 0.5, 4, max_batch=8, stage1=stage1) as c:
+        c.insert(_dev(keys), _dev(pres), torch.tensor(ids, device="cuda"))
+        out = c.lookup(_dev(qs), _dev(qp), torch.tensor(qi, device="cuda"))
+        torch.cuda.synchronize()
+        g = {k: v.cpu().numpy() for k, v in out.items()}
+    assert list(g["status"]) == [L.LACACHE_HIT, L.LACACHE_HIT, L.LACACHE_HIT, L.LACACHE_MISS_KEY,
+                                 L.LACACHE_REJECT]
+    # query 0: candidates 1, 2, 4 tie at 1.0 -> id order; entry 1's prefix e6 fails, entry 2's e7 passes
+    assert list(g["cand_id"][0]) == [1, 2, 4, 3] and g["entry_id"][0] == 2
+    assert np.all(g["cand_score"][0, :3] == 1.0) and g["cand_score"][0, 3] == 0.5
+    assert g["entry_id"][1] == 1 and g["token_matches"][1] == 2
+    assert g["entry_id"][2] == 3 and g["key_score"][2] == 1.0
+    assert g["n_cand"][3] == 0 and g["key_score"][3] == 0.0 and np.isnan(g["prefix_score"][3])
+    assert g["entry_id"][4] == -1 and g["prefix_score"][4] == 0.0 and g["token_matches"][4] == 0
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+def test_empty_cache_is_all_key_misses(stage1):
+    with L.LaCache(64, 4, 128, 0.9, 0.8, 4, max_batch=8, stage1=stage1) as c:
+        q = _dev(np.eye(64)[:3])
+        out = c.lookup(q, q, torch.zeros((3, 4), dtype=torch.int32, device="cuda"))
+        torch.cuda.synchronize()
+        assert torch.all(out["status"] == L.LACACHE_MISS_KEY)
+        assert torch.all(out["key_score"] == -math.inf) and torch.all(out["entry_id"] == -1)
+        assert torch.all(out["cand_id"] == -1) and c.last_launch()[0] == 0
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+def test_host_buffer_lookup_matches_device_lookup(stage1):
+    w = wl.WORKLOADS["tiny-4k"]
+    with new_cache(w, stage1) as cache:
+        fill(cache, w)
+        q = wl.batch(w, 0, device="cuda")
+        g = gpu_lookup(cache, q)
+        hq = {k: q[k].cpu().pin_memory() for k in ("emb", "prefix", "ids")}
+        out = L.alloc_result(w.batch, w.top_c, "cpu", pinned=True)
+        L.lacache_lookup_host(cache.h, hq["emb"], hq["prefix"], hq["ids"], out)
+        for k, v in out.items():
+            assert np.array_equal(v.numpy(), g[k], equal_nan=True), k
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+def test_serve_loop_appends_misses_like_the_oracle(stage1):
+    w = wl.WORKLOADS["serve-2m"].scaled(n=20_000, batch=64, clusters=200)
+    steps = 12
+    loop = oracle.ServeLoop(w.n + steps * w.batch, w.d, w.k, params(w))
+    st = oracle_store(w)
+    loop.insert(st.key, st.prefix, st.ids)
+    with new_cache(w, stage1, capacity=w.n + steps * w.batch) as cache:
+        fill(cache, w)
+        for step in range(steps):
+            q = wl.batch(w, step, device="cuda")
+            out = cache.lookup(q["emb"], q["prefix"], q["ids"])
+            first, m = cache.append_misses(q["emb"], q["prefix"], q["ids"], out["status"])
+            g = {k: v.cpu().numpy() for k, v in out.items()}
+            oq = oracle_queries(q)
+            res, ofirst, om = loop.step(oq)
+            rep = compare(g, res, loop.params)
+            assert rep.band == 0 and (first, m) == (ofirst, om) and cache.size == loop.n
+        # the appended rows are the non-HIT queries, in order, bit for bit
+        n = cache.size - w.n
+        key = torch.empty((n, w.d), dtype=torch.bfloat16, device="cuda")
+        ids = torch.empty((n, w.k), dtype=torch.int32, device="cuda")
+        L.lacache_read_rows(cache.h, w.n, n, key=key, ids=ids)
+        torch.cuda.synchronize()
+        assert np.array_equal(wl.bf16_bits(key), loop.store.key[w.n:loop.n])
+        assert np.array_equal(ids.cpu().numpy(), loop.store.ids[w.n:loop.n])
+
+
+def test_insert_is_all_or_nothing_on_capacity():
+    with L.LaCache(64, 2, 10, 0.9, 0.8, 2, max_batch=4) as c:
+        rows = _dev(np.eye(64)[:8])
+        ids = torch.zeros((8, 2), dtype=torch.int32, device="cuda")
+        assert c.insert(rows, rows, ids) == 0
+        with pytest.raises(L.LacacheError) as e:
+            c.insert(rows, rows, ids)
+        assert e.value.status == L.LACACHE_ERR_CAPACITY and c.size == 8
+        assert c.insert(rows[:2], rows[:2], ids[:2]) == 8 and c.size == 10
+
+
+def test_invalid_lookup_arguments():
+    with L.LaCache(64, 2, 10, 0.9, 0.8, 2, max_batch=4) as c:
+        q = _dev(np.eye(64)[:8])
+        ids = torch.zeros((8, 2), dtype=torch.int32, device="cuda")
+        with pytest.raises(L.LacacheError) as e:
+            c.lookup(q, q, ids)                              # B = 8 > max_batch
+        assert e.value.status == L.LACACHE_ERR_INVALID_ARG
+        flat = torch.zeros(64 * 4 + 1, dtype=torch.bfloat16, device="cuda")
+        with pytest.raises(L.LacacheError):
+            c.lookup(flat[1:].view(4, 64), q[:4], ids[:4])    # misaligned embedding pointer
+
+
+@pytest.mark.parametrize("stage1", PATHS)
+def test_mid_cache_full_size(stage1):
+    """The benchmark workload at full size: 1,048,576 entries, d = 768, B = 32, every query checked."""
+    rep = run_parity(wl.WORKLOADS["mid-1m"], stage1)
+    assert rep.exact + rep.band == 32 and rep.band <= 1
+    assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0

@@ -1,0 +1,70 @@
+"""The C-ABI library builds, loads and exports every entry point include/lacache.h declares (CPU only: no
+compute calls are made here)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_01718_gb300 import build, lacache
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "lacache.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return lacache.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"^\s*(?:lacache_status|const char\*)\s+(lacache_\w+)\s*\(", text, re.M)))
+
+
+def test_header_declares_the_binding_names():
+    assert declared_functions() == sorted(lacache.EXPORTS)
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert ctypes.cast(getattr(lib, name), ctypes.c_void_p).value
+
+
+def test_status_strings(lib):
+    assert lacache.status_string(lacache.LACACHE_OK) == "ok"
+    assert lacache.status_string(lacache.LACACHE_ERR_CAPACITY) == "capacity exceeded"
+    assert lacache.status_string(99) == "unknown status"
+
+
+def test_struct_layouts_match_the_header():
+    # lacache_config: 2 x int32, int64, 2 x float, 6 x int32 = 48 bytes; lacache_result: 10 pointers
+    assert ctypes.sizeof(lacache.lacache_config) == 48
+    assert lacache.lacache_config.capacity.offset == 8
+    assert ctypes.sizeof(lacache.lacache_result) == 80
+
+
+def test_null_arguments_are_rejected_without_a_device(lib):
+    h = ctypes.c_void_p()
+    assert lib.lacache_create(None, ctypes.byref(h)) == lacache.LACACHE_ERR_INVALID_ARG
+    assert lib.lacache_create(ctypes.byref(lacache.make_config(64, 4, 16, .9, .8, 4, max_batch=8)), None) == \
+        lacache.LACACHE_ERR_INVALID_ARG
+    assert lib.lacache_destroy(None) == lacache.LACACHE_OK
+    assert lib.lacache_sync(None) == lacache.LACACHE_ERR_INVALID_ARG
+    n = ctypes.c_int64()
+    assert lib.lacache_size(None, ctypes.byref(n)) == lacache.LACACHE_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("field,value,status", [
+    ("d", 12, lacache.LACACHE_ERR_UNSUPPORTED), ("d", 0, lacache.LACACHE_ERR_INVALID_ARG),
+    ("top_c", 33, lacache.LACACHE_ERR_UNSUPPORTED), ("k", 0, lacache.LACACHE_ERR_INVALID_ARG),
+    ("check_mode", 7, lacache.LACACHE_ERR_INVALID_ARG), ("token_match_min", 9, lacache.LACACHE_ERR_INVALID_ARG),
+    ("tau_c", float("nan"), lacache.LACACHE_ERR_INVALID_ARG), ("max_batch", 0, lacache.LACACHE_ERR_INVALID_ARG),
+])
+def test_invalid_configs_are_rejected_before_touching_a_device(lib, field, value, status):
+    cfg = lacache.make_config(64, 8, 1024, 0.9, 0.8, 8, max_batch=16)
+    setattr(cfg, field, value)
+    h = ctypes.c_void_p(1)
+    assert lib.lacache_create(ctypes.byref(cfg), ctypes.byref(h)) == status
+    assert h.value is None
