@@ -160,6 +160,26 @@ lacache_status lacache_last_launch(const lacache_t* h, int32_t* n_splits, int32_
 lacache_status lacache_stage_timing(lacache_t* h, int32_t max_lookups);
 lacache_status lacache_stage_times(lacache_t* h, double* stage1_ms, double* stage2_ms, int64_t* lookups);
 
+/* Lookup that allocates nothing, for callers that cannot allocate device memory. Examples: a serving runtime or
+ * framework whose allocator owns all device memory, code that must not trigger the device synchronization that
+ * cudaMalloc and cudaFree can cause, and plug-ins with a fixed memory budget. The paper has no counterpart; this
+ * is a deployment variant of lacache_lookup.
+ *
+ * The cache rows are caller-owned device arrays in the store's layout: key_dev and prefix_dev [n x d] bf16
+ * (16-byte aligned), ids_dev [n x k] int32. Queries and outputs are as for lacache_lookup. From *cfg it uses
+ * d, k, tau_c, tau_a, top_c, token_match_min, check_mode, device and stage1; capacity and max_batch are ignored.
+ * The stage-1 scratch lives in an 8 MiB file-scope device array of the library, which every GPU that loads the
+ * library holds until the process exits. A batch needs B * (8 * top_c + 4) bytes of it; larger batches return
+ * LACACHE_ERR_UNSUPPORTED and nothing runs. The first call on a device does a one-time set-up (it looks up the
+ * array's device address), so make that first call before any stream capture. All calls on a device share the
+ * array: calls that overlap on the GPU (other streams, other host threads) race and give undefined results, so
+ * issue them on one stream. A device-side timeout is not reported by this entry point (its outputs are then
+ * undefined). Asynchronous on cuda_stream. */
+lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int64_t n, const void* key_dev,
+                                      const void* prefix_dev, const int32_t* ids_dev, int32_t B,
+                                      const void* q_emb_dev, const void* q_prefix_dev, const int32_t* q_ids_dev,
+                                      const lacache_result* out, void* cuda_stream);
+
 /* Static description of a status code. */
 const char* lacache_status_string(lacache_status s);
 

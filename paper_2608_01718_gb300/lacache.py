@@ -20,7 +20,7 @@ LACACHE_MISS_KEY, LACACHE_HIT, LACACHE_REJECT = 0, 1, 2
 
 EXPORTS = ["lacache_create", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
            "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
-           "lacache_stage_timing", "lacache_stage_times", "lacache_status_string"]
+           "lacache_stage_timing", "lacache_stage_times", "lacache_lookup_noalloc", "lacache_status_string"]
 
 
 class lacache_config(ctypes.Structure):
@@ -70,6 +70,8 @@ def load() -> ctypes.CDLL:
         "lacache_last_launch": ([vp, p32, p32], i32),
         "lacache_stage_timing": ([vp, i32], i32),
         "lacache_stage_times": ([vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double), p64], i32),
+        "lacache_lookup_noalloc": ([ctypes.POINTER(lacache_config), i64, vp, vp, vp, i32, vp, vp, vp,
+                                    ctypes.POINTER(lacache_result), vp], i32),
         "lacache_status_string": ([i32], ctypes.c_char_p),
     }
     for name, (args, res) in sig.items():
@@ -186,6 +188,16 @@ def lacache_stage_times(h: int) -> tuple[float, float, int]:
     t1, t2, n = ctypes.c_double(), ctypes.c_double(), ctypes.c_int64()
     _check("lacache_stage_times", load().lacache_stage_times(h, ctypes.byref(t1), ctypes.byref(t2), ctypes.byref(n)))
     return t1.value, t2.value, n.value
+
+
+def lacache_lookup_noalloc(cfg: lacache_config, key, prefix, ids, q_emb, q_prefix, q_ids, out: dict,
+                           cuda_stream=None) -> None:
+    """Lookup against caller-owned cache rows with no device allocation (see include/lacache.h)."""
+    res = _result_struct(out)
+    n = int(ids.shape[0]) if ids is not None else 0
+    _check("lacache_lookup_noalloc", load().lacache_lookup_noalloc(
+        ctypes.byref(cfg), n, _ptr(key), _ptr(prefix), _ptr(ids), int(q_emb.shape[0]), _ptr(q_emb),
+        _ptr(q_prefix), _ptr(q_ids), ctypes.byref(res), _stream(cuda_stream, cfg.device)))
 
 
 def alloc_result(batch: int, top_c: int, device, candidates: bool = True, pinned: bool = False) -> dict:

@@ -1,0 +1,73 @@
+"""lacache_lookup_noalloc: the lookup for callers that cannot allocate device memory.
+
+Callers under a runtime or framework allocator that owns all device memory, or that must not trigger the
+synchronization cudaMalloc/cudaFree can cause, cannot create a handle (lacache_create allocates the store and the
+stage-1 scratch). This entry point takes the cache rows as the caller's device arrays and keeps its scratch in a
+fixed device array of the library. The test checks it against lacache_lookup on the same rows, two calls in a
+row, and that a batch too large for the fixed scratch is refused. This file is named so pytest collects it last.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_01718_gb300 import build
+from paper_2608_01718_gb300 import lacache as L
+from paper_2608_01718_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+TOL = 2e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def library():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    build.build()
+    L.load()
+
+
+def _rows(w):
+    keys, pres, ids = [], [], []
+    for ch in wl.iter_store(w, "cuda"):
+        keys.append(ch["key"])
+        pres.append(ch["prefix"])
+        ids.append(ch["ids"])
+    return torch.cat(keys).contiguous(), torch.cat(pres).contiguous(), torch.cat(ids).contiguous()
+
+
+def _same(a: dict, b: dict):
+    for name in ("status", "entry_id", "n_cand", "token_matches", "cand_id", "cand_matches"):
+        assert torch.equal(a[name], b[name]), name
+    for name in ("key_score", "prefix_score", "cand_score", "cand_prefix_score"):
+        x, y = a[name].cpu().numpy(), b[name].cpu().numpy()
+        both_nan = np.isnan(x) & np.isnan(y)
+        assert np.all(both_nan | (np.abs(x - y) <= TOL) | (x == y)), name
+
+
+@pytest.mark.parametrize("stage1", [L.LACACHE_STAGE1_TENSOR, L.LACACHE_STAGE1_SIMT], ids=["tensor", "simt"])
+def test_noalloc_lookup_matches_the_handle_lookup(stage1):
+    w = wl.WORKLOADS["mid-1m"].scaled(n=50_000, batch=96)
+    key, pre, ids = _rows(w)
+    with L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch, stage1=stage1) as cache:
+        cache.insert(key, pre, ids)
+        for step in (0, 1):                       # two calls in a row share the fixed scratch
+            q = wl.batch(w, step, device="cuda")
+            ref = cache.lookup(q["emb"], q["prefix"], q["ids"])
+            out = L.alloc_result(w.batch, w.top_c, "cuda")
+            L.lacache_lookup_noalloc(cache.cfg, key, pre, ids, q["emb"], q["prefix"], q["ids"], out)
+            torch.cuda.synchronize()
+            _same(out, ref)
+            assert int((out["status"] == L.LACACHE_HIT).sum()) > 0
+
+
+def test_noalloc_refuses_a_batch_larger_than_its_scratch():
+    d, top_c = 64, 32
+    cfg = L.make_config(d, 4, 1, 0.9, 0.8, top_c, max_batch=1)
+    B = (8 << 20) // (8 * top_c + 4) + 1           # one query more than fits the 8 MiB scratch
+    q = torch.zeros((B, d), dtype=torch.bfloat16, device="cuda")
+    qi = torch.zeros((B, 4), dtype=torch.int32, device="cuda")
+    out = L.alloc_result(B, top_c, "cuda", candidates=False)
+    with pytest.raises(L.LacacheError) as e:
+        L.lacache_lookup_noalloc(cfg, None, None, None, q, q, qi, out)
+    assert e.value.status == L.LACACHE_ERR_UNSUPPORTED
