@@ -259,7 +259,6 @@ def run_ours(args, w):
     torch.cuda.synchronize()
     cache.sync()
     kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_SIMT: "simt"}[cache.last_launch()[1]]
-    L.lacache_stage_timing(cache.h, args.steps)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -276,6 +275,12 @@ def run_ours(args, w):
     clock = clocks.stop()
     cache.sync()
     elapsed_ms = ev0.elapsed_time(ev1)
+    # Second pass over the same steps with the library's stage events (recorded on the lookup's stream around
+    # each kernel) for the per-kernel times of the roofline. The events sit between the two kernels, so this pass
+    # is kept out of the throughput measurement above.
+    L.lacache_stage_timing(cache.h, args.steps)
+    for i in range(args.steps):
+        step(i)
     t1_ms, t2_ms, timed = L.lacache_stage_times(cache.h)
     L.lacache_stage_timing(cache.h, 0)
     if world > 1:
@@ -304,19 +309,29 @@ def run_ours(args, w):
     peaks, peak_src = load_peaks()
     s1_bytes, s2_bytes, flops = algorithmic(w, w.batch)
     t1_avg_s = t1_ms / max(1, timed) / 1e3
-    achieved = s1_bytes / t1_avg_s / 1e9
     traffic = kernel_traffic(kernel_name, w.name)
     value = world * args.steps * w.batch / (elapsed_ms / 1e3)
+    # the stage-1 kernel is bound by HBM below the ridge (flops per byte of the measured peaks), else by the
+    # tensor pipe; a kernel timed back to back for over a second is compared with the sustained bf16 peak
+    ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    if flops / s1_bytes < ridge:
+        roof = {"bound": "hbm", "achieved": s1_bytes / t1_avg_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "peak_source": f"{peak_src} (copy bandwidth)"}
+    else:
+        sustained = elapsed_ms > 1000.0 and "bf16_tflops_sustained" in peaks
+        peak = peaks["bf16_tflops_sustained"] if sustained else peaks["bf16_tflops"]
+        roof = {"bound": "tensor", "achieved": flops / t1_avg_s / 1e12, "peak": peak, "unit": "TFLOP/s",
+                "peak_source": f"{peak_src} ({'sustained' if sustained else 'burst'} bf16 dense)"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": workload_config(w) | {"parallelism": f"replicas{world}" if world > 1 else "single"},
         "stage1_kernel": kernel_name,
-        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peaks["hbm_gbs"], "unit": "GB/s",
-                     "frac": achieved / peaks["hbm_gbs"], "traffic": traffic, "kernel": f"stage1_{kernel_name}",
-                     "peak_source": f"{peak_src} (copy bandwidth)",
-                     "algorithmic_bytes_per_launch": s1_bytes, "avg_launch_ms": t1_avg_s * 1e3},
+        "roofline": roof | {"traffic": traffic, "kernel": f"stage1_{kernel_name}",
+                            "algorithmic_bytes_per_launch": s1_bytes, "algorithmic_flops_per_launch": flops,
+                            "avg_launch_ms": t1_avg_s * 1e3},
         "tensor": {"achieved_tflops": flops / (elapsed_ms / args.steps / 1e3) / 1e12,
                    "peak_tflops": peaks["bf16_tflops"],
                    "frac": flops / (elapsed_ms / args.steps / 1e3) / 1e12 / peaks["bf16_tflops"]},
@@ -328,7 +343,11 @@ def run_ours(args, w):
         "clocks": clock,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        rows = min(w.n, 1 << 20)
+        # a bounded sample: as many store rows as take about 15 s of oracle time (all of them if fewer)
+        probe = min(w.n, 8192)
+        store, oq = oracle_sample(w, probe, 0, "cuda")
+        per_row = time_oracle(store, oq, w) / probe
+        rows = int(min(w.n, max(probe, 15.0 / per_row)))
         store, oq = oracle_sample(w, rows, 0, "cuda")
         t = time_oracle(store, oq, w)
         line["cpu_baseline"] = {

@@ -9,10 +9,6 @@
 
 #include "internal.cuh"
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
 struct lacache {
   lacache_config cfg;
   int num_sms;
@@ -29,9 +25,10 @@ struct lacache {
   int32_t* append_count_host;  // pinned
   unsigned char* stage_in;   // device staging for lookup_host inputs
   unsigned char* stage_out;  // device staging for lookup_host results
+  unsigned char* stage_host; // pinned host copy of stage_out
   int last_splits;
   int last_kernel;
-  EncodeTiledFn encode;
+  lc::EncodeTiledFn encode;
   cudaEvent_t* events;       // [3 x event_cap] stage-timing events, or NULL
   int event_cap;
   int event_used;
@@ -129,27 +126,28 @@ size_t stage_out_bytes(const lacache_config& c) {
   return (size_t)c.max_batch * (21 + (size_t)c.top_c * 16) + 10 * 16;
 }
 
-// Device staging layout of the results of lookup_host (each array 16-byte aligned).
-lacache_result staged_result(lacache* h, int B) {
-  unsigned char* p = h->stage_out;
-  const size_t mb = (size_t)h->cfg.max_batch, tc = (size_t)h->cfg.top_c;
-  auto take = [&](size_t bytes) {
+// Layout of the results of lookup_host in the device staging buffer (and in its pinned host copy): the arrays of
+// a B-query batch packed back to back, each 16-byte aligned, so that one copy brings them all back.
+lacache_result staged_result(unsigned char* base, int B, int top_c, bool cand, size_t* bytes) {
+  unsigned char* p = base;
+  auto take = [&](size_t n) {
     unsigned char* r = p;
-    p += (bytes + 15) & ~(size_t)15;
+    p += (n + 15) & ~(size_t)15;
     return r;
   };
-  (void)B;
+  const size_t b = (size_t)B, bc = (size_t)B * top_c;
   lacache_result r;
-  r.entry_id = (int32_t*)take(mb * 4);
-  r.key_score = (float*)take(mb * 4);
-  r.prefix_score = (float*)take(mb * 4);
-  r.token_matches = (int32_t*)take(mb * 4);
-  r.n_cand = (int32_t*)take(mb * 4);
-  r.cand_id = (int32_t*)take(mb * tc * 4);
-  r.cand_score = (float*)take(mb * tc * 4);
-  r.cand_prefix_score = (float*)take(mb * tc * 4);
-  r.cand_matches = (int32_t*)take(mb * tc * 4);
-  r.status = (uint8_t*)take(mb);
+  r.entry_id = (int32_t*)take(b * 4);
+  r.key_score = (float*)take(b * 4);
+  r.prefix_score = (float*)take(b * 4);
+  r.token_matches = (int32_t*)take(b * 4);
+  r.n_cand = (int32_t*)take(b * 4);
+  r.status = (uint8_t*)take(b);
+  r.cand_id = cand ? (int32_t*)take(bc * 4) : nullptr;
+  r.cand_score = cand ? (float*)take(bc * 4) : nullptr;
+  r.cand_prefix_score = cand ? (float*)take(bc * 4) : nullptr;
+  r.cand_matches = cand ? (int32_t*)take(bc * 4) : nullptr;
+  *bytes = (size_t)(p - base);
   return r;
 }
 
@@ -175,17 +173,7 @@ void free_all(lacache* h) {
   cudaFree(h->stage_in);
   cudaFree(h->stage_out);
   if (h->append_count_host) cudaFreeHost(h->append_count_host);
-}
-
-bool encode_2d(lacache* h, CUtensorMap* m, const void* base, int64_t inner, int64_t outer, uint32_t box_inner,
-               uint32_t box_outer) {
-  const cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)outer};
-  const cuuint64_t strides[1] = {(cuuint64_t)inner * 2};
-  const cuuint32_t box[2] = {box_inner, box_outer};
-  const cuuint32_t estr[2] = {1, 1};
-  return h->encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  if (h->stage_host) cudaFreeHost(h->stage_host);
 }
 
 lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* q_prefix, const int32_t* q_ids,
@@ -212,10 +200,7 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
     cudaError_t e;
     if (kernel == LACACHE_STAGE1_TENSOR) {
       if (!h->encode) return LACACHE_ERR_CUDA;
-      CUtensorMap tq, tk;
-      if (!encode_2d(h, &tq, q_emb, c.d, B, 64, 128) || !encode_2d(h, &tk, h->key, c.d, h->n, 64, 256))
-        return LACACHE_ERR_CUDA;
-      e = lc::launch_stage1_tensor(a, &tq, &tk, h->num_sms, h->max_splits, st, &splits);
+      e = lc::launch_stage1_tensor(a, h->encode, h->num_sms, h->max_splits, st, &splits);
     } else {
       e = lc::launch_stage1_simt(a, h->num_sms, h->max_splits, st, &splits);
     }
@@ -306,6 +291,7 @@ lacache_status lacache_create(const lacache_config* cfg, lacache_t** out) {
             cudaMalloc(&h->stage_in, stage_in_bytes(c)) == cudaSuccess &&
             cudaMalloc(&h->stage_out, stage_out_bytes(c)) == cudaSuccess &&
             cudaMallocHost(&h->append_count_host, 4) == cudaSuccess &&
+            cudaMallocHost(&h->stage_host, stage_out_bytes(c)) == cudaSuccess &&
             cudaMemset(h->dev_status, 0, 4) == cudaSuccess &&
             cudaMemset(h->part_cand, 0, (size_t)h->max_splits * c.max_batch * c.top_c * 8) == cudaSuccess &&
             cudaDeviceSynchronize() == cudaSuccess;
@@ -320,7 +306,7 @@ lacache_status lacache_create(const lacache_config* cfg, lacache_t** out) {
   if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
           cudaSuccess &&
       q == cudaDriverEntryPointSuccess)
-    h->encode = reinterpret_cast<EncodeTiledFn>(fn);
+    h->encode = reinterpret_cast<lc::EncodeTiledFn>(fn);
   *out = h;
   return LACACHE_OK;
 }
@@ -393,30 +379,31 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
   if (e == cudaSuccess) e = cudaMemcpyAsync(q_pre, q_prefix_host, emb, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(q_ids, q_ids_host, (size_t)B * c.k * 4, cudaMemcpyHostToDevice, st);
   if (e != cudaSuccess) return LACACHE_ERR_CUDA;
-  lacache_result dev = staged_result(h, B);
-  if (!out_host->cand_id) dev.cand_id = nullptr;
-  if (!out_host->cand_score) dev.cand_score = nullptr;
-  if (!out_host->cand_prefix_score) dev.cand_prefix_score = nullptr;
-  if (!out_host->cand_matches) dev.cand_matches = nullptr;
+  const bool cand = out_host->cand_id || out_host->cand_score || out_host->cand_prefix_score ||
+                    out_host->cand_matches;
+  size_t bytes = 0;
+  lacache_result dev = staged_result(h->stage_out, B, c.top_c, cand, &bytes);
+  lacache_result host = staged_result(h->stage_host, B, c.top_c, cand, &bytes);
   lacache_status s = run_lookup(h, B, q_emb, q_pre, q_ids, dev, st);
   if (s != LACACHE_OK) return s;
+  if (cudaMemcpyAsync(h->stage_host, h->stage_out, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
+      cudaStreamSynchronize(st) != cudaSuccess)
+    return LACACHE_ERR_CUDA;
   const size_t b4 = (size_t)B * 4, bc4 = (size_t)B * c.top_c * 4;
   struct Copy {
     void* dst;
     const void* src;
     size_t bytes;
   } copies[] = {
-      {out_host->entry_id, dev.entry_id, b4},         {out_host->status, dev.status, (size_t)B},
-      {out_host->key_score, dev.key_score, b4},       {out_host->prefix_score, dev.prefix_score, b4},
-      {out_host->token_matches, dev.token_matches, b4}, {out_host->n_cand, dev.n_cand, b4},
-      {out_host->cand_id, dev.cand_id, bc4},          {out_host->cand_score, dev.cand_score, bc4},
-      {out_host->cand_prefix_score, dev.cand_prefix_score, bc4}, {out_host->cand_matches, dev.cand_matches, bc4},
+      {out_host->entry_id, host.entry_id, b4},         {out_host->status, host.status, (size_t)B},
+      {out_host->key_score, host.key_score, b4},       {out_host->prefix_score, host.prefix_score, b4},
+      {out_host->token_matches, host.token_matches, b4}, {out_host->n_cand, host.n_cand, b4},
+      {out_host->cand_id, host.cand_id, bc4},          {out_host->cand_score, host.cand_score, bc4},
+      {out_host->cand_prefix_score, host.cand_prefix_score, bc4}, {out_host->cand_matches, host.cand_matches, bc4},
   };
-  for (const Copy& cp : copies) {
-    if (!cp.dst) continue;
-    if (cudaMemcpyAsync(cp.dst, cp.src, cp.bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess) return LACACHE_ERR_CUDA;
-  }
-  return from_cuda(cudaStreamSynchronize(st));
+  for (const Copy& cp : copies)
+    if (cp.dst && cp.src) memcpy(cp.dst, cp.src, cp.bytes);
+  return LACACHE_OK;
 }
 
 lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,

@@ -1,6 +1,7 @@
 // Internal declarations shared by the lookup kernels and the C-ABI host code of liblacache.so.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
@@ -83,10 +84,16 @@ struct Stage2Args {
   lacache_result out;            // device pointers
 };
 
+// cuTensorMapEncodeTiled, obtained from the driver at run time.
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
 // Launchers (host). Each returns the CUDA error of the launch. `splits` is the number of partial lists written.
 cudaError_t launch_stage1_simt(const Stage1Args& a, int num_sms, int max_splits, cudaStream_t st, int* splits);
-cudaError_t launch_stage1_tensor(const Stage1Args& a, const void* tmap_q, const void* tmap_k, int num_sms,
-                                 int max_splits, cudaStream_t st, int* splits);
+// Encodes its own TMA descriptors for a.q and a.keys with `encode`.
+cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int num_sms, int max_splits,
+                                 cudaStream_t st, int* splits);
 cudaError_t launch_stage2(const Stage2Args& a, cudaStream_t st);
 
 // Largest split count any stage-1 launcher uses for a given SM count (sizes the scratch).

@@ -26,10 +26,6 @@ constexpr int kMaxDevices = 64;
 // host-side stand-in; kernels receive the device address found by cudaGetSymbolAddress below.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
 struct DeviceSetup {
   bool ready;
   unsigned char* scratch;   // device address of g_noalloc_scratch on this device
@@ -38,7 +34,7 @@ struct DeviceSetup {
 
 std::mutex g_setup_mutex;
 DeviceSetup g_setup[kMaxDevices];
-EncodeTiledFn g_encode = nullptr;
+lc::EncodeTiledFn g_encode = nullptr;
 
 // One-time set-up for `dev`, which must be the current device: the device address of the scratch array, the SM
 // count, and the TMA descriptor encoder. Nothing here allocates.
@@ -56,7 +52,7 @@ lacache_status setup_device(int dev, DeviceSetup* out) {
       if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
               cudaSuccess &&
           q == cudaDriverEntryPointSuccess)
-        g_encode = reinterpret_cast<EncodeTiledFn>(fn);
+        g_encode = reinterpret_cast<lc::EncodeTiledFn>(fn);
     }
     s.scratch = static_cast<unsigned char*>(ptr);
     s.num_sms = sms;
@@ -64,16 +60,6 @@ lacache_status setup_device(int dev, DeviceSetup* out) {
   }
   *out = s;
   return LACACHE_OK;
-}
-
-bool encode_rows(CUtensorMap* m, const void* base, int64_t d, int64_t rows, uint32_t box_rows) {
-  const cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
-  const cuuint64_t strides[1] = {(cuuint64_t)d * 2};
-  const cuuint32_t box[2] = {64, box_rows};
-  const cuuint32_t estr[2] = {1, 1};
-  return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
@@ -142,12 +128,8 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
       const int kernel = c.stage1 == LACACHE_STAGE1_AUTO ? LACACHE_STAGE1_TENSOR : c.stage1;
       cudaError_t e;
       if (kernel == LACACHE_STAGE1_TENSOR) {
-        CUtensorMap tq, tk;
-        if (!g_encode || !encode_rows(&tq, q_emb_dev, c.d, B, 128) || !encode_rows(&tk, key_dev, c.d, n, 256)) {
-          e = cudaErrorInvalidValue;
-        } else {
-          e = lc::launch_stage1_tensor(a, &tq, &tk, s.num_sms, max_splits, st, &splits);
-        }
+        e = g_encode ? lc::launch_stage1_tensor(a, g_encode, s.num_sms, max_splits, st, &splits)
+                     : cudaErrorInvalidValue;
       } else {
         e = lc::launch_stage1_simt(a, s.num_sms, max_splits, st, &splits);
       }

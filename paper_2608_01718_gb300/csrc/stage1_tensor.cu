@@ -18,6 +18,7 @@
 // Every mbarrier wait is bounded: on a timeout the CTA records LACACHE_ERR_DEVICE_TIMEOUT in the status word, the
 // other roles see an abort flag and stop, in-flight copies and MMAs are drained, TMEM is freed and the CTA exits.
 #include <cuda.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include "internal.cuh"
@@ -36,6 +37,7 @@ constexpr int TMEM_COLS = 2 * BN;           // two accumulators
 constexpr int kThreads = 192;
 constexpr int kEpiWarps = 4;
 constexpr long long kWaitCycles = 2000000000LL;   // about one second of SM clock
+constexpr int kDefaultPrefetch = 0;
 constexpr int kBarriers = 2 * STAGES + 5;          // full, empty, tmem_full x2, tmem_empty x2, drain
 constexpr size_t kStashBytes = 32 * 129 * 4;          // epilogue's rare-path chunk stash
 constexpr size_t kSmemBytes = 1024 + (size_t)STAGES * STAGE_BYTES + kBarriers * 8 + 16 + kStashBytes;
@@ -56,6 +58,8 @@ struct TcParams {
   int units;
   int64_t n_tiles;
   int k_steps;
+  int a_rows;     // rows of the query box: B rounded up to 8 when B <= 128, else 128
+  int prefetch;   // key boxes prefetched into L2 ahead of the ring (0 = off)
   uint64_t* part_cand;
   float* part_best;
   unsigned int* dev_status;
@@ -101,6 +105,12 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
       ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
       : "memory");
+}
+// Bring a box into L2 without a shared-memory destination: raises the bytes in flight beyond the ring.
+__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap* map, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];"
+               ::"l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y)
+               : "memory");
 }
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
@@ -253,6 +263,11 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  // Launched as a programmatic dependent of the previous lookup's stage 2: the set-up above overlaps it, and no
+  // global memory is read or written before the preceding grids have completed. Then let this lookup's stage 2
+  // be scheduled; it waits for this grid's completion before reading anything.
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   auto fail = [&]() {
     *abort_flag = 1u;
@@ -267,8 +282,22 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
         const int qt = u % p.q_tiles, sp = u / p.q_tiles;
         const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
+        // L2 prefetch cursor, p.prefetch key boxes ahead of the loads within this unit's key range
+        int64_t pf_t = t_begin;
+        int pf_ks = 0;
+        auto pf_issue = [&]() {
+          if (pf_t < t_end) {
+            tma_prefetch_l2(&tmap_k, pf_ks * BK, (int)(pf_t * BN));
+            if (++pf_ks == p.k_steps) {
+              pf_ks = 0;
+              ++pf_t;
+            }
+          }
+        };
+        for (int i = 0; i < p.prefetch; ++i) pf_issue();
         for (int64_t t = t_begin; ok && t < t_end; ++t) {
           for (int ks = 0; ks < p.k_steps; ++ks, ++it) {
+            if (p.prefetch) pf_issue();
             const int s = it % STAGES;
             const uint32_t ph = (it / STAGES) & 1u;
             if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) {
@@ -276,7 +305,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               ok = false;
               break;
             }
-            mbar_expect_tx(full_bar(s), STAGE_BYTES);
+            mbar_expect_tx(full_bar(s), (uint32_t)(p.a_rows * BK * 2 + B_BYTES));
             tma_load_2d(a_smem + s * A_BYTES, &tmap_q, full_bar(s), ks * BK, qt * BM);
             tma_load_2d(b_smem + s * B_BYTES, &tmap_k, full_bar(s), ks * BK, (int)(t * BN));
           }
@@ -412,6 +441,18 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
+// Key boxes to prefetch into L2 ahead of the shared-memory ring. LACACHE_TC_PREFETCH overrides the default
+// (a tuning knob; any value gives the same results).
+int prefetch_distance() {
+  static int value = -1;
+  if (value < 0) {
+    const char* env = getenv("LACACHE_TC_PREFETCH");
+    int v = env ? atoi(env) : kDefaultPrefetch;
+    value = v < 0 ? 0 : (v > 64 ? 64 : v);
+  }
+  return value;
+}
+
 int gcd_int(int a, int b) {
   while (b) {
     const int t = a % b;
@@ -426,14 +467,36 @@ cudaError_t launch_cpad(const CUtensorMap* tq, const CUtensorMap* tk, const TcPa
   cudaError_t e = cudaFuncSetAttribute(stage1_tensor_kernel<CPAD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kSmemBytes);
   if (e != cudaSuccess) return e;
-  stage1_tensor_kernel<CPAD><<<grid, kThreads, kSmemBytes, st>>>(*tq, *tk, p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, stage1_tensor_kernel<CPAD>, *tq, *tk, p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+bool encode_rows(EncodeTiledFn encode, CUtensorMap* m, const void* base, int64_t d, int64_t rows,
+                 uint32_t box_rows) {
+  const cuuint64_t dims[2] = {(cuuint64_t)d, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)d * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)BK, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace
 
-cudaError_t launch_stage1_tensor(const Stage1Args& a, const void* tmap_q, const void* tmap_k, int num_sms,
-                                 int max_splits, cudaStream_t st, int* splits) {
+cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int num_sms, int max_splits,
+                                 cudaStream_t st, int* splits) {
   TcParams p;
   p.n = a.n;
   p.d = a.d;
@@ -443,6 +506,15 @@ cudaError_t launch_stage1_tensor(const Stage1Args& a, const void* tmap_q, const 
   p.q_tiles = (a.B + BM - 1) / BM;
   p.n_tiles = (a.n + BN - 1) / BN;
   p.k_steps = (a.d + BK - 1) / BK;
+  p.prefetch = prefetch_distance();
+  // A batch of at most 128 queries is loaded as a box of B rows (rounded up to 8) rather than 128: boxes that
+  // are mostly out of bounds stream measurably slower. The MMA still computes 128 rows; rows past B hold stale
+  // shared memory and their TMEM lanes are never read.
+  p.a_rows = a.B >= BM ? BM : ((a.B + 7) / 8) * 8;
+  CUtensorMap tq, tk;
+  if (!encode_rows(encode, &tq, a.q, a.d, a.B, (uint32_t)p.a_rows) ||
+      !encode_rows(encode, &tk, a.keys, a.d, a.n, (uint32_t)BN))
+    return cudaErrorInvalidValue;
   // splits such that q_tiles * splits is a multiple of the SM count (whole waves of units)
   int s = num_sms / gcd_int(num_sms, p.q_tiles);
   if ((int64_t)s > p.n_tiles) s = (int)p.n_tiles;
@@ -455,12 +527,10 @@ cudaError_t launch_stage1_tensor(const Stage1Args& a, const void* tmap_q, const 
   p.dev_status = a.dev_status;
   *splits = s;
   const int grid = p.units < num_sms ? p.units : num_sms;
-  const CUtensorMap* tq = static_cast<const CUtensorMap*>(tmap_q);
-  const CUtensorMap* tk = static_cast<const CUtensorMap*>(tmap_k);
-  if (a.top_c <= 4) return launch_cpad<4>(tq, tk, p, grid, st);
-  if (a.top_c <= 8) return launch_cpad<8>(tq, tk, p, grid, st);
-  if (a.top_c <= 16) return launch_cpad<16>(tq, tk, p, grid, st);
-  return launch_cpad<32>(tq, tk, p, grid, st);
+  if (a.top_c <= 4) return launch_cpad<4>(&tq, &tk, p, grid, st);
+  if (a.top_c <= 8) return launch_cpad<8>(&tq, &tk, p, grid, st);
+  if (a.top_c <= 16) return launch_cpad<16>(&tq, &tk, p, grid, st);
+  return launch_cpad<32>(&tq, &tk, p, grid, st);
 }
 
 }  // namespace lc

@@ -74,6 +74,12 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
   const int q = blockIdx.x;
   const int C = a.top_c;
 
+  // Launched as a programmatic dependent of stage 1: wait until every preceding grid on the stream has completed
+  // and its writes are visible, before reading anything (a no-op when launched without the attribute).
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // The next lookup's stage 1 may be scheduled now; it too waits for this grid before touching memory.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
   // 1a. best key score over all entries (max over the splits' maxima)
   float best = -INFINITY;
   for (int s = threadIdx.x; s < a.splits; s += kThreads) best = fmaxf(best, a.part_best[(int64_t)s * a.B + q]);
@@ -199,15 +205,34 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
 
 }  // namespace
 
+// Programmatic dependent launch: the grid may be scheduled while stage 1 is still running (its CTAs then sit in
+// griddepcontrol.wait), which hides the launch gap between the two kernels.
+template <int CPAD>
+cudaError_t launch_cpad(const Stage2Args& a, cudaStream_t st) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(a.B);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, stage2_kernel<CPAD>, a);
+}
+
 cudaError_t launch_stage2(const Stage2Args& a, cudaStream_t st) {
+  cudaError_t e;
   if (a.top_c <= 4)
-    stage2_kernel<4><<<a.B, kThreads, 0, st>>>(a);
+    e = launch_cpad<4>(a, st);
   else if (a.top_c <= 8)
-    stage2_kernel<8><<<a.B, kThreads, 0, st>>>(a);
+    e = launch_cpad<8>(a, st);
   else if (a.top_c <= 16)
-    stage2_kernel<16><<<a.B, kThreads, 0, st>>>(a);
+    e = launch_cpad<16>(a, st);
   else
-    stage2_kernel<32><<<a.B, kThreads, 0, st>>>(a);
+    e = launch_cpad<32>(a, st);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -168,3 +168,63 @@ def _compare_candidates(gpu, res, g, b, rep, msg):
             assert pos and abs(o_scores[pos[0]] - gs) <= TOL, f"{msg}: tied candidate {gid} not in oracle order"
     for i in range(ng, c):
         assert gpu["cand_id"][g, i] == -1 and np.isnan(gpu["cand_score"][g, i])
+
+
+class StreamedOracle:
+    """The oracle for caches too large for host memory: the store streams through it chunk by chunk.
+
+    Each generated chunk is inserted into the GPU cache and its key bytes go through the oracle's block-wise key
+    check (A_q is a union over blocks). The prefix rows and ids of the entries stage 2 needs are then regenerated
+    from the generator, never read back from the device.
+    """
+
+    def __init__(self, w: wl.Workload, q: dict, sample, p: oracle.Params):
+        self.w, self.q, self.p = w, q, p
+        self.sample = np.asarray(sample)
+        self.oq = oracle_queries(q, torch.as_tensor(self.sample))
+        self.kc = oracle.KeyCheck(self.oq["emb"], p.tau_c)
+
+    def fill(self, cache: L.LaCache | None, device="cuda") -> None:
+        dtype = L.LACACHE_F32 if self.w.key_dtype == "f32" else L.LACACHE_BF16
+        for ch in wl.iter_store(self.w, device):
+            if cache is not None:
+                cache.insert(ch["key"], ch["prefix"], ch["ids"], dtype)
+            self.kc.add_rows(_bits(ch["key"], self.w.key_dtype == "f32"), ch["j0"])
+            del ch
+        torch.cuda.synchronize()
+
+    def result(self) -> oracle.Result:
+        c = self.p.top_c
+        need = set()
+        for b in range(len(self.sample)):
+            _, j = self.kc.above(b)
+            need.update(int(x) for x in j[:c + 1])
+        ids = np.array(sorted(need), dtype=np.int64)
+        rows = wl.store_rows(self.w, torch.as_tensor(ids), "cuda")
+        f32 = self.w.key_dtype == "f32"
+        pre = _bits(rows["prefix"], f32)
+        tok = rows["ids"].cpu().numpy()
+        where = {int(j): i for i, j in enumerate(ids)}
+        return oracle.decide(self.kc, self.oq["prefix"], self.oq["ids"], self.p,
+                             lambda js: pre[[where[int(j)] for j in js]],
+                             lambda js: tok[[where[int(j)] for j in js]])
+
+    def pair_scores(self, b, j):
+        row = wl.store_rows(self.w, torch.as_tensor([j]), "cuda")
+        f32 = self.w.key_dtype == "f32"
+        kc = oracle.KeyCheck(self.oq["emb"][b:b + 1], -np.inf)
+        kc.add_rows(_bits(row["key"], f32), j)
+        r, m = oracle.lookahead(self.oq["prefix"][b], self.oq["ids"][b], _bits(row["prefix"], f32),
+                                row["ids"].cpu().numpy())
+        return float(kc.best[0]), float(r[0]), int(m[0]), self.w.k
+
+
+def stratified_sample(classes, per_class: int, seed: int = 0):
+    """Query rows to check: up to per_class of each generator class, chosen by a seeded permutation."""
+    rng = np.random.default_rng(seed)
+    cls = np.asarray(classes)
+    rows = []
+    for c in np.unique(cls):
+        idx = np.nonzero(cls == c)[0]
+        rows.extend(rng.permutation(idx)[:per_class].tolist())
+    return np.sort(np.array(rows, dtype=np.int64))

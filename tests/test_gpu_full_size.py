@@ -1,0 +1,130 @@
+"""Parity at the full sizes of the large workloads, in the launch configuration the benchmark uses.
+
+large-16m (70 GB store) and batch-4m (8192 queries) check a stratified sample of queries against the streamed
+oracle. serve-2m runs all 1000 steps: the oracle replays the first steps from its own state, and every step is
+checked for the properties that hold at any size (the append log, bit-exact appended rows, and both checks passing
+for every HIT).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_01718_gb300 import build
+from paper_2608_01718_gb300 import lacache as L
+from paper_2608_01718_gb300 import workloads as wl
+
+from parity import (TOL, StreamedOracle, compare, fill, new_cache, oracle_queries, oracle_store, params,
+                    stratified_sample)
+
+pytestmark = [pytest.mark.gpu, pytest.mark.slow]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def library():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    build.build()
+    L.load()
+
+
+def _check_streamed(w, per_class):
+    q = wl.batch(w, 0, device="cuda")
+    sample = stratified_sample(q["class"], per_class)
+    p = params(w)
+    so = StreamedOracle(w, q, sample, p)
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+        so.fill(cache)
+        assert cache.size == w.n
+        out = cache.lookup(q["emb"], q["prefix"], q["ids"])
+        torch.cuda.synchronize()
+        cache.sync()
+        g = {k: v.cpu().numpy() for k, v in out.items()}
+    res = so.result()
+    rep = compare(g, res, p, rows=sample, pair_scores=so.pair_scores)
+    assert rep.exact + rep.band == len(sample)
+    assert rep.band <= max(1, len(sample) // 50)
+    assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
+    # the generator's labels, as a sanity rate over the whole batch (not parity)
+    cls, tgt = q["class"].numpy(), q["target"].numpy()
+    near = cls == wl.NEAR
+    assert np.mean(g["entry_id"][near] == tgt[near]) >= 0.99
+    assert np.mean(g["status"][cls == wl.COLLISION] == L.LACACHE_REJECT) >= 0.99
+    return rep
+
+
+def test_large_cache_near_hbm_capacity():
+    """16,777,216 entries x 1024 dims (34 GB of keys), B = 128, Zipf(1.1) targets."""
+    _check_streamed(wl.WORKLOADS["large-16m"], per_class=12)
+
+
+def test_large_batch_tensor_core_regime():
+    """4,194,304 entries x 768, B = 8192 (64 query tiles), top_c = 16."""
+    _check_streamed(wl.WORKLOADS["batch-4m"], per_class=60)
+
+
+def test_serve_loop_thousand_steps():
+    """2,097,152 initial entries, 1000 batches of 256, every miss appended (about 2.24M entries at the end)."""
+    w = wl.WORKLOADS["serve-2m"]
+    capacity = w.n + w.steps * w.batch
+    p = params(w)
+    replay = 2
+    st = oracle_store(w)
+    loop = oracle.ServeLoop(w.n + replay * w.batch, w.d, w.k, p)
+    loop.insert(st.key, st.prefix, st.ids)
+    del st
+    origin = {}          # appended entry id -> (step, query index) of the query it holds
+    hits_checked = 0
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR, capacity=capacity) as cache:
+        fill(cache, w)
+        for step in range(w.steps):
+            q = wl.batch(w, step, device="cuda")
+            n_before = cache.size
+            out = cache.lookup(q["emb"], q["prefix"], q["ids"])
+            first, m = cache.append_misses(q["emb"], q["prefix"], q["ids"], out["status"])
+            status = out["status"].cpu().numpy()
+            miss = np.nonzero(status != L.LACACHE_HIT)[0]
+            assert first == n_before and m == len(miss) and cache.size == n_before + m
+            # the appended rows are the non-HIT queries of this step, in query order, bit for bit
+            key = torch.empty((m, w.d), dtype=torch.bfloat16, device="cuda")
+            pre = torch.empty_like(key)
+            ids = torch.empty((m, w.k), dtype=torch.int32, device="cuda")
+            L.lacache_read_rows(cache.h, first, m, key=key, prefix=pre, ids=ids)
+            sel = torch.as_tensor(miss, device="cuda")
+            assert torch.equal(key.view(torch.int16), q["emb"][sel].view(torch.int16))
+            assert torch.equal(pre.view(torch.int16), q["prefix"][sel].view(torch.int16))
+            assert torch.equal(ids, q["ids"][sel])
+            origin.update({first + i: (step, int(qi)) for i, qi in enumerate(miss)})
+            if step < replay:
+                g = {k: v.cpu().numpy() for k, v in out.items()}
+                res, ofirst, om = loop.step(oracle_queries(q))
+                rep = compare(g, res, p)
+                assert rep.band == 0 and (ofirst, om) == (first, m)
+            if step % 97 == 0:
+                hits_checked += _check_hits(w, p, q, out, origin)
+        assert cache.size > w.n + 100 * w.steps
+        assert hits_checked > 100
+
+
+def _check_hits(w, p, q, out, origin):
+    """Every HIT passes both checks against its entry's row, regenerated from the generator."""
+    status = out["status"].cpu().numpy()
+    hit = np.nonzero(status == L.LACACHE_HIT)[0]
+    ent = out["entry_id"].cpu().numpy()[hit]
+    oq = oracle_queries(q, torch.as_tensor(hit))
+    initial = ent < w.n
+    rows_k = np.zeros((len(hit), w.d), np.uint16)
+    rows_p = np.zeros((len(hit), w.d), np.uint16)
+    if initial.any():
+        r = wl.store_rows(w, torch.as_tensor(ent[initial]), "cuda")
+        rows_k[initial], rows_p[initial] = wl.bf16_bits(r["key"]), wl.bf16_bits(r["prefix"])
+    for i in np.nonzero(~initial)[0]:
+        step, qi = origin[int(ent[i])]
+        src = wl.batch(w, step, device="cuda")
+        rows_k[i], rows_p[i] = wl.bf16_bits(src["emb"][qi:qi + 1])[0], wl.bf16_bits(src["prefix"][qi:qi + 1])[0]
+    for i in range(len(hit)):
+        kc = oracle.KeyCheck(oq["emb"][i:i + 1], -np.inf)
+        kc.add_rows(rows_k[i:i + 1], 0)
+        r, _ = oracle.lookahead(oq["prefix"][i], oq["ids"][i], rows_p[i:i + 1], oq["ids"][i:i + 1])
+        assert kc.best[0] >= p.tau_c - TOL and r[0] >= p.tau_a - TOL
+    return len(hit)
