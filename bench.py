@@ -216,6 +216,21 @@ def run_reference(args, w):
     return 0
 
 
+def combine_ranks(elapsed_ms: float, e2e_s: float, world: int, steps: int, e2e_steps: int, batch: int,
+                  device=None) -> dict:
+    """Whole-job numbers from every rank's own timings: the slowest rank's time (all ranks started together after
+    a barrier) and the queries all ranks processed. With one rank no process group is needed."""
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        t = torch.tensor([elapsed_ms, e2e_s], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms, e2e_s = float(t[0]), float(t[1])
+    return {"elapsed_ms": elapsed_ms, "e2e_s": e2e_s,
+            "value": world * steps * batch / (elapsed_ms / 1e3),
+            "e2e_value": world * e2e_steps * batch / e2e_s}
+
+
 def workload_config(w):
     return {"workload": w.name, "entries": w.n, "d": w.d, "k": w.k, "batch": w.batch, "top_c": w.top_c,
             "tau_c": w.tau_c, "tau_a": w.tau_a, "mix_near_random_collision": list(w.mix),
@@ -283,10 +298,6 @@ def run_ours(args, w):
         step(i)
     t1_ms, t2_ms, timed = L.lacache_stage_times(cache.h)
     L.lacache_stage_timing(cache.h, 0)
-    if world > 1:
-        t = torch.tensor([elapsed_ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
 
     # end to end through the host-buffer entry point: H2D of the batch and D2H of the decisions every step
     hq = [{k: batches[i][k].cpu().pin_memory() for k in ("emb", "prefix", "ids")} for i in range(nb)]
@@ -299,10 +310,8 @@ def run_ours(args, w):
     for i in range(args.e2e_steps):
         L.lacache_lookup_host(cache.h, hq[i % nb]["emb"], hq[i % nb]["prefix"], hq[i % nb]["ids"], hout[i % nb])
     e2e_s = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    job = combine_ranks(elapsed_ms, e2e_s, world, args.steps, args.e2e_steps, w.batch, device="cuda")
+    elapsed_ms, e2e_s = job["elapsed_ms"], job["e2e_s"]
     h2d = w.batch * (2 * w.d * 2 + w.k * 4)
     d2h = w.batch * (4 + 1 + 4 + 4 + 4 + 4)
 
@@ -310,7 +319,7 @@ def run_ours(args, w):
     s1_bytes, s2_bytes, flops = algorithmic(w, w.batch)
     t1_avg_s = t1_ms / max(1, timed) / 1e3
     traffic = kernel_traffic(kernel_name, w.name)
-    value = world * args.steps * w.batch / (elapsed_ms / 1e3)
+    value = job["value"]
     # the stage-1 kernel is bound by HBM below the ridge (flops per byte of the measured peaks), else by the
     # tensor pipe; a kernel timed back to back for over a second is compared with the sustained bf16 peak
     ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
@@ -336,7 +345,7 @@ def run_ours(args, w):
                    "peak_tflops": peaks["bf16_tflops"],
                    "frac": flops / (elapsed_ms / args.steps / 1e3) / 1e12 / peaks["bf16_tflops"]},
         "stage_ms": {"stage1": t1_ms / max(1, timed), "stage2": t2_ms / max(1, timed), "timed_lookups": timed},
-        "e2e": {"value": world * args.e2e_steps * w.batch / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d,
+        "e2e": {"value": job["e2e_value"], "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
                 "api": "lacache_lookup_host (pinned host buffers, synchronous)"},
         "gpu_launches": 2 * args.steps,

@@ -160,6 +160,14 @@ lacache_status lacache_last_launch(const lacache_t* h, int32_t* n_splits, int32_
 lacache_status lacache_stage_timing(lacache_t* h, int32_t max_lookups);
 lacache_status lacache_stage_times(lacache_t* h, double* stage1_ms, double* stage2_ms, int64_t* lookups);
 
+/* Test support for failure detection. The next `lookups` lookups that run the tensor-core stage 1 make its first
+ * CTA withhold one of its TMA loads: nothing is copied and nothing arrives on that pipeline stage, so the MMA
+ * issuer's bounded wait (about one second) runs out. The kernel then records LACACHE_ERR_DEVICE_TIMEOUT, its other
+ * roles stop, its issued copies and MMAs drain, TMEM is freed and it exits. The context stays usable: the next
+ * lacache_sync reports the timeout and later lookups run normally. The affected lookup's outputs are undefined.
+ * 0 cancels. */
+lacache_status lacache_inject_stall(lacache_t* h, int32_t lookups);
+
 /* Lookup that allocates nothing, for callers that cannot allocate device memory. Examples: a serving runtime or
  * framework whose allocator owns all device memory, code that must not trigger the device synchronization that
  * cudaMalloc and cudaFree can cause, and plug-ins with a fixed memory budget. The paper has no counterpart; this

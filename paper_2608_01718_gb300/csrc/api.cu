@@ -29,6 +29,7 @@ struct lacache {
   int last_splits;
   int last_kernel;
   lc::EncodeTiledFn encode;
+  int inject_stall;          // lookups left that withhold one stage-1 load (failure-detection tests)
   cudaEvent_t* events;       // [3 x event_cap] stage-timing events, or NULL
   int event_cap;
   int event_used;
@@ -185,7 +186,7 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
   if (h->events && h->event_used < h->event_cap) ev = h->events + 3 * h->event_used++;
   if (ev && cudaEventRecord(ev[0], st) != cudaSuccess) return LACACHE_ERR_CUDA;
   if (h->n > 0) {
-    Stage1Args a;
+    Stage1Args a{};
     a.keys = h->key;
     a.n = h->n;
     a.d = c.d;
@@ -197,6 +198,10 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
     a.part_best = h->part_best;
     a.dev_status = h->dev_status;
     kernel = c.stage1 == LACACHE_STAGE1_AUTO ? LACACHE_STAGE1_TENSOR : c.stage1;
+    if (h->inject_stall > 0 && kernel == LACACHE_STAGE1_TENSOR) {
+      a.inject_stall = 1;
+      --h->inject_stall;
+    }
     cudaError_t e;
     if (kernel == LACACHE_STAGE1_TENSOR) {
       if (!h->encode) return LACACHE_ERR_CUDA;
@@ -505,6 +510,12 @@ lacache_status lacache_stage_times(lacache_t* h, double* stage1_ms, double* stag
   if (stage1_ms) *stage1_ms = t1;
   if (stage2_ms) *stage2_ms = t2;
   if (lookups) *lookups = used;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_inject_stall(lacache_t* h, int32_t lookups) {
+  if (!h || lookups < 0) return LACACHE_ERR_INVALID_ARG;
+  h->inject_stall = lookups;
   return LACACHE_OK;
 }
 

@@ -63,6 +63,7 @@ struct Stage1Args {
   uint64_t* part_cand;
   float* part_best;
   unsigned int* dev_status;
+  int inject_stall;           // test support: CTA 0 of the tensor kernel withholds one load (see lacache.h)
 };
 
 struct Stage2Args {

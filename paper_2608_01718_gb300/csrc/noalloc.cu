@@ -114,7 +114,7 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
 
     int splits = 0;
     if (result == LACACHE_OK && n > 0) {
-      lc::Stage1Args a;
+      lc::Stage1Args a{};
       a.keys = reinterpret_cast<const __nv_bfloat16*>(key_dev);
       a.n = n;
       a.d = c.d;

@@ -60,6 +60,7 @@ struct TcParams {
   int k_steps;
   int a_rows;     // rows of the query box: B rounded up to 8 when B <= 128, else 128
   int prefetch;   // key boxes prefetched into L2 ahead of the ring (0 = off)
+  int inject_stall;  // test support: CTA 0 withholds its second load, so its MMA issuer's bounded wait runs out
   uint64_t* part_cand;
   float* part_best;
   unsigned int* dev_status;
@@ -279,6 +280,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---------------- TMA producer ----------------
       uint32_t it = 0;
       bool ok = true;
+      const uint32_t withheld = (p.inject_stall && blockIdx.x == 0) ? 1u : 0xFFFFFFFFu;
       for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
         const int qt = u % p.q_tiles, sp = u / p.q_tiles;
         const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
@@ -305,6 +307,7 @@ __global__ void __launch_bounds__(kThreads, 1)
               ok = false;
               break;
             }
+            if (it == withheld) continue;   // nothing arrives on this stage: its consumer's wait runs out
             mbar_expect_tx(full_bar(s), (uint32_t)(p.a_rows * BK * 2 + B_BYTES));
             tma_load_2d(a_smem + s * A_BYTES, &tmap_q, full_bar(s), ks * BK, qt * BM);
             tma_load_2d(b_smem + s * B_BYTES, &tmap_k, full_bar(s), ks * BK, (int)(t * BN));
@@ -314,7 +317,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       // drain: the last load issued into each stage has landed before the CTA may exit
       const uint32_t first = it > (uint32_t)STAGES ? it - STAGES : 0u;
       for (uint32_t i = first; i < it; ++i)
-        if (!mbar_wait(full_bar(i % STAGES), (i / STAGES) & 1u, nullptr)) fail();
+        if (i != withheld && !mbar_wait(full_bar(i % STAGES), (i / STAGES) & 1u, nullptr)) fail();
     }
   } else if (warp == 1) {
     if (lane == 0) {
@@ -525,6 +528,7 @@ cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int 
   p.part_cand = a.part_cand;
   p.part_best = a.part_best;
   p.dev_status = a.dev_status;
+  p.inject_stall = a.inject_stall;
   *splits = s;
   const int grid = p.units < num_sms ? p.units : num_sms;
   if (a.top_c <= 4) return launch_cpad<4>(&tq, &tk, p, grid, st);

@@ -20,7 +20,8 @@ LACACHE_MISS_KEY, LACACHE_HIT, LACACHE_REJECT = 0, 1, 2
 
 EXPORTS = ["lacache_create", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
            "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
-           "lacache_stage_timing", "lacache_stage_times", "lacache_lookup_noalloc", "lacache_status_string"]
+           "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_lookup_noalloc",
+           "lacache_status_string"]
 
 
 class lacache_config(ctypes.Structure):
@@ -70,6 +71,7 @@ def load() -> ctypes.CDLL:
         "lacache_last_launch": ([vp, p32, p32], i32),
         "lacache_stage_timing": ([vp, i32], i32),
         "lacache_stage_times": ([vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double), p64], i32),
+        "lacache_inject_stall": ([vp, i32], i32),
         "lacache_lookup_noalloc": ([ctypes.POINTER(lacache_config), i64, vp, vp, vp, i32, vp, vp, vp,
                                     ctypes.POINTER(lacache_result), vp], i32),
         "lacache_status_string": ([i32], ctypes.c_char_p),
@@ -188,6 +190,10 @@ def lacache_stage_times(h: int) -> tuple[float, float, int]:
     t1, t2, n = ctypes.c_double(), ctypes.c_double(), ctypes.c_int64()
     _check("lacache_stage_times", load().lacache_stage_times(h, ctypes.byref(t1), ctypes.byref(t2), ctypes.byref(n)))
     return t1.value, t2.value, n.value
+
+
+def lacache_inject_stall(h: int, lookups: int) -> None:
+    _check("lacache_inject_stall", load().lacache_inject_stall(h, lookups))
 
 
 def lacache_lookup_noalloc(cfg: lacache_config, key, prefix, ids, q_emb, q_prefix, q_ids, out: dict,

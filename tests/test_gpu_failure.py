@@ -1,0 +1,44 @@
+"""Failure detection on the GPU without a fault: a stage-1 wait that runs out is reported, not hung.
+
+lacache_inject_stall makes the tensor kernel's first CTA withhold one TMA load (no copy is issued). The MMA
+issuer's bounded wait then runs out (about a second). The kernel records the timeout in the status word, drains
+and exits, and lacache_sync reports LACACHE_ERR_DEVICE_TIMEOUT. The context must stay usable: the next lookup
+matches the one taken before the injection.
+"""
+import pytest
+import torch
+
+from paper_2608_01718_gb300 import build
+from paper_2608_01718_gb300 import lacache as L
+from paper_2608_01718_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def library():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    build.build()
+    L.load()
+
+
+def test_stage1_wait_timeout_is_reported_and_the_context_stays_usable():
+    w = wl.WORKLOADS["mid-1m"].scaled(n=40_000)
+    with L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch,
+                   stage1=L.LACACHE_STAGE1_TENSOR) as cache:
+        for ch in wl.iter_store(w, "cuda"):
+            cache.insert(ch["key"], ch["prefix"], ch["ids"])
+        q = wl.batch(w, 0, device="cuda")
+        before = {k: v.clone() for k, v in cache.lookup(q["emb"], q["prefix"], q["ids"]).items()}
+        cache.sync()
+        L.lacache_inject_stall(cache.h, 1)
+        cache.lookup(q["emb"], q["prefix"], q["ids"])
+        with pytest.raises(L.LacacheError) as e:
+            cache.sync()
+        assert e.value.status == L.LACACHE_ERR_DEVICE_TIMEOUT
+        cache.sync()                                   # the status word was cleared
+        after = cache.lookup(q["emb"], q["prefix"], q["ids"])
+        cache.sync()
+        for k in ("status", "entry_id", "cand_id", "n_cand"):
+            assert torch.equal(after[k], before[k]), k
