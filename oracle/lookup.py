@@ -46,6 +46,22 @@ class Params:
     top_c: int
     check_mode: int = CHECK_EMB
     token_match_min: int | None = None     # None: all k ids must match
+    # Ensemble of m lookahead checks (section 3.4, "Analysis"): the prefix row holds one embedding per model,
+    # segments of these dimensions, each with its own threshold. None: a single check with tau_a over the row.
+    prefix_dims: tuple | None = None
+    tau_a_models: tuple | None = None
+
+    def segments(self, row_len: int):
+        """(start, end, threshold) of each lookahead check over a prefix row of row_len values."""
+        if self.prefix_dims is None:
+            return [(0, row_len, self.tau_a)]
+        out, start = [], 0
+        for dim, tau in zip(self.prefix_dims, self.tau_a_models):
+            out.append((start, start + dim, tau))
+            start += dim
+        if start != row_len:
+            raise ValueError(f"prefix dims {self.prefix_dims} do not add up to the row length {row_len}")
+        return out
 
 
 @dataclasses.dataclass
@@ -81,6 +97,7 @@ class Result:
     cand_score: np.ndarray        # f64 [B, c]; s, NaN padded
     cand_prefix_score: np.ndarray  # f64 [B, c]; r, NaN padded
     cand_matches: np.ndarray      # int32 [B, c]; m, -1 padded
+    prefix_scores: np.ndarray     # f64 [B, models]; every model's r for the candidate of prefix_score
     margin: np.ndarray            # f64 [B]; decision margin: smallest score change altering status/entry_id
     list_margin: np.ndarray       # f64 [B]; smallest score change altering C_q or its order
     literal_margin: np.ndarray    # f64 [B]; min(|max_j s - tau_c|, s_(1) - s_(2))
@@ -131,20 +148,31 @@ class KeyCheck:
         return s[order], j[order]
 
 
-def lookahead(p_bits, t_ids, cand_prefix_bits, cand_ids):
+def lookahead(p_bits, t_ids, cand_prefix_bits, cand_ids, segments=None):
     """Stage 2 for one query against the prefix rows of its candidates.
 
-    r_j = <p, P_j>, the cosine similarity sim(f_k(x), f_k(x')) of the two prefix embeddings.
+    r_j = <p, P_j>, the cosine similarity sim(f_k(x), f_k(x')) of the two prefix embeddings; with an ensemble,
+    one such similarity per model over that model's segment of the row (columns of r).
     m_j = #{i < k : t_i = T_ji}, the positions where the two k-token prefixes carry the same token id.
     """
-    r = widen(cand_prefix_bits) @ widen(p_bits)
+    P = widen(cand_prefix_bits)
+    p = widen(p_bits)
+    if segments is None:
+        r = P @ p
+    else:
+        r = np.stack([P[:, a:b] @ p[a:b] for a, b, _ in segments], axis=1)
     m = (np.asarray(cand_ids, dtype=np.int64) == np.asarray(t_ids, dtype=np.int64)[None, :]).sum(axis=1)
     return r, m
 
 
-def passes(r, m, params: Params, k: int):
+def passes(r, m, params: Params, k: int, segments=None):
+    """Pass bits of the candidates. With an ensemble, the lookahead check passes only if every model's
+    similarity clears that model's threshold (section 3.4: all m checks must hold)."""
     tmin = k if params.token_match_min is None else params.token_match_min
-    emb_ok = r >= params.tau_a
+    if segments is None:
+        emb_ok = r >= params.tau_a
+    else:
+        emb_ok = np.all(r >= np.array([t for _, _, t in segments])[None, :], axis=1)
     tok_ok = m >= tmin
     if params.check_mode == CHECK_EMB:
         return emb_ok
@@ -161,6 +189,8 @@ def decide(kc: KeyCheck, q_prefix_bits, q_ids, params: Params,
     q_ids = np.asarray(q_ids, dtype=np.int32)
     B = kc.q.shape[0]
     k = q_ids.shape[1]
+    segs = params.segments(np.asarray(q_prefix_bits).shape[1]) if params.prefix_dims is not None else None
+    n_models = len(segs) if segs else 1
     c = params.top_c
     tau_c, tau_a = params.tau_c, params.tau_a
     uses_r = params.check_mode in (CHECK_EMB, CHECK_BOTH)
@@ -173,6 +203,7 @@ def decide(kc: KeyCheck, q_prefix_bits, q_ids, params: Params,
         n_cand=np.zeros(B, np.int32), n_above=np.zeros(B, np.int64),
         cand_id=np.full((B, c), -1, np.int32), cand_score=np.full((B, c), np.nan),
         cand_prefix_score=np.full((B, c), np.nan), cand_matches=np.full((B, c), -1, np.int32),
+        prefix_scores=np.full((B, n_models), np.nan),
         margin=np.full(B, np.inf), list_margin=np.full(B, np.inf), literal_margin=np.full(B, np.inf),
         next_id=np.full(B, -1, np.int32), next_score=np.full(B, np.nan))
 
@@ -187,36 +218,39 @@ def decide(kc: KeyCheck, q_prefix_bits, q_ids, params: Params,
         res.cand_score[b, :nc] = cs
         served = None
         if nc:
-            r, m = lookahead(q_prefix_bits[b], q_ids[b], prefix_rows(cj), id_rows(cj))
-            ok = passes(r, m, params, k)
+            rr, m = lookahead(q_prefix_bits[b], q_ids[b], prefix_rows(cj), id_rows(cj), segs)
+            ok = passes(rr, m, params, k, segs)
+            rm = rr if segs else rr[:, None]          # [nc, models]
+            r = rm[:, 0]                              # model 0: the reported prefix score
             res.cand_prefix_score[b, :nc] = r
             res.cand_matches[b, :nc] = m
             hits = np.nonzero(ok)[0]
+            shown = int(hits[0]) if hits.size else 0
             if hits.size:
                 served = int(hits[0])
                 res.status[b] = HIT
                 res.entry_id[b] = cj[served]
                 res.key_score[b] = cs[served]
-                res.prefix_score[b] = r[served]
-                res.token_matches[b] = m[served]
             else:
                 res.status[b] = REJECT
-                res.prefix_score[b] = r[0]
-                res.token_matches[b] = m[0]
+            res.prefix_score[b] = r[shown]
+            res.prefix_scores[b] = rm[shown]
+            res.token_matches[b] = m[shown]
         next_ok = False
         if n_above > c:
             # the best entry just outside C_q: only needed to know whether the cut can change the decision
             jn = j_sorted[c:c + 1]
-            rn, mn = lookahead(q_prefix_bits[b], q_ids[b], prefix_rows(jn), id_rows(jn))
-            next_ok = bool(passes(rn, mn, params, k)[0])
+            rn, mn = lookahead(q_prefix_bits[b], q_ids[b], prefix_rows(jn), id_rows(jn), segs)
+            next_ok = bool(passes(rn, mn, params, k, segs)[0])
             res.next_id[b], res.next_score[b] = jn[0], s_sorted[c]
 
         # decision margin: the smallest score change that alters status or entry_id
         gaps = []
         if nc:
+            taus = [t for _, _, t in segs] if segs else [tau_a]
             for i in range((served if served is not None else nc - 1) + 1):   # candidates examined
                 if uses_r and (not uses_m or m[i] >= tmin):
-                    gaps.append(abs(r[i] - tau_a))
+                    gaps.append(min(abs(rm[i, h] - taus[h]) for h in range(len(taus))))
         if served is not None:
             gaps.append(cs[served] - tau_c)                         # j* falls out of A_q
             if served == c - 1 and n_above > c:

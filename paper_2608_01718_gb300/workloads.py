@@ -13,11 +13,15 @@ used here. The recipe:
   ``cluster_sigma`` (per-component std ``cluster_sigma / sqrt(d)``); prefix embedding = an independent uniform unit
   vector; prefix ids uniform over the vocabulary;
 * queries, shuffled within the batch:
-  - near-duplicate (benign paraphrase): normalise(key_t + noise of norm ``near_sigma``), carrying entry t's exact
-    prefix embedding and ids (same greedy response prefix);
+  - near-duplicate (benign paraphrase): normalise(key_t + noise of norm ``near_sigma``), carrying entry t's
+    prefix embedding (exact, or plus noise of norm ``near_prefix_sigma`` per model) and its ids (same greedy
+    response prefix);
   - random: a uniform unit vector with a fresh prefix;
   - collision (the threat model's key collision): normalise(key_t + noise of norm ``coll_sigma``) with a fresh
     prefix embedding and fresh ids (a semantically distinct response);
+  - mimic (ensemble workloads only): a collision whose response prefix is close to the victim's under the first
+    embedding model and fresh under the others (the in-context attack whose prefix partly aligns, Figure 6);
+* ensemble workloads hold one prefix embedding per model, concatenated in the prefix row, each a unit vector;
 * targets t are uniform over the entries present at generation time, or Zipf(s) over a seeded permutation of them.
 
 Noise is read as a vector whose expected norm is sigma. Read per component instead, a near-duplicate at d=384 and
@@ -35,8 +39,8 @@ from typing import Iterator
 
 import torch
 
-NEAR, RANDOM, COLLISION = 0, 1, 2
-CLASS_NAMES = {NEAR: "near-duplicate", RANDOM: "random", COLLISION: "collision"}
+NEAR, RANDOM, COLLISION, MIMIC = 0, 1, 2, 3
+CLASS_NAMES = {NEAR: "near-duplicate", RANDOM: "random", COLLISION: "collision", MIMIC: "mimic"}
 
 # rows per generated store chunk; fixed so that chunk i is always the same rows
 CHUNK_ROWS = 1 << 18
@@ -62,13 +66,27 @@ class Workload:
     zipf: float | None = None   # Zipf exponent over targets, None = uniform
     steps: int = 1              # serve-loop steps (batches); 1 = a single lookup
     seed: int = 20260801
+    # Ensemble of m lookahead checks: one prefix embedding per model (these dimensions, concatenated in the
+    # prefix row), each with its own threshold. None: one prefix embedding of dimension d checked with tau_a.
+    prefix_dims: tuple | None = None
+    tau_a_models: tuple | None = None
+    near_prefix_sigma: float = 0.0   # noise norm on a near-duplicate's prefix embeddings (0: exact copies)
 
     def scaled(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)
 
     @property
+    def dims(self) -> tuple:
+        return self.prefix_dims if self.prefix_dims is not None else (self.d,)
+
+    @property
+    def pd(self) -> int:
+        """Length of a prefix row (all models' embeddings)."""
+        return sum(self.dims)
+
+    @property
     def store_bytes(self) -> int:
-        return self.n * (4 * self.d + 4 * self.k)
+        return self.n * (2 * self.d + 2 * self.pd + 4 * self.k)
 
 
 WORKLOADS = {
@@ -87,6 +105,12 @@ WORKLOADS = {
     # Streaming serve loop: 1000 batches, every miss appended.
     "serve-2m": Workload("serve-2m", n=1 << 21, d=768, k=32, vocab=128256, clusters=4096, batch=256,
                          mix=(0.45, 0.35, 0.2), tau_c=0.90, tau_a=0.80, top_c=8, steps=1000),
+    # Ensemble of three lookahead checks (BGE-large, MiniLM and MPNet dimensions), with prefix-mimicking
+    # collisions that only the ensemble rejects.
+    "ensemble-1m": Workload("ensemble-1m", n=1 << 20, d=768, k=16, vocab=128256, clusters=4096, batch=32,
+                            mix=(0.45, 0.25, 0.15, 0.15), tau_c=0.90, tau_a=0.70, top_c=8,
+                            prefix_dims=(1024, 384, 768), tau_a_models=(0.70, 0.70, 0.70),
+                            near_prefix_sigma=0.3),
 }
 
 
@@ -103,6 +127,11 @@ def _gen(w: Workload, tag: str, index: int, device) -> torch.Generator:
 
 def _unit(x: torch.Tensor) -> torch.Tensor:
     return x / x.norm(dim=1, keepdim=True)
+
+
+def _unit_segments(x: torch.Tensor, dims: tuple) -> torch.Tensor:
+    """Normalise each model's segment of a prefix row separately."""
+    return torch.cat([_unit(part) for part in torch.split(x, list(dims), dim=1)], dim=1)
 
 
 def centres(w: Workload, device="cpu") -> torch.Tensor:
@@ -127,7 +156,7 @@ def store_chunk(w: Workload, index: int, device="cpu", cent: torch.Tensor | None
     noise = torch.randn((rows, w.d), generator=g, device=device) * (w.cluster_sigma / math.sqrt(w.d))
     key = _unit(cent[cluster] + noise)
     del noise
-    prefix = _unit(torch.randn((rows, w.d), generator=g, device=device))
+    prefix = _unit_segments(torch.randn((rows, w.pd), generator=g, device=device), w.dims)
     ids = torch.randint(0, w.vocab, (rows, w.k), generator=g, device=device, dtype=torch.int32)
     dt = _emb_dtype(w)
     return {"j0": j0, "key": key.to(dt), "prefix": prefix.to(dt), "ids": ids, "cluster": cluster}
@@ -143,7 +172,7 @@ def store_rows(w: Workload, rows: torch.Tensor, device="cpu") -> dict:
     """Regenerate selected rows of the initial store (chunk by chunk)."""
     rows = rows.to("cpu", torch.int64)
     out_key = torch.empty((len(rows), w.d), dtype=_emb_dtype(w), device=device)
-    out_pre = torch.empty((len(rows), w.d), dtype=_emb_dtype(w), device=device)
+    out_pre = torch.empty((len(rows), w.pd), dtype=_emb_dtype(w), device=device)
     out_ids = torch.empty((len(rows), w.k), dtype=torch.int32, device=device)
     if len(rows) == 0:
         return {"key": out_key, "prefix": out_pre, "ids": out_ids}
@@ -161,10 +190,12 @@ def store_rows(w: Workload, rows: torch.Tensor, device="cpu") -> dict:
 
 
 def class_counts(w: Workload) -> tuple:
-    near = int(round(w.batch * w.mix[0]))
-    coll = int(round(w.batch * w.mix[2]))
-    near = min(near, w.batch)
-    coll = min(coll, w.batch - near)
+    """(near-duplicate, random, collision[, mimic]) query counts of a batch."""
+    near = min(int(round(w.batch * w.mix[0])), w.batch)
+    coll = min(int(round(w.batch * w.mix[2])), w.batch - near)
+    if len(w.mix) > 3:
+        mimic = min(int(round(w.batch * w.mix[3])), w.batch - near - coll)
+        return near, w.batch - near - coll - mimic, coll, mimic
     return near, w.batch - near - coll, coll
 
 
@@ -172,8 +203,11 @@ def query_plan(w: Workload, step: int = 0, n_entries: int | None = None) -> dict
     """Class and target entry of every query of batch ``step`` (drawn on the CPU: small)."""
     n_entries = w.n if n_entries is None else n_entries
     g = _gen(w, "plan", step, "cpu")
-    near, rand, coll = class_counts(w)
-    classes = torch.tensor([NEAR] * near + [RANDOM] * rand + [COLLISION] * coll, dtype=torch.int64)
+    counts = class_counts(w)
+    near, rand, coll = counts[:3]
+    mimic = counts[3] if len(counts) > 3 else 0
+    classes = torch.tensor([NEAR] * near + [RANDOM] * rand + [COLLISION] * coll + [MIMIC] * mimic,
+                           dtype=torch.int64)
     classes = classes[torch.randperm(w.batch, generator=g)]
     if w.zipf is None:
         target = torch.randint(0, max(n_entries, 1), (w.batch,), generator=g)
@@ -204,13 +238,24 @@ def make_queries(w: Workload, plan: dict, step: int = 0, device="cpu", target_ro
     base = target_rows["key"].to(torch.float32)
     noise = torch.randn((B, w.d), generator=g, device=device)
     rnd = torch.randn((B, w.d), generator=g, device=device)
-    fresh_pre = _unit(torch.randn((B, w.d), generator=g, device=device)).to(torch.bfloat16)
+    fresh_pre = _unit_segments(torch.randn((B, w.pd), generator=g, device=device), w.dims).to(torch.bfloat16)
     fresh_ids = torch.randint(0, w.vocab, (B, w.k), generator=g, device=device, dtype=torch.int32)
     scale = torch.where(cls == NEAR, w.near_sigma, w.coll_sigma).to(torch.float32)[:, None] / math.sqrt(w.d)
     q = torch.where((cls == RANDOM)[:, None], rnd, base + noise * scale)
     q = _unit(q).to(torch.bfloat16)
     near = (cls == NEAR)[:, None]
-    pre = torch.where(near, target_rows["prefix"].to(torch.bfloat16), fresh_pre)
+    tpre = target_rows["prefix"].to(torch.float32)
+    if w.near_prefix_sigma > 0:
+        # a paraphrase's response prefix: the target's prefix embeddings plus noise of the given norm per model
+        pn = torch.randn((B, w.pd), generator=g, device=device)
+        seg_scale = torch.cat([torch.full((dim,), w.near_prefix_sigma / math.sqrt(dim), device=device)
+                               for dim in w.dims])
+        tpre = _unit_segments(tpre + pn * seg_scale, w.dims)
+    pre = torch.where(near, tpre.to(torch.bfloat16), fresh_pre)
+    # a prefix-mimicking collision: close to the victim's response prefix under the first model only
+    d0 = w.dims[0]
+    mimic = (cls == MIMIC)[:, None]
+    pre[:, :d0] = torch.where(mimic, tpre[:, :d0].to(torch.bfloat16), pre[:, :d0])
     ids = torch.where(near, target_rows["ids"], fresh_ids)
     return {"emb": q.contiguous(), "prefix": pre.contiguous(), "ids": ids.contiguous(),
             "class": plan["class"].clone(), "target": plan["target"].clone()}

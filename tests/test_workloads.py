@@ -60,3 +60,23 @@ def test_labels_predict_oracle_decisions_on_tiny_cache():
     # every near-duplicate and collision has a full candidate list (the target's cluster clears tau_c)
     assert np.all(res.n_cand[near | coll] == w.top_c)
     assert np.min(res.margin) > 2e-3
+
+
+def test_ensemble_workload_labels_predict_oracle_decisions():
+    """Sanity rate on a small ensemble cache: with all three checks, near-duplicates hit and both kinds of
+    collision are rejected; with the first check alone the prefix-mimicking collisions get through."""
+    w = wl.WORKLOADS["ensemble-1m"].scaled(n=4096, clusters=64, batch=64)
+    st = _store_bits(w)
+    q = wl.batch(w, 0)
+    oq = {"emb": wl.bf16_bits(q["emb"]), "prefix": wl.bf16_bits(q["prefix"]), "ids": q["ids"].numpy()}
+    cls, tgt = q["class"].numpy(), q["target"].numpy()
+    ens = oracle.lookup(st, oq, oracle.Params(w.tau_c, 0.0, w.top_c, prefix_dims=w.prefix_dims,
+                                              tau_a_models=w.tau_a_models))
+    near, mimic, coll = cls == wl.NEAR, cls == wl.MIMIC, cls == wl.COLLISION
+    assert mimic.sum() > 0
+    assert np.all(ens.status[near] == oracle.HIT) and np.all(ens.entry_id[near] == tgt[near])
+    assert np.all(ens.status[mimic | coll] == oracle.REJECT)
+    first = oracle.lookup(st, oq, oracle.Params(w.tau_c, 0.0, w.top_c, prefix_dims=w.prefix_dims,
+                                                tau_a_models=(w.tau_a_models[0], -2.0, -2.0)))
+    assert np.all(first.status[mimic] == oracle.HIT)
+    assert np.all(ens.prefix_scores[near, 0] > 0.9) and ens.prefix_scores.shape == (w.batch, 3)
