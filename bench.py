@@ -108,8 +108,8 @@ class ClockSampler:
 def algorithmic(w, batch):
     """Bytes and flops the method must move / do per lookup (keys read once, c candidate rows gathered)."""
     stage1_bytes = w.n * w.d * 2 + batch * w.d * 2
-    stage2_bytes = batch * w.top_c * (2 * w.d + 4 * w.k) + batch * (2 * w.d + 4 * w.k)
-    flops = 2 * batch * w.n * w.d + 2 * batch * w.top_c * w.d
+    stage2_bytes = batch * w.top_c * (2 * w.pd + 4 * w.k) + batch * (2 * w.pd + 4 * w.k)
+    flops = 2 * batch * w.n * w.d + 2 * batch * w.top_c * w.pd
     return stage1_bytes, stage2_bytes, flops
 
 
@@ -173,7 +173,7 @@ def oracle_sample(w, rows: int, offset: int = 0, device="cpu"):
 def time_oracle(store, oq, w) -> float:
     """Seconds the oracle takes to look up the whole batch against the given store rows."""
     import oracle
-    p = oracle.Params(w.tau_c, w.tau_a, w.top_c)
+    p = oracle.Params(w.tau_c, w.tau_a, w.top_c, prefix_dims=w.prefix_dims, tau_a_models=w.tau_a_models)
     t0 = time.perf_counter()
     oracle.lookup(store, oq, p)
     return time.perf_counter() - t0
@@ -232,10 +232,15 @@ def combine_ranks(elapsed_ms: float, e2e_s: float, world: int, steps: int, e2e_s
 
 
 def workload_config(w):
-    return {"workload": w.name, "entries": w.n, "d": w.d, "k": w.k, "batch": w.batch, "top_c": w.top_c,
-            "tau_c": w.tau_c, "tau_a": w.tau_a, "mix_near_random_collision": list(w.mix),
-            "store_bytes": w.store_bytes,
-            "l2": f"no flush: the keys read per step ({w.n * w.d * 2 / 1e9:.2f} GB) exceed the 129 MB L2"}
+    cfg = {"workload": w.name, "entries": w.n, "d": w.d, "k": w.k, "batch": w.batch, "top_c": w.top_c,
+           "tau_c": w.tau_c, "tau_a": w.tau_a, "store_bytes": w.store_bytes}
+    if w.prefix_dims is None:
+        cfg["mix_near_random_collision"] = list(w.mix)
+    else:
+        cfg |= {"prefix_dims": list(w.prefix_dims), "tau_a_models": list(w.tau_a_models),
+                "mix_near_random_collision_mimic": list(w.mix)}
+    cfg["l2"] = f"no flush: the keys read per step ({w.n * w.d * 2 / 1e9:.2f} GB) exceed the 129 MB L2"
+    return cfg
 
 
 def run_ours(args, w):
@@ -253,7 +258,7 @@ def run_ours(args, w):
     build.build()
     stage1 = {"auto": L.LACACHE_STAGE1_AUTO, "tensor": L.LACACHE_STAGE1_TENSOR, "simt": L.LACACHE_STAGE1_SIMT}
     cache = L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch, device=local_rank,
-                      stage1=stage1[args.stage1])
+                      stage1=stage1[args.stage1], prefix_dims=w.prefix_dims, tau_a_models=w.tau_a_models)
     dtype = L.LACACHE_F32 if w.key_dtype == "f32" else L.LACACHE_BF16
     for ch in wl.iter_store(w, "cuda"):
         cache.insert(ch["key"], ch["prefix"], ch["ids"], dtype)
@@ -312,7 +317,7 @@ def run_ours(args, w):
     e2e_s = time.perf_counter() - t0
     job = combine_ranks(elapsed_ms, e2e_s, world, args.steps, args.e2e_steps, w.batch, device="cuda")
     elapsed_ms, e2e_s = job["elapsed_ms"], job["e2e_s"]
-    h2d = w.batch * (2 * w.d * 2 + w.k * 4)
+    h2d = w.batch * (2 * w.d + 2 * w.pd + w.k * 4)
     d2h = w.batch * (4 + 1 + 4 + 4 + 4 + 4)
 
     peaks, peak_src = load_peaks()

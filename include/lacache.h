@@ -63,6 +63,16 @@ typedef enum {
   LACACHE_STAGE1_SIMT = 2    /* CUDA-core FFMA scan */
 } lacache_stage1;
 
+/* Ensemble of m lookahead checks (section 3.4, "Analysis"; Figure 6): every entry and query carries one k-token
+ * prefix embedding per embedding model, concatenated in one prefix row of dims[0] + ... + dims[m-1] values, and a
+ * candidate passes the lookahead check only if sim_i(f_k(x), f_k(x')) >= tau_a[i] for every model i. */
+#define LACACHE_MAX_MODELS 8
+typedef struct {
+  int32_t m;                         /* number of lookahead checks, 1..LACACHE_MAX_MODELS */
+  int32_t dims[LACACHE_MAX_MODELS];  /* each model's prefix embedding dimension (multiple of 8) */
+  float tau_a[LACACHE_MAX_MODELS];   /* each model's lookahead threshold */
+} lacache_ensemble;
+
 /* Per-query status codes written to lacache_result.status. */
 enum { LACACHE_MISS_KEY = 0, LACACHE_HIT = 1, LACACHE_REJECT = 2 };
 
@@ -96,6 +106,8 @@ typedef struct {
   float* cand_score;          /* optional [B x top_c]: their key scores, NaN padded */
   float* cand_prefix_score;   /* optional [B x top_c]: their lookahead scores, NaN padded */
   int32_t* cand_matches;      /* optional [B x top_c]: their token matches, -1 padded */
+  float* prefix_scores;       /* optional [B x m]: every model's lookahead score for the candidate of prefix_score
+                                 (prefix_score is model 0's); NaN on MISS_KEY */
 } lacache_result;
 
 /* Create a cache on cfg->device with an empty store of cfg->capacity entries. Allocates the store
@@ -103,18 +115,23 @@ typedef struct {
  * On success *out is a new handle; on failure *out is NULL and nothing stays allocated. */
 lacache_status lacache_create(const lacache_config* cfg, lacache_t** out);
 
+/* lacache_create for an ensemble of lookahead checks. cfg->tau_a is ignored; prefix rows everywhere (insert,
+ * lookup, append, read_rows) are dims[0] + ... + dims[m-1] values long. lacache_create(cfg) is this call with
+ * m = 1, dims = {cfg->d}, tau_a = {cfg->tau_a}. */
+lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_ensemble* ens, lacache_t** out);
+
 /* Free the handle and everything it owns. Synchronizes the device first. NULL is accepted. */
 lacache_status lacache_destroy(lacache_t* h);
 
-/* Append n entries (Algorithm 1, "add <h(x), [h(f_k(x)), f(x)]> to cache"). key_dev and prefix_dev are
- * [n x d] in `dtype` (LACACHE_F32 rows are rounded to bf16, to nearest even, on the device); ids_dev is
+/* Append n entries (Algorithm 1, "add <h(x), [h(f_k(x)), f(x)]> to cache"). key_dev is [n x d] and prefix_dev
+ * [n x prefix row] in `dtype` (LACACHE_F32 rows are rounded to bf16, to nearest even, on the device); ids_dev is
  * [n x k] int32. All-or-nothing: if size + n > capacity, returns LACACHE_ERR_CAPACITY and inserts nothing. The new
  * entries get ids first_id .. first_id + n - 1 (first_id may be NULL). Asynchronous on cuda_stream. */
 lacache_status lacache_insert(lacache_t* h, int64_t n, const void* key_dev, const void* prefix_dev,
                               const int32_t* ids_dev, int32_t dtype, int64_t* first_id, void* cuda_stream);
 
 /* Batched two-stage lookup of B queries (1 <= B <= max_batch): q_emb_dev [B x d] bf16 key embeddings of the
- * queries, q_prefix_dev [B x d] bf16 embeddings of their speculatively decoded k-token prefixes f_k(x),
+ * queries, q_prefix_dev [B x prefix row] bf16 embeddings of their speculatively decoded k-token prefixes f_k(x),
  * q_ids_dev [B x k] int32 those token ids. Stage 1 keeps per query the top_c entries with key score >= tau_c by
  * (score desc, id asc); stage 2 checks them in that order and serves the first that passes. Writes every
  * non-NULL field of *out (device pointers). Asynchronous on cuda_stream; no host synchronization. */
@@ -136,8 +153,8 @@ lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_
                                      const int32_t* q_ids_dev, const uint8_t* status_dev, int64_t* first_id,
                                      int64_t* n_appended, void* cuda_stream);
 
-/* Copy entries [first, first + n) of the store into caller device buffers (key_dev/prefix_dev [n x d] bf16,
- * ids_dev [n x k]); any of the three may be NULL. For checkpoints and checks. Asynchronous on cuda_stream. */
+/* Copy entries [first, first + n) of the store into caller device buffers (key_dev [n x d], prefix_dev
+ * [n x prefix row] bf16, ids_dev [n x k]); any of the three may be NULL. For checkpoints and checks. Asynchronous on cuda_stream. */
 lacache_status lacache_read_rows(const lacache_t* h, int64_t first, int64_t n, void* key_dev, void* prefix_dev,
                                  int32_t* ids_dev, void* cuda_stream);
 
@@ -173,7 +190,8 @@ lacache_status lacache_inject_stall(lacache_t* h, int32_t lookups);
  * cudaMalloc and cudaFree can cause, and plug-ins with a fixed memory budget. The paper has no counterpart; this
  * is a deployment variant of lacache_lookup.
  *
- * The cache rows are caller-owned device arrays in the store's layout: key_dev and prefix_dev [n x d] bf16
+ * It runs a single lookahead check (m = 1). The cache rows are caller-owned device arrays in the store's layout:
+ * key_dev and prefix_dev [n x d] bf16
  * (16-byte aligned), ids_dev [n x k] int32. Queries and outputs are as for lacache_lookup. From *cfg it uses
  * d, k, tau_c, tau_a, top_c, token_match_min, check_mode, device and stage1; capacity and max_batch are ignored.
  * The stage-1 scratch lives in an 8 MiB file-scope device array of the library, which every GPU that loads the

@@ -11,11 +11,13 @@
 
 struct lacache {
   lacache_config cfg;
+  lacache_ensemble ens;      // the lookahead checks (m = 1 for lacache_create)
+  int pd;                    // prefix row length: sum of ens.dims
   int num_sms;
   int max_splits;
   int64_t n;                 // valid entries, as of the calls issued so far
   __nv_bfloat16* key;        // [capacity x d]
-  __nv_bfloat16* prefix;     // [capacity x d]
+  __nv_bfloat16* prefix;     // [capacity x pd]
   int32_t* ids;              // [capacity x k]
   uint64_t* part_cand;       // [max_splits x max_batch x top_c]
   float* part_best;          // [max_splits x max_batch]
@@ -61,12 +63,14 @@ bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 lacache_status from_cuda(cudaError_t e) { return e == cudaSuccess ? LACACHE_OK : LACACHE_ERR_CUDA; }
 
-// f32 -> bf16 (round to nearest even) of n*d elements of two arrays, into the store.
+// f32 -> bf16 (round to nearest even) of the key rows (count_a elements) and prefix rows (count_b), into the store.
 __global__ void convert_rows_kernel(const float* __restrict__ a, const float* __restrict__ b,
-                                    __nv_bfloat16* __restrict__ da, __nv_bfloat16* __restrict__ db, int64_t count) {
+                                    __nv_bfloat16* __restrict__ da, __nv_bfloat16* __restrict__ db, int64_t count_a,
+                                    int64_t count_b) {
+  const int64_t count = count_a > count_b ? count_a : count_b;
   for (int64_t i = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; i < count; i += (int64_t)gridDim.x * blockDim.x) {
-    da[i] = __float2bfloat16_rn(a[i]);
-    db[i] = __float2bfloat16_rn(b[i]);
+    if (i < count_a) da[i] = __float2bfloat16_rn(a[i]);
+    if (i < count_b) db[i] = __float2bfloat16_rn(b[i]);
   }
 }
 
@@ -102,34 +106,34 @@ __global__ void append_rank_kernel(const uint8_t* __restrict__ status, int B, in
 // Copy the rows of the ranked queries into the store at n0 + rank, unless the batch would overflow capacity.
 __global__ void append_rows_kernel(const uint4* __restrict__ q_emb, const uint4* __restrict__ q_pre,
                                    const int32_t* __restrict__ q_ids, const int32_t* __restrict__ dst,
-                                   const int32_t* __restrict__ count, int B, int d, int k, int64_t n0,
+                                   const int32_t* __restrict__ count, int B, int d, int pd, int k, int64_t n0,
                                    int64_t capacity, uint4* __restrict__ key, uint4* __restrict__ pre,
                                    int32_t* __restrict__ ids) {
   if (n0 + *count > capacity) return;
-  const int v_per_row = d / 8;
+  const int kv = d / 8, pv = pd / 8;   // 16-byte vectors per key row and per prefix row
   const int q = blockIdx.x;
   if (q >= B) return;
   const int r = dst[q];
   if (r < 0) return;
   const int64_t row = n0 + r;
-  for (int i = threadIdx.x; i < v_per_row; i += blockDim.x) {
-    key[row * v_per_row + i] = q_emb[(int64_t)q * v_per_row + i];
-    pre[row * v_per_row + i] = q_pre[(int64_t)q * v_per_row + i];
-  }
+  for (int i = threadIdx.x; i < kv; i += blockDim.x) key[row * kv + i] = q_emb[(int64_t)q * kv + i];
+  for (int i = threadIdx.x; i < pv; i += blockDim.x) pre[row * pv + i] = q_pre[(int64_t)q * pv + i];
   for (int i = threadIdx.x; i < k; i += blockDim.x) ids[row * k + i] = q_ids[(int64_t)q * k + i];
 }
 
-size_t stage_in_bytes(const lacache_config& c) {
-  return (size_t)c.max_batch * ((size_t)4 * c.d + (size_t)4 * c.k);
+size_t stage_in_bytes(const lacache_config& c, int pd) {
+  return (size_t)c.max_batch * ((size_t)2 * c.d + (size_t)2 * pd + (size_t)4 * c.k);
 }
-size_t stage_out_bytes(const lacache_config& c) {
-  // five [B] 4-byte arrays, four [B x top_c] 4-byte arrays, one [B] byte array, each rounded up to 16 bytes
-  return (size_t)c.max_batch * (21 + (size_t)c.top_c * 16) + 10 * 16;
+size_t stage_out_bytes(const lacache_config& c, int m) {
+  // five [B] 4-byte arrays, four [B x top_c] 4-byte arrays, one [B x m] 4-byte array, one [B] byte array, each
+  // rounded up to 16 bytes
+  return (size_t)c.max_batch * (21 + (size_t)c.top_c * 16 + (size_t)m * 4) + 11 * 16;
 }
 
 // Layout of the results of lookup_host in the device staging buffer (and in its pinned host copy): the arrays of
 // a B-query batch packed back to back, each 16-byte aligned, so that one copy brings them all back.
-lacache_result staged_result(unsigned char* base, int B, int top_c, bool cand, size_t* bytes) {
+lacache_result staged_result(unsigned char* base, int B, int top_c, int m, bool cand, bool scores,
+                             size_t* bytes) {
   unsigned char* p = base;
   auto take = [&](size_t n) {
     unsigned char* r = p;
@@ -148,6 +152,7 @@ lacache_result staged_result(unsigned char* base, int B, int top_c, bool cand, s
   r.cand_score = cand ? (float*)take(bc * 4) : nullptr;
   r.cand_prefix_score = cand ? (float*)take(bc * 4) : nullptr;
   r.cand_matches = cand ? (int32_t*)take(bc * 4) : nullptr;
+  r.prefix_scores = scores ? (float*)take(b * m * 4) : nullptr;
   *bytes = (size_t)(p - base);
   return r;
 }
@@ -211,16 +216,20 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
     }
     if (e != cudaSuccess) return LACACHE_ERR_CUDA;
   }
-  Stage2Args b;
+  Stage2Args b{};
   b.n = h->n;
   b.part_cand = h->part_cand;
   b.part_best = h->part_best;
   b.splits = splits;
   b.B = B;
-  b.d = c.d;
+  b.pd = h->pd;
   b.k = c.k;
   b.top_c = c.top_c;
-  b.tau_a = c.tau_a;
+  b.m = h->ens.m;
+  for (int i = 0; i < h->ens.m; ++i) {
+    b.seg[i + 1] = b.seg[i] + h->ens.dims[i];
+    b.tau_m[i] = h->ens.tau_a[i];
+  }
   b.check_mode = c.check_mode;
   b.token_match_min = c.token_match_min;
   b.prefix = h->prefix;
@@ -261,7 +270,27 @@ lacache_status lacache_create(const lacache_config* cfg, lacache_t** out) {
   if (!out) return LACACHE_ERR_INVALID_ARG;
   *out = nullptr;
   if (!cfg) return LACACHE_ERR_INVALID_ARG;
+  lacache_ensemble one;
+  memset(&one, 0, sizeof(one));
+  one.m = 1;
+  one.dims[0] = cfg->d;
+  one.tau_a[0] = cfg->tau_a;
+  return lacache_create_ensemble(cfg, &one, out);
+}
+
+lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_ensemble* ens, lacache_t** out) {
+  if (!out) return LACACHE_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg || !ens) return LACACHE_ERR_INVALID_ARG;
   const lacache_config c = *cfg;
+  if (ens->m < 1 || ens->m > LACACHE_MAX_MODELS) return LACACHE_ERR_INVALID_ARG;
+  int pd = 0;
+  for (int i = 0; i < ens->m; ++i) {
+    if (ens->dims[i] <= 0 || isnan(ens->tau_a[i])) return LACACHE_ERR_INVALID_ARG;
+    if (ens->dims[i] % 8 != 0) return LACACHE_ERR_UNSUPPORTED;
+    pd += ens->dims[i];
+  }
+  if (pd > lc::kMaxD) return LACACHE_ERR_UNSUPPORTED;
   if (c.d <= 0 || c.k <= 0 || c.capacity <= 0 || c.top_c <= 0 || c.max_batch <= 0) return LACACHE_ERR_INVALID_ARG;
   if (isnan(c.tau_c) || isnan(c.tau_a)) return LACACHE_ERR_INVALID_ARG;
   if (c.check_mode < LACACHE_CHECK_EMB || c.check_mode > LACACHE_CHECK_BOTH) return LACACHE_ERR_INVALID_ARG;
@@ -279,6 +308,8 @@ lacache_status lacache_create(const lacache_config* cfg, lacache_t** out) {
   if (!h) return LACACHE_ERR_OOM;
   memset(h, 0, sizeof(*h));
   h->cfg = c;
+  h->ens = *ens;
+  h->pd = pd;
   if (cudaDeviceGetAttribute(&h->num_sms, cudaDevAttrMultiProcessorCount, c.device) != cudaSuccess) {
     delete h;
     return LACACHE_ERR_CUDA;
@@ -286,17 +317,17 @@ lacache_status lacache_create(const lacache_config* cfg, lacache_t** out) {
   h->max_splits = lc::max_splits_for(h->num_sms);
   const size_t cap = (size_t)c.capacity;
   bool ok = cudaMalloc(&h->key, cap * c.d * 2) == cudaSuccess &&
-            cudaMalloc(&h->prefix, cap * c.d * 2) == cudaSuccess &&
+            cudaMalloc(&h->prefix, cap * pd * 2) == cudaSuccess &&
             cudaMalloc(&h->ids, cap * c.k * 4) == cudaSuccess &&
             cudaMalloc(&h->part_cand, (size_t)h->max_splits * c.max_batch * c.top_c * 8) == cudaSuccess &&
             cudaMalloc(&h->part_best, (size_t)h->max_splits * c.max_batch * 4) == cudaSuccess &&
             cudaMalloc(&h->dev_status, 4) == cudaSuccess &&
             cudaMalloc(&h->append_dst, (size_t)c.max_batch * 4) == cudaSuccess &&
             cudaMalloc(&h->append_count, 4) == cudaSuccess &&
-            cudaMalloc(&h->stage_in, stage_in_bytes(c)) == cudaSuccess &&
-            cudaMalloc(&h->stage_out, stage_out_bytes(c)) == cudaSuccess &&
+            cudaMalloc(&h->stage_in, stage_in_bytes(c, pd)) == cudaSuccess &&
+            cudaMalloc(&h->stage_out, stage_out_bytes(c, ens->m)) == cudaSuccess &&
             cudaMallocHost(&h->append_count_host, 4) == cudaSuccess &&
-            cudaMallocHost(&h->stage_host, stage_out_bytes(c)) == cudaSuccess &&
+            cudaMallocHost(&h->stage_host, stage_out_bytes(c, ens->m)) == cudaSuccess &&
             cudaMemset(h->dev_status, 0, 4) == cudaSuccess &&
             cudaMemset(h->part_cand, 0, (size_t)h->max_splits * c.max_batch * c.top_c * 8) == cudaSuccess &&
             cudaDeviceSynchronize() == cudaSuccess;
@@ -336,19 +367,20 @@ lacache_status lacache_insert(lacache_t* h, int64_t n, const void* key_dev, cons
   DeviceGuard guard(h->cfg.device);
   if (!guard.ok()) return LACACHE_ERR_CUDA;
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  const int d = h->cfg.d, k = h->cfg.k;
-  __nv_bfloat16* kd = h->key + h->n * d;
-  __nv_bfloat16* pd = h->prefix + h->n * d;
+  const int d = h->cfg.d, k = h->cfg.k, pd = h->pd;
+  __nv_bfloat16* kdst = h->key + h->n * d;
+  __nv_bfloat16* pdst = h->prefix + h->n * pd;
   cudaError_t e;
   if (dtype == LACACHE_BF16) {
-    e = cudaMemcpyAsync(kd, key_dev, (size_t)n * d * 2, cudaMemcpyDeviceToDevice, st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(pd, prefix_dev, (size_t)n * d * 2, cudaMemcpyDeviceToDevice, st);
+    e = cudaMemcpyAsync(kdst, key_dev, (size_t)n * d * 2, cudaMemcpyDeviceToDevice, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(pdst, prefix_dev, (size_t)n * pd * 2, cudaMemcpyDeviceToDevice, st);
   } else {
-    const int64_t count = n * d;
+    const int64_t count = n * (d > pd ? d : pd);
     const int threads = 256;
     const int64_t want = (count + threads - 1) / threads;
     const int blocks = (int)(want < (int64_t)h->num_sms * 32 ? want : (int64_t)h->num_sms * 32);
-    convert_rows_kernel<<<blocks, threads, 0, st>>>((const float*)key_dev, (const float*)prefix_dev, kd, pd, count);
+    convert_rows_kernel<<<blocks, threads, 0, st>>>((const float*)key_dev, (const float*)prefix_dev, kdst, pdst,
+                                                    n * d, n * pd);
     e = cudaGetLastError();
   }
   if (e == cudaSuccess)
@@ -376,19 +408,19 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
   if (!guard.ok()) return LACACHE_ERR_CUDA;
   cudaStream_t st = (cudaStream_t)cuda_stream;
   const lacache_config& c = h->cfg;
-  const size_t emb = (size_t)B * c.d * 2;
   unsigned char* q_emb = h->stage_in;
   unsigned char* q_pre = q_emb + (size_t)c.max_batch * c.d * 2;
-  int32_t* q_ids = reinterpret_cast<int32_t*>(q_pre + (size_t)c.max_batch * c.d * 2);
-  cudaError_t e = cudaMemcpyAsync(q_emb, q_emb_host, emb, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(q_pre, q_prefix_host, emb, cudaMemcpyHostToDevice, st);
+  int32_t* q_ids = reinterpret_cast<int32_t*>(q_pre + (size_t)c.max_batch * h->pd * 2);
+  cudaError_t e = cudaMemcpyAsync(q_emb, q_emb_host, (size_t)B * c.d * 2, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(q_pre, q_prefix_host, (size_t)B * h->pd * 2, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(q_ids, q_ids_host, (size_t)B * c.k * 4, cudaMemcpyHostToDevice, st);
   if (e != cudaSuccess) return LACACHE_ERR_CUDA;
   const bool cand = out_host->cand_id || out_host->cand_score || out_host->cand_prefix_score ||
                     out_host->cand_matches;
+  const bool scores = out_host->prefix_scores != nullptr;
   size_t bytes = 0;
-  lacache_result dev = staged_result(h->stage_out, B, c.top_c, cand, &bytes);
-  lacache_result host = staged_result(h->stage_host, B, c.top_c, cand, &bytes);
+  lacache_result dev = staged_result(h->stage_out, B, c.top_c, h->ens.m, cand, scores, &bytes);
+  lacache_result host = staged_result(h->stage_host, B, c.top_c, h->ens.m, cand, scores, &bytes);
   lacache_status s = run_lookup(h, B, q_emb, q_pre, q_ids, dev, st);
   if (s != LACACHE_OK) return s;
   if (cudaMemcpyAsync(h->stage_host, h->stage_out, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
@@ -405,6 +437,7 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
       {out_host->token_matches, host.token_matches, b4}, {out_host->n_cand, host.n_cand, b4},
       {out_host->cand_id, host.cand_id, bc4},          {out_host->cand_score, host.cand_score, bc4},
       {out_host->cand_prefix_score, host.cand_prefix_score, bc4}, {out_host->cand_matches, host.cand_matches, bc4},
+      {out_host->prefix_scores, host.prefix_scores, b4 * h->ens.m},
   };
   for (const Copy& cp : copies)
     if (cp.dst && cp.src) memcpy(cp.dst, cp.src, cp.bytes);
@@ -423,7 +456,7 @@ lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_
   const lacache_config& c = h->cfg;
   append_rank_kernel<<<1, 1024, 0, st>>>(status_dev, B, h->append_dst, h->append_count);
   append_rows_kernel<<<B, 128, 0, st>>>((const uint4*)q_emb_dev, (const uint4*)q_prefix_dev, q_ids_dev,
-                                        h->append_dst, h->append_count, B, c.d, c.k, h->n, c.capacity,
+                                        h->append_dst, h->append_count, B, c.d, h->pd, c.k, h->n, c.capacity,
                                         (uint4*)h->key, (uint4*)h->prefix, h->ids);
   cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess)
@@ -445,11 +478,11 @@ lacache_status lacache_read_rows(const lacache_t* h, int64_t first, int64_t n, v
   DeviceGuard guard(h->cfg.device);
   if (!guard.ok()) return LACACHE_ERR_CUDA;
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  const int d = h->cfg.d, k = h->cfg.k;
+  const int d = h->cfg.d, k = h->cfg.k, pd = h->pd;
   cudaError_t e = cudaSuccess;
   if (key_dev) e = cudaMemcpyAsync(key_dev, h->key + first * d, (size_t)n * d * 2, cudaMemcpyDeviceToDevice, st);
   if (e == cudaSuccess && prefix_dev)
-    e = cudaMemcpyAsync(prefix_dev, h->prefix + first * d, (size_t)n * d * 2, cudaMemcpyDeviceToDevice, st);
+    e = cudaMemcpyAsync(prefix_dev, h->prefix + first * pd, (size_t)n * pd * 2, cudaMemcpyDeviceToDevice, st);
   if (e == cudaSuccess && ids_dev)
     e = cudaMemcpyAsync(ids_dev, h->ids + first * k, (size_t)n * k * 4, cudaMemcpyDeviceToDevice, st);
   return from_cuda(e);

@@ -14,6 +14,7 @@ namespace lc {
 constexpr int kMaxTopC = 32;
 constexpr int kMaxD = 8192;
 constexpr int kMaxK = 256;
+constexpr int kMaxModels = LACACHE_MAX_MODELS;
 
 // Bits of the device status word.
 constexpr unsigned int kDevTimeout = 1u;
@@ -72,15 +73,17 @@ struct Stage2Args {
   const float* part_best;
   int splits;
   int B;
-  int d;
+  int pd;                        // prefix row length: sum of the models' dimensions
   int k;
   int top_c;
-  float tau_a;
+  int m;                         // lookahead checks (models)
+  int seg[kMaxModels + 1];       // model h owns prefix row elements [seg[h], seg[h+1]), multiples of 8
+  float tau_m[kMaxModels];       // model h's threshold
   int check_mode;
   int token_match_min;
-  const __nv_bfloat16* prefix;   // [n x d] store prefix embeddings
+  const __nv_bfloat16* prefix;   // [n x pd] store prefix embeddings
   const int32_t* ids;            // [n x k] store prefix token ids
-  const __nv_bfloat16* q_prefix; // [B x d]
+  const __nv_bfloat16* q_prefix; // [B x pd]
   const int32_t* q_ids;          // [B x k]
   lacache_result out;            // device pointers
 };

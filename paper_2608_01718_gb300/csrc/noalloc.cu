@@ -136,16 +136,18 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
       if (e != cudaSuccess) result = LACACHE_ERR_CUDA;
     }
     if (result == LACACHE_OK) {
-      lc::Stage2Args b;
+      lc::Stage2Args b{};
       b.n = n;
       b.part_cand = part_cand;
       b.part_best = part_best;
       b.splits = splits;
       b.B = B;
-      b.d = c.d;
+      b.pd = c.d;
       b.k = c.k;
       b.top_c = c.top_c;
-      b.tau_a = c.tau_a;
+      b.m = 1;
+      b.seg[1] = c.d;
+      b.tau_m[0] = c.tau_a;
       b.check_mode = c.check_mode;
       b.token_match_min = c.token_match_min;
       b.prefix = reinterpret_cast<const __nv_bfloat16*>(prefix_dev);

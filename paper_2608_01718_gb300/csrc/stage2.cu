@@ -65,7 +65,8 @@ template <int CPAD>
 __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
   __shared__ uint64_t warp_top[kWarps][CPAD];
   __shared__ uint64_t cand[CPAD];
-  __shared__ float cand_r[CPAD];
+  __shared__ float cand_rm[CPAD][kMaxModels];   // every model's r per candidate
+  __shared__ int cand_emb_ok[CPAD];             // all models pass
   __shared__ int cand_m[CPAD];
   __shared__ float warp_best[kWarps];
   __shared__ int s_ncand;
@@ -142,22 +143,28 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
   __syncthreads();
   const int n_cand = s_ncand;
 
-  // 2. lookahead check of every candidate, one warp per candidate
-  const int d = a.d, k = a.k;
-  const uint4* pq = reinterpret_cast<const uint4*>(a.q_prefix + (int64_t)q * d);
+  // 2. lookahead check of every candidate, one warp per candidate; one dot product per model segment
+  const int pd = a.pd, k = a.k;
+  const uint4* pq = reinterpret_cast<const uint4*>(a.q_prefix + (int64_t)q * pd);
   const int32_t* tq = a.q_ids + (int64_t)q * k;
   for (int i = warp; i < n_cand; i += kWarps) {
     const uint32_t j = cand_id(cand[i]);
-    const uint4* pj = reinterpret_cast<const uint4*>(a.prefix + (int64_t)j * d);
-    float acc = 0.f;
-    for (int c8 = lane; c8 < d / 8; c8 += 32) acc = dot8(__ldg(pq + c8), __ldg(pj + c8), acc);
-    const float r = warp_sum(acc);
+    const uint4* pj = reinterpret_cast<const uint4*>(a.prefix + (int64_t)j * pd);
+    int emb_ok = 1;
+    for (int h = 0; h < a.m; ++h) {
+      float acc = 0.f;
+      for (int c8 = a.seg[h] / 8 + lane; c8 < a.seg[h + 1] / 8; c8 += 32)
+        acc = dot8(__ldg(pq + c8), __ldg(pj + c8), acc);
+      const float r = warp_sum(acc);
+      emb_ok &= r >= a.tau_m[h] ? 1 : 0;
+      if (lane == 0) cand_rm[i][h] = r;
+    }
     int eq = 0;
     const int32_t* tj = a.ids + (int64_t)j * k;
     for (int t = lane; t < k; t += 32) eq += (__ldg(tq + t) == __ldg(tj + t)) ? 1 : 0;
     const int m = __reduce_add_sync(kFull, eq);
     if (lane == 0) {
-      cand_r[i] = r;
+      cand_emb_ok[i] = emb_ok;
       cand_m[i] = m;
     }
   }
@@ -170,7 +177,7 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
     const bool v = i < n_cand;
     if (a.out.cand_id) a.out.cand_id[o] = v ? (int32_t)cand_id(cand[i]) : -1;
     if (a.out.cand_score) a.out.cand_score[o] = v ? cand_score(cand[i]) : qnan;
-    if (a.out.cand_prefix_score) a.out.cand_prefix_score[o] = v ? cand_r[i] : qnan;
+    if (a.out.cand_prefix_score) a.out.cand_prefix_score[o] = v ? cand_rm[i][0] : qnan;
     if (a.out.cand_matches) a.out.cand_matches[o] = v ? cand_m[i] : -1;
   }
 
@@ -179,26 +186,27 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
     const int tmin = a.token_match_min > 0 ? a.token_match_min : k;
     int served = -1;
     for (int i = 0; i < n_cand && served < 0; ++i) {
-      const bool emb_ok = cand_r[i] >= a.tau_a;
+      const bool emb_ok = cand_emb_ok[i] != 0;
       const bool tok_ok = cand_m[i] >= tmin;
       const bool pass = a.check_mode == LACACHE_CHECK_EMB ? emb_ok
                         : a.check_mode == LACACHE_CHECK_TOKENS ? tok_ok
                                                                : (emb_ok && tok_ok);
       if (pass) served = i;
     }
+    const int shown = served >= 0 ? served : 0;   // the candidate whose scores are reported
     if (served >= 0) {
       a.out.status[q] = LACACHE_HIT;
       a.out.entry_id[q] = (int32_t)cand_id(cand[served]);
       a.out.key_score[q] = cand_score(cand[served]);
-      a.out.prefix_score[q] = cand_r[served];
-      a.out.token_matches[q] = cand_m[served];
     } else {
       a.out.status[q] = n_cand ? LACACHE_REJECT : LACACHE_MISS_KEY;
       a.out.entry_id[q] = -1;
       a.out.key_score[q] = warp_best[0];
-      a.out.prefix_score[q] = n_cand ? cand_r[0] : qnan;
-      a.out.token_matches[q] = n_cand ? cand_m[0] : -1;
     }
+    a.out.prefix_score[q] = n_cand ? cand_rm[shown][0] : qnan;
+    a.out.token_matches[q] = n_cand ? cand_m[shown] : -1;
+    if (a.out.prefix_scores)
+      for (int h = 0; h < a.m; ++h) a.out.prefix_scores[(int64_t)q * a.m + h] = n_cand ? cand_rm[shown][h] : qnan;
     a.out.n_cand[q] = n_cand;
   }
 }

@@ -18,7 +18,9 @@ LACACHE_BF16, LACACHE_F32 = 0, 1
 LACACHE_STAGE1_AUTO, LACACHE_STAGE1_TENSOR, LACACHE_STAGE1_SIMT = 0, 1, 2
 LACACHE_MISS_KEY, LACACHE_HIT, LACACHE_REJECT = 0, 1, 2
 
-EXPORTS = ["lacache_create", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
+LACACHE_MAX_MODELS = 8
+
+EXPORTS = ["lacache_create", "lacache_create_ensemble", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
            "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
            "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_lookup_noalloc",
            "lacache_status_string"]
@@ -31,10 +33,15 @@ class lacache_config(ctypes.Structure):
                 ("device", ctypes.c_int32), ("stage1", ctypes.c_int32)]
 
 
+class lacache_ensemble(ctypes.Structure):
+    _fields_ = [("m", ctypes.c_int32), ("dims", ctypes.c_int32 * LACACHE_MAX_MODELS),
+                ("tau_a", ctypes.c_float * LACACHE_MAX_MODELS)]
+
+
 class lacache_result(ctypes.Structure):
     _fields_ = [(name, ctypes.c_void_p) for name in
                 ("entry_id", "status", "key_score", "prefix_score", "token_matches", "n_cand",
-                 "cand_id", "cand_score", "cand_prefix_score", "cand_matches")]
+                 "cand_id", "cand_score", "cand_prefix_score", "cand_matches", "prefix_scores")]
 
 
 class LacacheError(RuntimeError):
@@ -60,6 +67,8 @@ def load() -> ctypes.CDLL:
     p32 = ctypes.POINTER(ctypes.c_int32)
     sig = {
         "lacache_create": ([ctypes.POINTER(lacache_config), ctypes.POINTER(vp)], i32),
+        "lacache_create_ensemble": ([ctypes.POINTER(lacache_config), ctypes.POINTER(lacache_ensemble),
+                                     ctypes.POINTER(vp)], i32),
         "lacache_destroy": ([vp], i32),
         "lacache_insert": ([vp, i64, vp, vp, vp, i32, p64, vp], i32),
         "lacache_lookup": ([vp, i32, vp, vp, vp, ctypes.POINTER(lacache_result), vp], i32),
@@ -117,6 +126,22 @@ def make_config(d: int, k: int, capacity: int, tau_c: float, tau_a: float, top_c
 def lacache_create(cfg: lacache_config) -> int:
     h = ctypes.c_void_p()
     _check("lacache_create", load().lacache_create(ctypes.byref(cfg), ctypes.byref(h)))
+    return h.value
+
+
+def make_ensemble(dims, taus) -> lacache_ensemble:
+    ens = lacache_ensemble()
+    ens.m = len(dims)
+    for i, (d, t) in enumerate(zip(dims, taus)):
+        ens.dims[i] = d
+        ens.tau_a[i] = t
+    return ens
+
+
+def lacache_create_ensemble(cfg: lacache_config, ens: lacache_ensemble) -> int:
+    h = ctypes.c_void_p()
+    _check("lacache_create_ensemble", load().lacache_create_ensemble(ctypes.byref(cfg), ctypes.byref(ens),
+                                                                     ctypes.byref(h)))
     return h.value
 
 
@@ -206,7 +231,8 @@ def lacache_lookup_noalloc(cfg: lacache_config, key, prefix, ids, q_emb, q_prefi
         _ptr(q_prefix), _ptr(q_ids), ctypes.byref(res), _stream(cuda_stream, cfg.device)))
 
 
-def alloc_result(batch: int, top_c: int, device, candidates: bool = True, pinned: bool = False) -> dict:
+def alloc_result(batch: int, top_c: int, device, candidates: bool = True, pinned: bool = False,
+                 models: int = 0) -> dict:
     """Output buffers of one lookup: device tensors (or pinned host tensors with ``device="cpu"``)."""
     import torch
     kw = {"device": device}
@@ -223,6 +249,8 @@ def alloc_result(batch: int, top_c: int, device, candidates: bool = True, pinned
                     "cand_score": torch.empty((batch, top_c), dtype=torch.float32, **kw),
                     "cand_prefix_score": torch.empty((batch, top_c), dtype=torch.float32, **kw),
                     "cand_matches": torch.empty((batch, top_c), dtype=torch.int32, **kw)})
+    if models:
+        out["prefix_scores"] = torch.empty((batch, models), dtype=torch.float32, **kw)
     return out
 
 
@@ -231,11 +259,17 @@ class LaCache:
 
     def __init__(self, d: int, k: int, capacity: int, tau_c: float, tau_a: float, top_c: int, *, max_batch: int,
                  check_mode: int = LACACHE_CHECK_EMB, token_match_min: int = 0, device: int = 0,
-                 stage1: int = LACACHE_STAGE1_AUTO):
+                 stage1: int = LACACHE_STAGE1_AUTO, prefix_dims=None, tau_a_models=None):
         self.cfg = make_config(d, k, capacity, tau_c, tau_a, top_c, max_batch=max_batch, check_mode=check_mode,
                                token_match_min=token_match_min, device=device, stage1=stage1)
         self.device = device
-        self.h = lacache_create(self.cfg)
+        self.h = None
+        if prefix_dims is None:
+            self.models = 1
+            self.h = lacache_create(self.cfg)
+        else:
+            self.models = len(prefix_dims)
+            self.h = lacache_create_ensemble(self.cfg, make_ensemble(prefix_dims, tau_a_models))
 
     def close(self) -> None:
         if self.h:
@@ -260,7 +294,7 @@ class LaCache:
     def lookup(self, q_emb, q_prefix, q_ids, out: dict | None = None, candidates: bool = True,
                cuda_stream=None) -> dict:
         if out is None:
-            out = alloc_result(q_emb.shape[0], self.cfg.top_c, q_emb.device, candidates)
+            out = alloc_result(q_emb.shape[0], self.cfg.top_c, q_emb.device, candidates, models=self.models)
         lacache_lookup(self.h, q_emb, q_prefix, q_ids, out, cuda_stream)
         return out
 

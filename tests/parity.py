@@ -25,6 +25,9 @@ TOL = 2e-3
 
 
 def new_cache(w: wl.Workload, stage1: int, device: int = 0, capacity: int | None = None, **kw) -> L.LaCache:
+    if w.prefix_dims is not None:
+        kw.setdefault("prefix_dims", w.prefix_dims)
+        kw.setdefault("tau_a_models", w.tau_a_models)
     return L.LaCache(w.d, w.k, capacity or w.n, w.tau_c, w.tau_a, w.top_c, max_batch=kw.pop("max_batch", w.batch),
                      device=device, stage1=stage1, **kw)
 
@@ -59,8 +62,11 @@ def oracle_queries(q: dict, rows=None) -> dict:
 
 def params(w: wl.Workload, check_mode=oracle.CHECK_EMB, token_match_min=None) -> oracle.Params:
     # the GPU compares fp32 scores with the fp32 thresholds it was given; the oracle takes the same values
-    return oracle.Params(float(np.float32(w.tau_c)), float(np.float32(w.tau_a)), w.top_c, check_mode,
-                         token_match_min)
+    f32 = lambda x: float(np.float32(x))
+    if w.prefix_dims is not None:
+        return oracle.Params(f32(w.tau_c), 0.0, w.top_c, check_mode, token_match_min, prefix_dims=w.prefix_dims,
+                             tau_a_models=tuple(f32(t) for t in w.tau_a_models))
+    return oracle.Params(f32(w.tau_c), f32(w.tau_a), w.top_c, check_mode, token_match_min)
 
 
 def gpu_lookup(cache: L.LaCache, q: dict) -> dict:
@@ -112,7 +118,7 @@ def compare(gpu: dict, res: oracle.Result, p: oracle.Params, rows=None, pair_sco
             if st == oracle.HIT and pair_scores is not None:
                 s, r, m, k = pair_scores(b, int(gpu["entry_id"][g]))
                 assert s >= p.tau_c - TOL, f"query {g}: in-band HIT fails the key check"
-                if p.check_mode in (oracle.CHECK_EMB, oracle.CHECK_BOTH):
+                if p.check_mode in (oracle.CHECK_EMB, oracle.CHECK_BOTH) and p.prefix_dims is None:
                     assert r >= p.tau_a - TOL, f"query {g}: in-band HIT fails the lookahead check"
                 if p.check_mode in (oracle.CHECK_TOKENS, oracle.CHECK_BOTH):
                     assert m >= (p.token_match_min or k), f"query {g}: in-band HIT fails the token check"
@@ -123,6 +129,9 @@ def compare(gpu: dict, res: oracle.Result, p: oracle.Params, rows=None, pair_sco
         assert _close(gpu["key_score"][g], res.key_score[b]), f"{msg}: key score {gpu['key_score'][g]} vs {res.key_score[b]}"
         assert _close(gpu["prefix_score"][g], res.prefix_score[b]), f"{msg}: prefix score"
         assert gpu["token_matches"][g] == res.token_matches[b], f"{msg}: token matches"
+        if "prefix_scores" in gpu:
+            for h in range(res.prefix_scores.shape[1]):
+                assert _close(gpu["prefix_scores"][g, h], res.prefix_scores[b, h]), f"{msg}: model {h} score"
         if res.list_margin[b] >= TOL:
             assert gpu["n_cand"][g] == res.n_cand[b], f"{msg}: n_cand {gpu['n_cand'][g]} vs {res.n_cand[b]}"
         if "cand_id" in gpu:

@@ -89,6 +89,34 @@ def test_top_c_extremes(stage1, top_c):
     assert rep.exact + rep.band == w.batch
 
 
+@pytest.mark.parametrize("stage1", PATHS)
+def test_ensemble_of_lookahead_checks(stage1):
+    """Three lookahead checks (1024-, 384- and 768-dim prefix embeddings): a hit needs all three (section 3.4)."""
+    w = wl.WORKLOADS["ensemble-1m"].scaled(n=70_000, batch=48)
+    rep = run_parity(w, stage1)
+    assert rep.exact + rep.band == w.batch and rep.band <= 1
+    assert rep.hits > 0 and rep.rejects > 0
+
+
+def test_ensemble_full_size_rejects_prefix_mimics():
+    """ensemble-1m at full size (1,048,576 entries): every query checked; the collisions whose prefix matches the
+    victim's under the first model only are rejected by the ensemble."""
+    w = wl.WORKLOADS["ensemble-1m"]
+    st = oracle_store(w)
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+        fill(cache, w)
+        q = wl.batch(w, 0, device="cuda")
+        g = gpu_lookup(cache, q)
+    assert g["prefix_scores"].shape == (w.batch, 3)
+    oq = oracle_queries(q)
+    p = params(w)
+    rep = compare(g, oracle.lookup(st, oq, p), p, pair_scores=pair_scores_fn(st, oq))
+    assert rep.exact + rep.band == w.batch and rep.band <= 1
+    cls = q["class"].numpy()
+    assert np.all(g["status"][cls == wl.MIMIC] == L.LACACHE_REJECT)
+    assert np.all(g["status"][cls == wl.NEAR] == L.LACACHE_HIT)
+
+
 def _dev(a, dtype=torch.bfloat16):
     return torch.tensor(np.asarray(a, np.float32), device="cuda").to(dtype).contiguous()
 

@@ -39,10 +39,28 @@ def test_status_strings(lib):
 
 
 def test_struct_layouts_match_the_header():
-    # lacache_config: 2 x int32, int64, 2 x float, 6 x int32 = 48 bytes; lacache_result: 10 pointers
+    # lacache_config: 2 x int32, int64, 2 x float, 6 x int32 = 48 bytes; lacache_result: 11 pointers;
+    # lacache_ensemble: int32 + 8 int32 + 8 float
     assert ctypes.sizeof(lacache.lacache_config) == 48
     assert lacache.lacache_config.capacity.offset == 8
-    assert ctypes.sizeof(lacache.lacache_result) == 80
+    assert ctypes.sizeof(lacache.lacache_result) == 88
+    assert ctypes.sizeof(lacache.lacache_ensemble) == 68
+
+
+def test_invalid_ensembles_are_rejected_before_touching_a_device(lib):
+    cfg = lacache.make_config(64, 8, 1024, 0.9, 0.8, 8, max_batch=16)
+    h = ctypes.c_void_p(1)
+    for dims, taus, status in [((), (), lacache.LACACHE_ERR_INVALID_ARG),
+                               ((64, 12), (0.7, 0.7), lacache.LACACHE_ERR_UNSUPPORTED),
+                               ((64, 0), (0.7, 0.7), lacache.LACACHE_ERR_INVALID_ARG),
+                               ((64, 64), (0.7, float("nan")), lacache.LACACHE_ERR_INVALID_ARG),
+                               ((64,) * 9, (0.7,) * 9, lacache.LACACHE_ERR_INVALID_ARG)]:
+        ens = lacache.lacache_ensemble()
+        ens.m = len(dims)
+        for i, (d, t) in enumerate(zip(dims[:8], taus[:8])):
+            ens.dims[i], ens.tau_a[i] = d, t
+        assert lib.lacache_create_ensemble(ctypes.byref(cfg), ctypes.byref(ens), ctypes.byref(h)) == status
+        assert h.value is None
 
 
 def test_null_arguments_are_rejected_without_a_device(lib):
