@@ -11,6 +11,8 @@ from .bf16 import round_to_bf16, widen
 from .lookup import (CHECK_BOTH, CHECK_EMB, CHECK_TOKENS, HIT, MISS_KEY, REJECT, KeyCheck, Params, Result,
                      Store, decide, lookahead, lookup, passes)
 from .serve import ServeLoop
+from .calibrate import calibrate, nearest_rank, pair_similarities
 
 __all__ = ["round_to_bf16", "widen", "CHECK_BOTH", "CHECK_EMB", "CHECK_TOKENS", "HIT", "MISS_KEY", "REJECT",
-           "KeyCheck", "Params", "Result", "Store", "decide", "lookahead", "lookup", "passes", "ServeLoop"]
+           "KeyCheck", "Params", "Result", "Store", "decide", "lookahead", "lookup", "passes", "ServeLoop",
+           "calibrate", "nearest_rank", "pair_similarities"]
