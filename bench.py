@@ -376,9 +376,52 @@ def run_ours(args, w):
     return 0
 
 
+CALIBRATION = {"calib-1m": (1 << 20, 1024, 0.6, 10.0, 0.70)}   # pairs, d, paraphrase noise, percentile, cap
+
+
+def run_calibration(args):
+    """Threshold calibration (App. A.2) over n benign pairs: pair similarities + nearest-rank percentile."""
+    import torch
+
+    from paper_2608_01718_gb300 import build
+    from paper_2608_01718_gb300 import lacache as L
+    from paper_2608_01718_gb300 import workloads as wl
+    n, d, sigma, pct, cap = CALIBRATION[args.workload]
+    build.build()
+    x, y = wl.benign_pairs(n, d, sigma, device="cuda")
+    sims = torch.empty(n, dtype=torch.float32, device="cuda")
+    res = torch.empty(2, dtype=torch.float32, device="cuda")
+    ws = torch.empty(L.lacache_calibrate_workspace_bytes(), dtype=torch.uint8, device="cuda")
+    stream = torch.cuda.current_stream()
+    for _ in range(max(3, args.warmup)):
+        L.lacache_calibrate(x, y, pct, cap, sims, res, ws, stream)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        L.lacache_calibrate(x, y, pct, cap, sims, res, ws, stream)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    peaks, src = load_peaks()
+    bytes_ = 4 * n * d + 4 * n
+    line = {"metric": "calibration pairs/s (App. A.2 thresholds)", "value": n / (ms / 1e3), "unit": "pairs/s",
+            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": args.workload, "pairs": n, "d": d, "percentile": pct, "cap": cap},
+            "roofline": {"bound": "hbm", "achieved": bytes_ / (ms / 1e3) / 1e9, "peak": peaks["hbm_gbs"],
+                         "unit": "GB/s", "frac": bytes_ / (ms / 1e3) / 1e9 / peaks["hbm_gbs"],
+                         "peak_source": f"{src} (copy bandwidth)"},
+            "result": [float(v) for v in res.cpu()], "gpu_launches": 8 * args.steps}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
     from paper_2608_01718_gb300 import workloads as wl
+    if args.workload in CALIBRATION:
+        return run_calibration(args)
     w = wl.WORKLOADS[args.workload]
     if args.impl == "reference":
         return run_reference(args, w)

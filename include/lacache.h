@@ -28,6 +28,7 @@
 #ifndef LACACHE_H_
 #define LACACHE_H_
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -205,6 +206,19 @@ lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int64_t n, cons
                                       const void* prefix_dev, const int32_t* ids_dev, int32_t B,
                                       const void* q_emb_dev, const void* q_prefix_dev, const int32_t* q_ids_dev,
                                       const lacache_result* out, void* cuda_stream);
+
+/* Threshold calibration (App. A.2, "Threshold Calibration"). For n benign pairs (x_i, y_i), bf16 rows of x_dev and
+ * y_dev ([n x d] each, 16-byte aligned), writes sims_dev[i] = sim(x_i, y_i) (fp32 dot of unit vectors), then
+ * result_dev[0] = the nearest-rank `percentile` of the sims (the value of rank ceil(percentile / 100 * n) in
+ * ascending order, at least 1) and result_dev[1] = min(cap, result_dev[0]). The paper's rules are
+ * tau_c = min(0.80, P5 of the query-pair sims) and tau_a = min(0.70, P10 of the response-prefix sims), the latter
+ * per embedding model. sims_dev ([n] floats), result_dev (2 floats) and workspace_dev
+ * (lacache_calibrate_workspace_bytes() bytes, 16-byte aligned, any contents) are caller device buffers; nothing is
+ * allocated. Calls sharing a workspace must not overlap on the GPU. Asynchronous on cuda_stream. */
+lacache_status lacache_calibrate(int64_t n, int32_t d, const void* x_dev, const void* y_dev, double percentile,
+                                 float cap, float* sims_dev, float* result_dev, void* workspace_dev,
+                                 void* cuda_stream);
+size_t lacache_calibrate_workspace_bytes(void);
 
 /* Static description of a status code. */
 const char* lacache_status_string(lacache_status s);

@@ -22,7 +22,8 @@ LACACHE_MAX_MODELS = 8
 
 EXPORTS = ["lacache_create", "lacache_create_ensemble", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
            "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
-           "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_lookup_noalloc",
+           "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_calibrate", "lacache_calibrate_workspace_bytes",
+           "lacache_lookup_noalloc",
            "lacache_status_string"]
 
 
@@ -81,6 +82,8 @@ def load() -> ctypes.CDLL:
         "lacache_stage_timing": ([vp, i32], i32),
         "lacache_stage_times": ([vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double), p64], i32),
         "lacache_inject_stall": ([vp, i32], i32),
+        "lacache_calibrate": ([i64, i32, vp, vp, ctypes.c_double, ctypes.c_float, vp, vp, vp, vp], i32),
+        "lacache_calibrate_workspace_bytes": ([], ctypes.c_size_t),
         "lacache_lookup_noalloc": ([ctypes.POINTER(lacache_config), i64, vp, vp, vp, i32, vp, vp, vp,
                                     ctypes.POINTER(lacache_result), vp], i32),
         "lacache_status_string": ([i32], ctypes.c_char_p),
@@ -219,6 +222,17 @@ def lacache_stage_times(h: int) -> tuple[float, float, int]:
 
 def lacache_inject_stall(h: int, lookups: int) -> None:
     _check("lacache_inject_stall", load().lacache_inject_stall(h, lookups))
+
+
+def lacache_calibrate_workspace_bytes() -> int:
+    return int(load().lacache_calibrate_workspace_bytes())
+
+
+def lacache_calibrate(x, y, percentile: float, cap: float, sims, result, workspace, cuda_stream=None) -> None:
+    """Pair similarities of (x_i, y_i) into sims, then result = [nearest-rank percentile, min(cap, it)]."""
+    _check("lacache_calibrate", load().lacache_calibrate(int(x.shape[0]), int(x.shape[1]), _ptr(x), _ptr(y),
+                                                         float(percentile), float(cap), _ptr(sims), _ptr(result),
+                                                         _ptr(workspace), _stream(cuda_stream)))
 
 
 def lacache_lookup_noalloc(cfg: lacache_config, key, prefix, ids, q_emb, q_prefix, q_ids, out: dict,

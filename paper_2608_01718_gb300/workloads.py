@@ -273,3 +273,14 @@ def bf16_bits(t: torch.Tensor):
 
 def f32_array(t: torch.Tensor):
     return t.detach().to("cpu", torch.float32).contiguous().numpy()
+
+
+def benign_pairs(n: int, d: int, sigma: float, seed: int = 20260801, device="cpu"):
+    """n benign paraphrase pairs (x, x'): x a uniform unit vector and x' = normalise(x + noise of norm sigma),
+    both bf16 [n x d]. Stand-ins for the embeddings of the paper's 500 paraphrase pairs used to calibrate the
+    thresholds (App. A.2)."""
+    g = torch.Generator(device=device)
+    g.manual_seed(sub_seed(seed, f"benign/{n}/{d}/{sigma}", 0))
+    x = _unit(torch.randn((n, d), generator=g, device=device))
+    y = _unit(x + torch.randn((n, d), generator=g, device=device) * (sigma / math.sqrt(d)))
+    return x.to(torch.bfloat16).contiguous(), y.to(torch.bfloat16).contiguous()

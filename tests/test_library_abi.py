@@ -19,7 +19,7 @@ def lib():
 
 def declared_functions():
     text = open(HEADER).read()
-    return sorted(set(re.findall(r"^\s*(?:lacache_status|const char\*)\s+(lacache_\w+)\s*\(", text, re.M)))
+    return sorted(set(re.findall(r"^\s*(?:lacache_status|const char\*|size_t)\s+(lacache_\w+)\s*\(", text, re.M)))
 
 
 def test_header_declares_the_binding_names():
