@@ -12,7 +12,8 @@ from .lookup import (CHECK_BOTH, CHECK_EMB, CHECK_TOKENS, HIT, MISS_KEY, REJECT,
                      Store, decide, lookahead, lookup, passes)
 from .serve import ServeLoop
 from .calibrate import calibrate, nearest_rank, pair_similarities
+from .lsh import hamming, lookup_lsh, projections, signatures
 
 __all__ = ["round_to_bf16", "widen", "CHECK_BOTH", "CHECK_EMB", "CHECK_TOKENS", "HIT", "MISS_KEY", "REJECT",
            "KeyCheck", "Params", "Result", "Store", "decide", "lookahead", "lookup", "passes", "ServeLoop",
-           "calibrate", "nearest_rank", "pair_similarities"]
+           "calibrate", "nearest_rank", "pair_similarities", "hamming", "lookup_lsh", "projections", "signatures"]

@@ -128,15 +128,22 @@ class KeyCheck:
         K = widen(key_bits)
         if K.shape[0] == 0:
             return
-        s = self.q @ K.T
+        self.add_scores(self.q @ K.T, j0)
+
+    def add_scores(self, s, j0: int, admitted=None) -> None:
+        """Fold the scores s [B, rows] of rows j0.. into A_q. With an index, only the rows it admits
+        (admitted [B, rows] True) are searched at all; the others count for nothing."""
+        if s.shape[1] == 0:
+            return
+        ok = np.ones(s.shape, dtype=bool) if admitted is None else admitted
         for b in range(s.shape[0]):
-            sel = np.nonzero(s[b] >= self.tau_c)[0]
+            sel = np.nonzero(ok[b] & (s[b] >= self.tau_c))[0]
             if sel.size:
                 self._s[b].append(s[b, sel])
                 self._j[b].append(sel.astype(np.int64) + j0)
-        self.best = np.maximum(self.best, s.max(axis=1))
-        self.closest = np.minimum(self.closest, np.abs(s - self.tau_c).min(axis=1))
-        self.rows += K.shape[0]
+        self.best = np.maximum(self.best, np.where(ok, s, -np.inf).max(axis=1))
+        self.closest = np.minimum(self.closest, np.where(ok, np.abs(s - self.tau_c), np.inf).min(axis=1))
+        self.rows += s.shape[1]
 
     def above(self, b: int):
         """A_q for query b, ordered by (score descending, entry id ascending)."""

@@ -284,3 +284,18 @@ def benign_pairs(n: int, d: int, sigma: float, seed: int = 20260801, device="cpu
     x = _unit(torch.randn((n, d), generator=g, device=device))
     y = _unit(x + torch.randn((n, d), generator=g, device=device) * (sigma / math.sqrt(d)))
     return x.to(torch.bfloat16).contiguous(), y.to(torch.bfloat16).contiguous()
+
+
+def hyperplanes(bits: int, d: int, seed: int = 20260801, device="cpu") -> torch.Tensor:
+    """Random hyperplanes of the SimHash index, bf16 [bits x d] with standard normal entries."""
+    g = torch.Generator(device=device)
+    g.manual_seed(sub_seed(seed, f"hyperplanes/{bits}/{d}", 0))
+    return torch.randn((bits, d), generator=g, device=device).to(torch.bfloat16).contiguous()
+
+
+def lsh_radius(tau_c: float, bits: int, z: float = 4.0) -> int:
+    """A Hamming radius that keeps an entry at the key threshold with probability about Phi(z): the number of
+    differing bits at angle arccos(tau_c) is Binomial(bits, theta / pi)."""
+    theta = math.acos(max(-1.0, min(1.0, tau_c)))
+    p = theta / math.pi
+    return min(bits, int(math.ceil(bits * p + z * math.sqrt(bits * p * (1 - p)))))
