@@ -31,7 +31,7 @@ sys.path.insert(0, ROOT)
 METRIC = "lookups/sec at 1 GB300 (N entries, batch B, k) + % of HBM or bf16 roofline"
 UNIT = "queries/s"
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "simt": "stage1_simt.cu"}
+STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "simt": "stage1_simt.cu", "lsh": "lsh.cu"}
 
 
 def parse_args():
@@ -41,7 +41,8 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="mid-1m")
-    ap.add_argument("--stage1", choices=["auto", "tensor", "simt"], default="auto")
+    ap.add_argument("--stage1", choices=["auto", "tensor", "simt", "lsh"], default="auto")
+    ap.add_argument("--lsh-bits", type=int, default=256, help="SimHash signature bits for --stage1 lsh")
     ap.add_argument("--batches", type=int, default=8, help="distinct query batches cycled through")
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -256,7 +257,8 @@ def run_ours(args, w):
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
     build.build()
-    stage1 = {"auto": L.LACACHE_STAGE1_AUTO, "tensor": L.LACACHE_STAGE1_TENSOR, "simt": L.LACACHE_STAGE1_SIMT}
+    stage1 = {"auto": L.LACACHE_STAGE1_AUTO, "tensor": L.LACACHE_STAGE1_TENSOR, "simt": L.LACACHE_STAGE1_SIMT,
+              "lsh": L.LACACHE_STAGE1_LSH}
     cache = L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch, device=local_rank,
                       stage1=stage1[args.stage1], prefix_dims=w.prefix_dims, tau_a_models=w.tau_a_models)
     dtype = L.LACACHE_F32 if w.key_dtype == "f32" else L.LACACHE_BF16
@@ -265,6 +267,11 @@ def run_ours(args, w):
         del ch
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
+    lsh = None
+    if args.stage1 == "lsh":
+        lsh = {"bits": args.lsh_bits, "radius": wl.lsh_radius(w.tau_c, args.lsh_bits)}
+        L.lacache_enable_lsh(cache.h, lsh["bits"], lsh["radius"], wl.hyperplanes(lsh["bits"], w.d, device="cuda"))
+        torch.cuda.synchronize()
     nb = args.batches
     batches = [wl.batch(w, step=(rank * nb + i), device="cuda") for i in range(nb)]
     outs = [L.alloc_result(w.batch, w.top_c, "cuda", candidates=False) for _ in range(nb)]
@@ -278,7 +285,8 @@ def run_ours(args, w):
         step(i)
     torch.cuda.synchronize()
     cache.sync()
-    kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_SIMT: "simt"}[cache.last_launch()[1]]
+    kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_SIMT: "simt",
+                   L.LACACHE_STAGE1_LSH: "lsh"}[cache.last_launch()[1]]
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -343,6 +351,7 @@ def run_ours(args, w):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
         "config": workload_config(w) | {"parallelism": f"replicas{world}" if world > 1 else "single"},
         "stage1_kernel": kernel_name,
+        "lsh_index": lsh,
         "roofline": roof | {"traffic": traffic, "kernel": f"stage1_{kernel_name}",
                             "algorithmic_bytes_per_launch": s1_bytes, "algorithmic_flops_per_launch": flops,
                             "avg_launch_ms": t1_avg_s * 1e3},
@@ -353,7 +362,7 @@ def run_ours(args, w):
         "e2e": {"value": job["e2e_value"], "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
                 "api": "lacache_lookup_host (pinned host buffers, synchronous)"},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": (3 if lsh else 2) * args.steps,
         "clocks": clock,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

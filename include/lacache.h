@@ -61,7 +61,8 @@ typedef enum { LACACHE_BF16 = 0, LACACHE_F32 = 1 } lacache_dtype;
 typedef enum {
   LACACHE_STAGE1_AUTO = 0,
   LACACHE_STAGE1_TENSOR = 1, /* tcgen05 tensor-core scan (TMA-fed, TMEM accumulators) */
-  LACACHE_STAGE1_SIMT = 2    /* CUDA-core FFMA scan */
+  LACACHE_STAGE1_SIMT = 2,   /* CUDA-core FFMA scan */
+  LACACHE_STAGE1_LSH = 3     /* SimHash index, then the exact key check (requires lacache_enable_lsh) */
 } lacache_stage1;
 
 /* Ensemble of m lookahead checks (section 3.4, "Analysis"; Figure 6): every entry and query carries one k-token
@@ -153,6 +154,21 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
 lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
                                      const int32_t* q_ids_dev, const uint8_t* status_dev, int64_t* first_id,
                                      int64_t* n_appended, void* cuda_stream);
+
+/* The SimHash index of Eq. 1 (section 2; Algorithm 1's "search semantic cache with key h(x)"). Every entry gets a
+ * signature of `bits` bits (128, 256 or 512): bit i is set iff <r_i, key> >= 0 for the i-th row r_i of
+ * hyperplanes_dev ([bits x d] bf16, copied into the handle; random normal rows give random-hyperplane LSH). With
+ * cfg->stage1 == LACACHE_STAGE1_LSH a lookup applies the exact key check only to the entries whose signature
+ * differs from the query's in at most `radius` bits; stage 2 is unchanged. Existing entries are signed now and
+ * later inserts and appends are signed as they arrive. Allocates (capacity + max_batch) * bits / 8 bytes.
+ * Asynchronous on cuda_stream; calling it again replaces the index. */
+lacache_status lacache_enable_lsh(lacache_t* h, int32_t bits, int32_t radius, const void* hyperplanes_dev,
+                                  void* cuda_stream);
+
+/* Copy the SimHash signatures of entries [first, first + n) into sig_dev ([n x bits/32] uint32 words; bit i of
+ * word w is hyperplane 32w + i). LACACHE_ERR_INVALID_ARG if the index is not enabled. Asynchronous. */
+lacache_status lacache_read_signatures(const lacache_t* h, int64_t first, int64_t n, uint32_t* sig_dev,
+                                       void* cuda_stream);
 
 /* Copy entries [first, first + n) of the store into caller device buffers (key_dev [n x d], prefix_dev
  * [n x prefix row] bf16, ids_dev [n x k]); any of the three may be NULL. For checkpoints and checks. Asynchronous on cuda_stream. */

@@ -32,6 +32,11 @@ struct lacache {
   int last_kernel;
   lc::EncodeTiledFn encode;
   int inject_stall;          // lookups left that withhold one stage-1 load (failure-detection tests)
+  int lsh_bits;              // SimHash index: signature bits (0 = no index)
+  int lsh_radius;
+  uint32_t* sig;             // [capacity x lsh_bits/32] entry signatures
+  uint32_t* qsig;            // [max_batch x lsh_bits/32] query signatures of the current lookup
+  __nv_bfloat16* hyper;      // [lsh_bits x d] hyperplanes
   cudaEvent_t* events;       // [3 x event_cap] stage-timing events, or NULL
   int event_cap;
   int event_used;
@@ -166,7 +171,25 @@ void free_events(lacache* h) {
   h->event_cap = h->event_used = 0;
 }
 
+void free_lsh(lacache* h) {
+  cudaFree(h->sig);
+  cudaFree(h->qsig);
+  cudaFree(h->hyper);
+  h->sig = h->qsig = nullptr;
+  h->hyper = nullptr;
+  h->lsh_bits = 0;
+}
+
+// Signatures of store rows [first, first + n), when the index is enabled.
+cudaError_t sign_rows(lacache* h, int64_t first, int64_t n, cudaStream_t st) {
+  if (!h->lsh_bits || n <= 0) return cudaSuccess;
+  const int words = h->lsh_bits / 32;
+  return lc::launch_signatures(h->key + first * h->cfg.d, n, h->cfg.d, h->hyper, h->lsh_bits, h->sig + first * words,
+                               h->dev_status, h->encode, h->num_sms, st);
+}
+
 void free_all(lacache* h) {
+  free_lsh(h);
   free_events(h);
   cudaFree(h->key);
   cudaFree(h->prefix);
@@ -211,6 +234,13 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
     if (kernel == LACACHE_STAGE1_TENSOR) {
       if (!h->encode) return LACACHE_ERR_CUDA;
       e = lc::launch_stage1_tensor(a, h->encode, h->num_sms, h->max_splits, st, &splits);
+    } else if (kernel == LACACHE_STAGE1_LSH) {
+      e = lc::launch_signatures(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, h->dev_status, h->encode, h->num_sms,
+                                st);
+      if (e == cudaSuccess) {
+        lc::LshArgs l{h->sig, h->qsig, h->lsh_bits / 32, h->lsh_radius};
+        e = lc::launch_stage1_lsh(a, l, h->num_sms, h->max_splits, st, &splits);
+      }
     } else {
       e = lc::launch_stage1_simt(a, h->num_sms, h->max_splits, st, &splits);
     }
@@ -294,7 +324,7 @@ lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_
   if (c.d <= 0 || c.k <= 0 || c.capacity <= 0 || c.top_c <= 0 || c.max_batch <= 0) return LACACHE_ERR_INVALID_ARG;
   if (isnan(c.tau_c) || isnan(c.tau_a)) return LACACHE_ERR_INVALID_ARG;
   if (c.check_mode < LACACHE_CHECK_EMB || c.check_mode > LACACHE_CHECK_BOTH) return LACACHE_ERR_INVALID_ARG;
-  if (c.stage1 < LACACHE_STAGE1_AUTO || c.stage1 > LACACHE_STAGE1_SIMT) return LACACHE_ERR_INVALID_ARG;
+  if (c.stage1 < LACACHE_STAGE1_AUTO || c.stage1 > LACACHE_STAGE1_LSH) return LACACHE_ERR_INVALID_ARG;
   if (c.token_match_min > c.k) return LACACHE_ERR_INVALID_ARG;
   if (c.d % 8 != 0 || c.d > lc::kMaxD || c.k > lc::kMaxK || c.top_c > lc::kMaxTopC) return LACACHE_ERR_UNSUPPORTED;
   if (c.capacity > (int64_t)INT32_MAX || c.max_batch > (1 << 20)) return LACACHE_ERR_UNSUPPORTED;
@@ -385,6 +415,7 @@ lacache_status lacache_insert(lacache_t* h, int64_t n, const void* key_dev, cons
   }
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(h->ids + h->n * k, ids_dev, (size_t)n * k * 4, cudaMemcpyDeviceToDevice, st);
+  if (e == cudaSuccess) e = sign_rows(h, h->n, n, st);
   if (e != cudaSuccess) return LACACHE_ERR_CUDA;
   h->n += n;
   return LACACHE_OK;
@@ -465,10 +496,51 @@ lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_
   if (e != cudaSuccess) return LACACHE_ERR_CUDA;
   const int64_t m = *h->append_count_host;
   if (h->n + m > c.capacity) return LACACHE_ERR_CAPACITY;
+  if (sign_rows(h, h->n, m, st) != cudaSuccess) return LACACHE_ERR_CUDA;
   if (first_id) *first_id = h->n;
   if (n_appended) *n_appended = m;
   h->n += m;
   return LACACHE_OK;
+}
+
+lacache_status lacache_enable_lsh(lacache_t* h, int32_t bits, int32_t radius, const void* hyperplanes_dev,
+                                  void* cuda_stream) {
+  if (!h || !hyperplanes_dev || ((uintptr_t)hyperplanes_dev & 15u)) return LACACHE_ERR_INVALID_ARG;
+  if (bits != 128 && bits != 256 && bits != 512) return LACACHE_ERR_UNSUPPORTED;
+  if (radius < 0 || radius > bits) return LACACHE_ERR_INVALID_ARG;
+  if (!h->encode) return LACACHE_ERR_CUDA;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  if (h->lsh_bits && cudaStreamSynchronize(st) != cudaSuccess) return LACACHE_ERR_CUDA;
+  free_lsh(h);
+  const int words = bits / 32;
+  const lacache_config& c = h->cfg;
+  if (cudaMalloc(&h->sig, (size_t)c.capacity * words * 4) != cudaSuccess ||
+      cudaMalloc(&h->qsig, (size_t)c.max_batch * words * 4) != cudaSuccess ||
+      cudaMalloc(&h->hyper, (size_t)bits * c.d * 2) != cudaSuccess) {
+    cudaGetLastError();
+    free_lsh(h);
+    return LACACHE_ERR_OOM;
+  }
+  h->lsh_bits = bits;
+  h->lsh_radius = radius;
+  if (cudaMemcpyAsync(h->hyper, hyperplanes_dev, (size_t)bits * c.d * 2, cudaMemcpyDeviceToDevice, st) !=
+          cudaSuccess ||
+      sign_rows(h, 0, h->n, st) != cudaSuccess)
+    return LACACHE_ERR_CUDA;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_read_signatures(const lacache_t* h, int64_t first, int64_t n, uint32_t* sig_dev,
+                                       void* cuda_stream) {
+  if (!h || !h->lsh_bits || !sig_dev || first < 0 || n < 0 || first + n > h->n) return LACACHE_ERR_INVALID_ARG;
+  if (n == 0) return LACACHE_OK;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  const int words = h->lsh_bits / 32;
+  return from_cuda(cudaMemcpyAsync(sig_dev, h->sig + first * words, (size_t)n * words * 4, cudaMemcpyDeviceToDevice,
+                                   (cudaStream_t)cuda_stream));
 }
 
 lacache_status lacache_read_rows(const lacache_t* h, int64_t first, int64_t n, void* key_dev, void* prefix_dev,

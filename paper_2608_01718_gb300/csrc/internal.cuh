@@ -100,6 +100,23 @@ cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int 
                                  cudaStream_t st, int* splits);
 cudaError_t launch_stage2(const Stage2Args& a, cudaStream_t st);
 
+// SimHash signatures of n rows ([n x d] bf16) against `bits` hyperplanes ([bits x d] bf16), bits a multiple of 32:
+// sig[j * bits/32 + w] bit i is set iff <hyperplane 32w + i, row j> >= 0 (tensor-core GEMM, sign epilogue).
+cudaError_t launch_signatures(const __nv_bfloat16* rows, int64_t n, int d, const __nv_bfloat16* hyperplanes,
+                              int bits, uint32_t* sig, unsigned int* dev_status, EncodeTiledFn encode, int num_sms,
+                              cudaStream_t st);
+
+// The SimHash-indexed key check: entries whose signature is within `radius` of the query's get the exact key
+// check (threshold + top-c partial lists, as the other stage-1 kernels).
+struct LshArgs {
+  const uint32_t* sig;     // [n x words] entry signatures
+  const uint32_t* qsig;    // [B x words] query signatures
+  int words;
+  int radius;
+};
+cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits, cudaStream_t st,
+                              int* splits);
+
 // Largest split count any stage-1 launcher uses for a given SM count (sizes the scratch).
 inline int max_splits_for(int num_sms) { return num_sms; }
 

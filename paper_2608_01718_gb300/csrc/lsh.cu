@@ -1,0 +1,200 @@
+// Stage 1 through the SimHash index (Eq. 1; Algorithm 1's "search semantic cache with key h(x)"): the key check
+// sim(x, x') >= tau_c applied only to the entries whose signature is within `radius` bits of the query's.
+//
+// One CTA per contiguous split of the entries; one entry per thread per tile of 256. A thread loads its entry's
+// signature (16-byte loads) and counts the differing bits against each of up to 16 query signatures held in shared
+// memory. Admitted (query, entry) pairs are queued in shared memory; when the queue is half full, and at the end
+// of the split, all warps take queue items two at a time and compute the exact fp32 score over the gathered key row
+// (each lane's 8-element chunks in order, then a butterfly sum). The warp of each query then folds the scores
+// that clear tau_c into that query's top-c list. The partial lists have the format of the other stage-1 kernels,
+// so stage 2 is shared.
+#include "internal.cuh"
+
+namespace lc {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr int kTile = 256;          // entries per tile, one per thread
+constexpr int kQC = 16;             // queries per pass over the entries
+constexpr int kCap = 8192;          // queue capacity; a tile adds at most kTile * kQC = 4096 items
+constexpr unsigned kFull = 0xffffffffu;
+
+struct Item {
+  int32_t j;      // entry id
+  int32_t q;      // query within the pass
+};
+
+__device__ __forceinline__ float dot8(const uint4& u, const uint4& v, float acc) {
+  const __nv_bfloat162* a = reinterpret_cast<const __nv_bfloat162*>(&u);
+  const __nv_bfloat162* b = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    const float2 x = __bfloat1622float2(a[e]);
+    const float2 y = __bfloat1622float2(b[e]);
+    acc = fmaf(x.x, y.x, acc);
+    acc = fmaf(x.y, y.y, acc);
+  }
+  return acc;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  return v;
+}
+
+struct Shared {
+  uint32_t qsig[kQC][16];
+  uint64_t list[kQC][kMaxTopC];   // per query: sorted packed candidates of this split, 0 = empty
+  unsigned int best[kQC];         // score_order of the best admitted score
+  int count;                      // queued items
+  Item items[kCap];
+  float score[kCap];
+};
+
+// Exact scores of the queued items, then each query's warp folds its items into the query's list.
+__device__ void flush(Shared& sh, const Stage1Args& a, int q0, int qn) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int total = sh.count;
+  const int v = a.d / 8;
+  for (int base = warp * 2; base < total; base += kWarps * 2) {
+    float acc0 = 0.f, acc1 = 0.f;
+    const Item i0 = sh.items[base];
+    const bool two = base + 1 < total;
+    const Item i1 = two ? sh.items[base + 1] : i0;
+    const uint4* k0 = reinterpret_cast<const uint4*>(a.keys + (int64_t)i0.j * a.d);
+    const uint4* k1 = reinterpret_cast<const uint4*>(a.keys + (int64_t)i1.j * a.d);
+    const uint4* x0 = reinterpret_cast<const uint4*>(a.q + (int64_t)(q0 + i0.q) * a.d);
+    const uint4* x1 = reinterpret_cast<const uint4*>(a.q + (int64_t)(q0 + i1.q) * a.d);
+    for (int c = lane; c < v; c += 32) {
+      acc0 = dot8(__ldg(x0 + c), __ldg(k0 + c), acc0);
+      acc1 = dot8(__ldg(x1 + c), __ldg(k1 + c), acc1);
+    }
+    acc0 = warp_sum(acc0);
+    acc1 = warp_sum(acc1);
+    if (lane == 0) {
+      sh.score[base] = acc0;
+      if (two) sh.score[base + 1] = acc1;
+    }
+  }
+  __syncthreads();
+  const int C = a.top_c;
+  for (int qq = warp; qq < qn; qq += kWarps) {
+    float best = -INFINITY;
+    for (int base = 0; base < total; base += 32) {
+      const int idx = base + lane;
+      const bool mine = idx < total && sh.items[idx].q == qq;
+      const float sc = mine ? sh.score[idx] : -INFINITY;
+      best = fmaxf(best, sc);
+      unsigned pass = __ballot_sync(kFull, mine && sc >= a.tau_c);
+      while (pass) {   // lane 0 inserts the passing items of this group one by one
+        const int src = __ffs(pass) - 1;
+        pass &= pass - 1;
+        const float s = __shfl_sync(kFull, sc, src);
+        const int j = __shfl_sync(kFull, mine ? sh.items[idx].j : 0, src);
+        if (lane == 0) {
+          uint64_t x = pack_cand(s, (uint32_t)j);
+          uint64_t* L = sh.list[qq];
+          if (x > L[C - 1]) {
+            int p = C - 1;
+            while (p > 0 && L[p - 1] < x) {
+              L[p] = L[p - 1];
+              --p;
+            }
+            L[p] = x;
+          }
+        }
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(kFull, best, o));
+    if (lane == 0 && best > -INFINITY) atomicMax(&sh.best[qq], score_order(best));
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) sh.count = 0;
+  __syncthreads();
+}
+
+template <int W>
+__global__ void __launch_bounds__(kThreads) lsh_scan_kernel(Stage1Args a, LshArgs l, int splits) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  Shared& sh = *reinterpret_cast<Shared*>(smem_raw);
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const int s = blockIdx.x;
+  const int64_t j_begin = a.n * s / splits, j_end = a.n * (s + 1) / splits;
+  const int C = a.top_c;
+  for (int q0 = 0; q0 < a.B; q0 += kQC) {
+    const int qn = min(kQC, a.B - q0);
+    for (int i = threadIdx.x; i < kQC * W; i += kThreads) {
+      const int qq = i / W;
+      sh.qsig[qq][i % W] = qq < qn ? l.qsig[(int64_t)(q0 + qq) * W + i % W] : 0u;
+    }
+    for (int i = threadIdx.x; i < kQC * kMaxTopC; i += kThreads) sh.list[i / kMaxTopC][i % kMaxTopC] = 0;
+    if (threadIdx.x < kQC) sh.best[threadIdx.x] = score_order(-INFINITY);
+    if (threadIdx.x == 0) sh.count = 0;
+    __syncthreads();
+    for (int64_t t0 = j_begin; t0 < j_end; t0 += kTile) {
+      const int64_t j = t0 + threadIdx.x;
+      if (j < j_end) {
+        uint32_t e[W];
+        const uint4* src = reinterpret_cast<const uint4*>(l.sig + j * W);
+#pragma unroll
+        for (int w = 0; w < W / 4; ++w) {
+          const uint4 u = __ldg(src + w);
+          e[4 * w] = u.x;
+          e[4 * w + 1] = u.y;
+          e[4 * w + 2] = u.z;
+          e[4 * w + 3] = u.w;
+        }
+        for (int qq = 0; qq < qn; ++qq) {
+          int hd = 0;
+#pragma unroll
+          for (int w = 0; w < W; ++w) hd += __popc(e[w] ^ sh.qsig[qq][w]);
+          if (hd <= l.radius) {
+            const int slot = atomicAdd(&sh.count, 1);
+            sh.items[slot] = Item{(int32_t)j, qq};
+          }
+        }
+      }
+      __syncthreads();
+      if (sh.count > kCap - kTile * kQC) flush(sh, a, q0, qn);
+    }
+    flush(sh, a, q0, qn);
+    for (int i = threadIdx.x; i < qn * C; i += kThreads) {
+      const int qq = i / C;
+      a.part_cand[((int64_t)s * a.B + q0 + qq) * C + (i - qq * C)] = sh.list[qq][i - qq * C];
+    }
+    if (threadIdx.x < qn) a.part_best[(int64_t)s * a.B + q0 + threadIdx.x] = score_of_order(sh.best[threadIdx.x]);
+    __syncthreads();
+  }
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <int W>
+cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStream_t st) {
+  const size_t smem = sizeof(Shared);
+  cudaError_t e = cudaFuncSetAttribute(lsh_scan_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  lsh_scan_kernel<W><<<splits, kThreads, smem, st>>>(a, l, splits);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits, cudaStream_t st,
+                              int* splits) {
+  const int64_t tiles = (a.n + kTile - 1) / kTile;
+  int s = (int)(tiles < (int64_t)num_sms ? tiles : (int64_t)num_sms);
+  if (s > max_splits) s = max_splits;
+  if (s < 1) s = 1;
+  *splits = s;
+  switch (l.words) {   // 128, 256 or 512-bit signatures (16-byte loads)
+    case 4: return launch_w<4>(a, l, s, st);
+    case 8: return launch_w<8>(a, l, s, st);
+    case 16: return launch_w<16>(a, l, s, st);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace lc

@@ -61,6 +61,8 @@ struct TcParams {
   int a_rows;     // rows of the query box: B rounded up to 8 when B <= 128, else 128
   int prefetch;   // key boxes prefetched into L2 ahead of the ring (0 = off)
   int inject_stall;  // test support: CTA 0 withholds its second load, so its MMA issuer's bounded wait runs out
+  uint32_t* sig;     // signature mode: [n x sig_words] output words
+  int sig_words;
   uint64_t* part_cand;
   float* part_best;
   unsigned int* dev_status;
@@ -215,7 +217,10 @@ struct TopC {
   }
 };
 
-template <int CPAD>
+// SIGN = false: the key check (threshold + top-c partial lists). SIGN = true: the same GEMM with random hyperplanes
+// in place of the queries, and an epilogue that writes SimHash signatures: bit h of row j's signature is set iff
+// <r_h, row_j> >= 0; each warp's 32 hyperplanes form one 32-bit word, packed with a ballot per key column.
+template <int CPAD, bool SIGN>
 __global__ void __launch_bounds__(kThreads, 1)
     stage1_tensor_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
                          const TcParams p) {
@@ -375,6 +380,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       TopC<CPAD> top;
       top.init(p.tau_c);
       float best = -INFINITY;
+      const int word = (qt * BM + quad * 32) / 32;   // signature mode: this warp's word of every signature
       for (int64_t t = t_begin; t < t_end; ++t, ++tile_i) {
         const int b = tile_i & 1u;
         const uint32_t par = (tile_i >> 1) & 1u;
@@ -393,7 +399,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int ch = 0; ch < BN / 32; ++ch) {
           float v[32];
           tmem_ld32(tmem + lane_addr + (uint32_t)(b * BN + ch * 32), v);
-          if (active) {
+          if constexpr (SIGN) {
+            // lane e keeps the word of key column jc + e: bit `lane` of it is this thread's hyperplane's sign
+            const int64_t jc = j0 + ch * 32;
+            uint32_t mine = 0;
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              const uint32_t w = __ballot_sync(full, v[e] >= 0.f);
+              if (lane == e) mine = w;
+            }
+            if (word < p.sig_words && jc + lane < p.n) p.sig[(jc + lane) * p.sig_words + word] = mine;
+          } else if (active) {
             const int64_t jc = j0 + ch * 32;
             if (ragged) {
 #pragma unroll
@@ -426,7 +442,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) mbar_arrive(tempty_bar(b));
       }
       if (!ok) break;
-      if (active) {
+      if (active && !SIGN) {
         uint64_t* dst = p.part_cand + ((int64_t)sp * p.B + q) * p.top_c;
 #pragma unroll
         for (int i = 0; i < CPAD; ++i)
@@ -465,9 +481,9 @@ int gcd_int(int a, int b) {
   return a;
 }
 
-template <int CPAD>
+template <int CPAD, bool SIGN = false>
 cudaError_t launch_cpad(const CUtensorMap* tq, const CUtensorMap* tk, const TcParams& p, int grid, cudaStream_t st) {
-  cudaError_t e = cudaFuncSetAttribute(stage1_tensor_kernel<CPAD>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(stage1_tensor_kernel<CPAD, SIGN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)kSmemBytes);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -480,7 +496,7 @@ cudaError_t launch_cpad(const CUtensorMap* tq, const CUtensorMap* tk, const TcPa
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, stage1_tensor_kernel<CPAD>, *tq, *tk, p);
+  e = cudaLaunchKernelEx(&cfg, stage1_tensor_kernel<CPAD, SIGN>, *tq, *tk, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -498,9 +514,40 @@ bool encode_rows(EncodeTiledFn encode, CUtensorMap* m, const void* base, int64_t
 
 }  // namespace
 
+cudaError_t launch_signatures(const __nv_bfloat16* rows, int64_t n, int d, const __nv_bfloat16* hyperplanes,
+                              int bits, uint32_t* sig, unsigned int* dev_status, EncodeTiledFn encode, int num_sms,
+                              cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  TcParams p{};
+  p.n = n;
+  p.d = d;
+  p.B = bits;
+  p.tau_c = 0.f;
+  p.top_c = 1;
+  p.q_tiles = (bits + BM - 1) / BM;
+  p.n_tiles = (n + BN - 1) / BN;
+  p.k_steps = (d + BK - 1) / BK;
+  p.prefetch = 0;
+  p.a_rows = bits >= BM ? BM : ((bits + 7) / 8) * 8;
+  int s = num_sms / gcd_int(num_sms, p.q_tiles);
+  if ((int64_t)s > p.n_tiles) s = (int)p.n_tiles;
+  if (s < 1) s = 1;
+  p.splits = s;
+  p.units = p.q_tiles * s;
+  p.sig = sig;
+  p.sig_words = bits / 32;
+  p.dev_status = dev_status;
+  CUtensorMap tq, tk;
+  if (!encode_rows(encode, &tq, hyperplanes, d, bits, (uint32_t)p.a_rows) ||
+      !encode_rows(encode, &tk, rows, d, n, (uint32_t)BN))
+    return cudaErrorInvalidValue;
+  const int grid = p.units < num_sms ? p.units : num_sms;
+  return launch_cpad<4, true>(&tq, &tk, p, grid, st);
+}
+
 cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int num_sms, int max_splits,
                                  cudaStream_t st, int* splits) {
-  TcParams p;
+  TcParams p{};
   p.n = a.n;
   p.d = a.d;
   p.B = a.B;

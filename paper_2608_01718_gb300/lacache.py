@@ -15,14 +15,14 @@ LACACHE_OK, LACACHE_ERR_INVALID_ARG, LACACHE_ERR_CAPACITY, LACACHE_ERR_OOM = 0, 
 LACACHE_ERR_CUDA, LACACHE_ERR_DEVICE_TIMEOUT, LACACHE_ERR_UNSUPPORTED = 4, 5, 6
 LACACHE_CHECK_EMB, LACACHE_CHECK_TOKENS, LACACHE_CHECK_BOTH = 0, 1, 2
 LACACHE_BF16, LACACHE_F32 = 0, 1
-LACACHE_STAGE1_AUTO, LACACHE_STAGE1_TENSOR, LACACHE_STAGE1_SIMT = 0, 1, 2
+LACACHE_STAGE1_AUTO, LACACHE_STAGE1_TENSOR, LACACHE_STAGE1_SIMT, LACACHE_STAGE1_LSH = 0, 1, 2, 3
 LACACHE_MISS_KEY, LACACHE_HIT, LACACHE_REJECT = 0, 1, 2
 
 LACACHE_MAX_MODELS = 8
 
 EXPORTS = ["lacache_create", "lacache_create_ensemble", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
            "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
-           "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_calibrate", "lacache_calibrate_workspace_bytes",
+           "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_enable_lsh", "lacache_read_signatures", "lacache_calibrate", "lacache_calibrate_workspace_bytes",
            "lacache_lookup_noalloc",
            "lacache_status_string"]
 
@@ -82,6 +82,8 @@ def load() -> ctypes.CDLL:
         "lacache_stage_timing": ([vp, i32], i32),
         "lacache_stage_times": ([vp, ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_double), p64], i32),
         "lacache_inject_stall": ([vp, i32], i32),
+        "lacache_enable_lsh": ([vp, i32, i32, vp, vp], i32),
+        "lacache_read_signatures": ([vp, i64, i64, vp, vp], i32),
         "lacache_calibrate": ([i64, i32, vp, vp, ctypes.c_double, ctypes.c_float, vp, vp, vp, vp], i32),
         "lacache_calibrate_workspace_bytes": ([], ctypes.c_size_t),
         "lacache_lookup_noalloc": ([ctypes.POINTER(lacache_config), i64, vp, vp, vp, i32, vp, vp, vp,
@@ -222,6 +224,15 @@ def lacache_stage_times(h: int) -> tuple[float, float, int]:
 
 def lacache_inject_stall(h: int, lookups: int) -> None:
     _check("lacache_inject_stall", load().lacache_inject_stall(h, lookups))
+
+
+def lacache_enable_lsh(h: int, bits: int, radius: int, hyperplanes, cuda_stream=None) -> None:
+    """Build the SimHash index: signatures of every entry against hyperplanes ([bits x d] bf16)."""
+    _check("lacache_enable_lsh", load().lacache_enable_lsh(h, bits, radius, _ptr(hyperplanes), _stream(cuda_stream)))
+
+
+def lacache_read_signatures(h: int, first: int, n: int, out, cuda_stream=None) -> None:
+    _check("lacache_read_signatures", load().lacache_read_signatures(h, first, n, _ptr(out), _stream(cuda_stream)))
 
 
 def lacache_calibrate_workspace_bytes() -> int:

@@ -1,0 +1,103 @@
+"""GPU parity of the SimHash-indexed key check (Eq. 1; Algorithm 1's cache search) against the oracle.
+
+Signatures are sign decisions of fp32 tensor-core dot products; the oracle takes them in fp64. Bits whose
+projection is within 1e-4 of zero may legitimately differ: they are counted, and the queries whose outcome such
+a bit could change are excluded from the exact comparison (reported, at most a few)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_01718_gb300 import build
+from paper_2608_01718_gb300 import lacache as L
+from paper_2608_01718_gb300 import workloads as wl
+
+from parity import compare, fill, gpu_lookup, new_cache, oracle_queries, oracle_store, params
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def library():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    build.build()
+    L.load()
+
+
+def _unpack(words, bits):
+    w = words.astype(np.uint64)
+    out = np.zeros((w.shape[0], bits), dtype=bool)
+    for i in range(bits):
+        out[:, i] = (w[:, i // 32] >> np.uint64(i % 32)) & np.uint64(1)
+    return out
+
+
+@pytest.mark.parametrize("bits", [128, 256, 512])
+def test_signatures_match_the_oracle(bits):
+    w = wl.WORKLOADS["mid-1m"].scaled(n=20_000)
+    R = wl.hyperplanes(bits, w.d, device="cuda")
+    st = oracle_store(w)
+    with new_cache(w, L.LACACHE_STAGE1_LSH) as cache:
+        fill(cache, w)
+        L.lacache_enable_lsh(cache.h, bits, 40, R)
+        sig = torch.empty((w.n, bits // 32), dtype=torch.int32, device="cuda")
+        L.lacache_read_signatures(cache.h, 0, w.n, sig)
+        torch.cuda.synchronize()
+    got = _unpack(sig.cpu().numpy().view(np.uint32), bits)
+    want, amb = oracle.signatures(st.key, wl.bf16_bits(R))
+    diff = got != want
+    assert not np.any(diff & ~amb), "a signature bit differs away from a zero projection"
+    assert amb.mean() < 1e-3
+
+
+@pytest.mark.parametrize("bits", [128, 256])
+def test_lsh_lookup_matches_the_oracle(bits):
+    w = wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=40)
+    radius = wl.lsh_radius(w.tau_c, bits)
+    R = wl.hyperplanes(bits, w.d, device="cuda")
+    st = oracle_store(w)
+    with new_cache(w, L.LACACHE_STAGE1_LSH) as cache:
+        fill(cache, w)
+        L.lacache_enable_lsh(cache.h, bits, radius, R)
+        q = wl.batch(w, 0, device="cuda")
+        g = gpu_lookup(cache, q)
+    oq = oracle_queries(q)
+    p = params(w)
+    res, amb = oracle.lookup_lsh(st, oq, p, wl.bf16_bits(R), radius)
+    keep = np.nonzero(~amb)[0]
+    sub = oracle.Result(**{f: getattr(res, f)[keep] for f in res.__dataclass_fields__})
+    rep = compare(g, sub, p, rows=keep)
+    assert rep.exact + rep.band == len(keep) and len(keep) >= w.batch - 2
+    assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
+    # at this radius the index keeps every near-duplicate's target: the decisions equal the exact lookup's
+    exact = oracle.lookup(st, oq, p)
+    assert np.array_equal(res.status, exact.status) and np.array_equal(res.entry_id, exact.entry_id)
+
+
+def test_full_radius_equals_the_exact_scan_and_appends_are_signed():
+    w = wl.WORKLOADS["serve-2m"].scaled(n=30_000, batch=64, clusters=300)
+    R = wl.hyperplanes(256, w.d, device="cuda")
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR, capacity=w.n + 4 * w.batch) as exact_cache, \
+            new_cache(w, L.LACACHE_STAGE1_LSH, capacity=w.n + 4 * w.batch) as lsh_cache:
+        fill(exact_cache, w)
+        fill(lsh_cache, w)
+        L.lacache_enable_lsh(lsh_cache.h, 256, 256, R)        # radius = bits: nothing is pruned
+        for step in range(3):
+            q = wl.batch(w, step, device="cuda")
+            a = exact_cache.lookup(q["emb"], q["prefix"], q["ids"])
+            b = lsh_cache.lookup(q["emb"], q["prefix"], q["ids"])
+            assert torch.equal(a["status"], b["status"]) and torch.equal(a["entry_id"], b["entry_id"])
+            assert torch.equal(a["cand_id"], b["cand_id"])
+            assert torch.allclose(a["cand_score"], b["cand_score"], atol=2e-3, equal_nan=True)
+            exact_cache.append_misses(q["emb"], q["prefix"], q["ids"], a["status"])
+            first, m = lsh_cache.append_misses(q["emb"], q["prefix"], q["ids"], b["status"])
+        sig = torch.empty((m, 8), dtype=torch.int32, device="cuda")
+        L.lacache_read_signatures(lsh_cache.h, first, m, sig)
+        torch.cuda.synchronize()
+        # the appended entries are the last batch's non-HIT queries, in query order
+        miss = torch.nonzero(b["status"] != L.LACACHE_HIT).flatten()
+        assert len(miss) == m
+        rows = wl.bf16_bits(q["emb"][miss])
+    want, amb = oracle.signatures(rows, wl.bf16_bits(R))
+    assert not np.any((_unpack(sig.cpu().numpy().view(np.uint32), 256) != want) & ~amb)
