@@ -113,7 +113,8 @@ typedef struct {
 } lacache_result;
 
 /* Create a cache on cfg->device with an empty store of cfg->capacity entries. Allocates the store
- * (capacity * (4d + 4k) bytes), the stage-1 scratch (about SMs * max_batch * top_c * 12 bytes) and host staging.
+ * (capacity * (2d + 2 * prefix row + 4k) bytes), the stage-1 scratch (2 * SMs * max_batch * (8 * top_c + 4)
+ * bytes) and host staging.
  * On success *out is a new handle; on failure *out is NULL and nothing stays allocated. */
 lacache_status lacache_create(const lacache_config* cfg, lacache_t** out);
 

@@ -32,6 +32,8 @@ struct lacache {
   int last_kernel;
   lc::EncodeTiledFn encode;
   int inject_stall;          // lookups left that withhold one stage-1 load (failure-detection tests)
+  int* tile_ctr;             // two tile counters of the dynamic stage-1 schedule, used alternately
+  int64_t tc_launches;       // tensor stage-1 launches so far (selects the counter)
   int lsh_bits;              // SimHash index: signature bits (0 = no index)
   int lsh_radius;
   uint32_t* sig;             // [capacity x lsh_bits/32] entry signatures
@@ -199,6 +201,7 @@ void free_all(lacache* h) {
   cudaFree(h->dev_status);
   cudaFree(h->append_dst);
   cudaFree(h->append_count);
+  cudaFree(h->tile_ctr);
   cudaFree(h->stage_in);
   cudaFree(h->stage_out);
   if (h->append_count_host) cudaFreeHost(h->append_count_host);
@@ -233,7 +236,12 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
     cudaError_t e;
     if (kernel == LACACHE_STAGE1_TENSOR) {
       if (!h->encode) return LACACHE_ERR_CUDA;
+      // launch i claims tiles from counter i % 2 and zeroes counter (i + 1) % 2, which served launch i - 1 (that
+      // launch has completed before this one touches memory)
+      a.tile_ctr = h->tile_ctr + (h->tc_launches & 1);
+      a.tile_ctr_next = h->tile_ctr + ((h->tc_launches + 1) & 1);
       e = lc::launch_stage1_tensor(a, h->encode, h->num_sms, h->max_splits, st, &splits);
+      if (e == cudaSuccess) ++h->tc_launches;
     } else if (kernel == LACACHE_STAGE1_LSH) {
       e = lc::launch_signatures(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, h->dev_status, h->encode, h->num_sms,
                                 st);
@@ -354,6 +362,8 @@ lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_
             cudaMalloc(&h->dev_status, 4) == cudaSuccess &&
             cudaMalloc(&h->append_dst, (size_t)c.max_batch * 4) == cudaSuccess &&
             cudaMalloc(&h->append_count, 4) == cudaSuccess &&
+            cudaMalloc(&h->tile_ctr, 2 * sizeof(int)) == cudaSuccess &&
+            cudaMemset(h->tile_ctr, 0, 2 * sizeof(int)) == cudaSuccess &&
             cudaMalloc(&h->stage_in, stage_in_bytes(c, pd)) == cudaSuccess &&
             cudaMalloc(&h->stage_out, stage_out_bytes(c, ens->m)) == cudaSuccess &&
             cudaMallocHost(&h->append_count_host, 4) == cudaSuccess &&

@@ -65,6 +65,8 @@ struct Stage1Args {
   float* part_best;
   unsigned int* dev_status;
   int inject_stall;           // test support: CTA 0 of the tensor kernel withholds one load (see lacache.h)
+  int* tile_ctr;              // tensor kernel, one query tile: dynamic tile schedule on this zeroed counter
+  int* tile_ctr_next;         // the counter the next launch will use; zeroed by this launch (nullptr: static)
 };
 
 struct Stage2Args {
@@ -117,7 +119,8 @@ struct LshArgs {
 cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits, cudaStream_t st,
                               int* splits);
 
-// Largest split count any stage-1 launcher uses for a given SM count (sizes the scratch).
-inline int max_splits_for(int num_sms) { return num_sms; }
+// Largest split count any stage-1 launcher uses for a given SM count (sizes the scratch): the SimHash scan runs two
+// CTAs per SM, the other kernels at most one split per SM.
+inline int max_splits_for(int num_sms) { return 2 * num_sms; }
 
 }  // namespace lc

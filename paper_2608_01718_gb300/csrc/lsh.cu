@@ -1,9 +1,9 @@
 // Stage 1 through the SimHash index (Eq. 1; Algorithm 1's "search semantic cache with key h(x)"): the key check
 // sim(x, x') >= tau_c applied only to the entries whose signature is within `radius` bits of the query's.
 //
-// One CTA per contiguous split of the entries; one entry per thread per tile of 256. A thread loads its entry's
-// signature (16-byte loads) and counts the differing bits against each of up to 16 query signatures held in shared
-// memory. Admitted (query, entry) pairs are queued in shared memory; when the queue is half full, and at the end
+// One CTA per contiguous split of the entries (two per SM); one entry per thread per tile of 512. A thread loads
+// its entry's signature (16-byte loads) and counts the differing bits against each of up to 8 query signatures
+// held in shared memory. Admitted (query, entry) pairs are queued in shared memory; when the queue is half full, and at the end
 // of the split, all warps take queue items two at a time and compute the exact fp32 score over the gathered key row
 // (each lane's 8-element chunks in order, then a butterfly sum). The warp of each query then folds the scores
 // that clear tau_c into that query's top-c list. The partial lists have the format of the other stage-1 kernels,
@@ -13,10 +13,10 @@
 namespace lc {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
-constexpr int kTile = 256;          // entries per tile, one per thread
-constexpr int kQC = 16;             // queries per pass over the entries
+constexpr int kTile = kThreads;     // entries per tile, one per thread
+constexpr int kQC = 8;              // queries per pass over the entries
 constexpr int kCap = 8192;          // queue capacity; a tile adds at most kTile * kQC = 4096 items
 constexpr unsigned kFull = 0xffffffffu;
 
@@ -185,7 +185,7 @@ cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStre
 cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits, cudaStream_t st,
                               int* splits) {
   const int64_t tiles = (a.n + kTile - 1) / kTile;
-  int s = (int)(tiles < (int64_t)num_sms ? tiles : (int64_t)num_sms);
+  int s = (int)(tiles < 2 * (int64_t)num_sms ? tiles : 2 * (int64_t)num_sms);
   if (s > max_splits) s = max_splits;
   if (s < 1) s = 1;
   *splits = s;

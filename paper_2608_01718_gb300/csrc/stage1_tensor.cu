@@ -18,7 +18,6 @@
 // Every mbarrier wait is bounded: on a timeout the CTA records LACACHE_ERR_DEVICE_TIMEOUT in the status word, the
 // other roles see an abort flag and stop, in-flight copies and MMAs are drained, TMEM is freed and the CTA exits.
 #include <cuda.h>
-#include <stdlib.h>
 #include <string.h>
 
 #include "internal.cuh"
@@ -37,10 +36,10 @@ constexpr int TMEM_COLS = 2 * BN;           // two accumulators
 constexpr int kThreads = 192;
 constexpr int kEpiWarps = 4;
 constexpr long long kWaitCycles = 2000000000LL;   // about one second of SM clock
-constexpr int kDefaultPrefetch = 0;
-constexpr int kBarriers = 2 * STAGES + 5;          // full, empty, tmem_full x2, tmem_empty x2, drain
+constexpr int RING = 4;                             // tile-index ring of the dynamic schedule
+constexpr int kBarriers = 2 * STAGES + 5 + 2 * RING;  // full, empty, tmem_full x2, tmem_empty x2, drain, ring
 constexpr size_t kStashBytes = 32 * 129 * 4;          // epilogue's rare-path chunk stash
-constexpr size_t kSmemBytes = 1024 + (size_t)STAGES * STAGE_BYTES + kBarriers * 8 + 16 + kStashBytes;
+constexpr size_t kSmemBytes = 1024 + (size_t)STAGES * STAGE_BYTES + kBarriers * 8 + 16 + RING * 4 + kStashBytes;
 
 // tcgen05 instruction descriptor, kind::f16: D f32 (bits 4-5 = 1), A bf16 (bits 7-9 = 1), B bf16 (bits 10-12 =
 // 1), A and B K-major (bits 15, 16 = 0), N >> 3 in bits 17-22, M >> 4 in bits 24-28.
@@ -59,8 +58,9 @@ struct TcParams {
   int64_t n_tiles;
   int k_steps;
   int a_rows;     // rows of the query box: B rounded up to 8 when B <= 128, else 128
-  int prefetch;   // key boxes prefetched into L2 ahead of the ring (0 = off)
   int inject_stall;  // test support: CTA 0 withholds its second load, so its MMA issuer's bounded wait runs out
+  int* tile_ctr;      // dynamic schedule: tile counter to claim from (nullptr: static schedule)
+  int* tile_ctr_next; // the other counter, zeroed here for the next launch (it served the previous one)
   uint32_t* sig;     // signature mode: [n x sig_words] output words
   int sig_words;
   uint64_t* part_cand;
@@ -108,12 +108,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
       ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
       : "memory");
-}
-// Bring a box into L2 without a shared-memory destination: raises the bytes in flight beyond the ring.
-__device__ __forceinline__ void tma_prefetch_l2(const CUtensorMap* map, int x, int y) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];"
-               ::"l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y)
-               : "memory");
 }
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
@@ -232,7 +226,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   const uint32_t b_smem = base + STAGES * A_BYTES;
   uint64_t* bars = reinterpret_cast<uint64_t*>(gbase + (size_t)STAGES * STAGE_BYTES);
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kBarriers);
-  float* stash = reinterpret_cast<float*>(tmem_slot + 4);
+  volatile int* tid_ring = reinterpret_cast<volatile int*>(tmem_slot + 4);
+  float* stash = reinterpret_cast<float*>(tmem_slot + 4 + RING);
   volatile uint32_t* abort_flag = tmem_slot + 1;
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
@@ -240,6 +235,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
   auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
   const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
+  auto tid_full_bar = [&](int r) { return bar0 + 8u * (2 * STAGES + 5 + r); };
+  auto tid_empty_bar = [&](int r) { return bar0 + 8u * (2 * STAGES + 5 + RING + r); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
@@ -253,6 +250,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(tempty_bar(b), kEpiWarps);
     }
     mbar_init(drain_bar, 1);
+    for (int r = 0; r < RING; ++r) {
+      mbar_init(tid_full_bar(r), 1);
+      mbar_init(tid_empty_bar(r), 1 + kEpiWarps);   // the MMA issuer and the four epilogue warps
+    }
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -280,43 +281,54 @@ __global__ void __launch_bounds__(kThreads, 1)
     atomicOr(p.dev_status, kDevTimeout);
   };
 
+  // Dynamic schedule (one query tile): the producer claims key tiles from a global counter and hands their
+  // indices to the MMA issuer and the epilogue through a small ring; a CTA's claims increase, so ids still arrive
+  // in increasing order. Static schedule: units (query tile, split of the key tiles) in a fixed order.
+  const bool dyn = p.tile_ctr != nullptr;
+  if (dyn && threadIdx.x == 0 && blockIdx.x == 0) *p.tile_ctr_next = 0;   // for the next launch (see TcParams)
+
   if (warp == 0) {
     if (lane == 0) {
       // ---------------- TMA producer ----------------
       uint32_t it = 0;
       bool ok = true;
       const uint32_t withheld = (p.inject_stall && blockIdx.x == 0) ? 1u : 0xFFFFFFFFu;
-      for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-        const int qt = u % p.q_tiles, sp = u / p.q_tiles;
-        const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
-        // L2 prefetch cursor, p.prefetch key boxes ahead of the loads within this unit's key range
-        int64_t pf_t = t_begin;
-        int pf_ks = 0;
-        auto pf_issue = [&]() {
-          if (pf_t < t_end) {
-            tma_prefetch_l2(&tmap_k, pf_ks * BK, (int)(pf_t * BN));
-            if (++pf_ks == p.k_steps) {
-              pf_ks = 0;
-              ++pf_t;
-            }
+      auto load_tile = [&](int qt, int64_t t) -> bool {
+        for (int ks = 0; ks < p.k_steps; ++ks, ++it) {
+          const int s = it % STAGES;
+          const uint32_t ph = (it / STAGES) & 1u;
+          if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) {
+            fail();
+            return false;
           }
-        };
-        for (int i = 0; i < p.prefetch; ++i) pf_issue();
-        for (int64_t t = t_begin; ok && t < t_end; ++t) {
-          for (int ks = 0; ks < p.k_steps; ++ks, ++it) {
-            if (p.prefetch) pf_issue();
-            const int s = it % STAGES;
-            const uint32_t ph = (it / STAGES) & 1u;
-            if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) {
-              fail();
-              ok = false;
-              break;
-            }
-            if (it == withheld) continue;   // nothing arrives on this stage: its consumer's wait runs out
-            mbar_expect_tx(full_bar(s), (uint32_t)(p.a_rows * BK * 2 + B_BYTES));
-            tma_load_2d(a_smem + s * A_BYTES, &tmap_q, full_bar(s), ks * BK, qt * BM);
-            tma_load_2d(b_smem + s * B_BYTES, &tmap_k, full_bar(s), ks * BK, (int)(t * BN));
+          if (it == withheld) continue;   // nothing arrives on this stage: its consumer's wait runs out
+          mbar_expect_tx(full_bar(s), (uint32_t)(p.a_rows * BK * 2 + B_BYTES));
+          tma_load_2d(a_smem + s * A_BYTES, &tmap_q, full_bar(s), ks * BK, qt * BM);
+          tma_load_2d(b_smem + s * B_BYTES, &tmap_k, full_bar(s), ks * BK, (int)(t * BN));
+        }
+        return true;
+      };
+      if (dyn) {
+        int64_t next = atomicAdd(p.tile_ctr, 1);
+        for (uint32_t r = 0; ok; ++r) {
+          const int64_t t = next;
+          const bool done = t >= p.n_tiles;
+          if (!done) next = atomicAdd(p.tile_ctr, 1);   // claim one ahead: hides the atomic's latency
+          const int slot = r % RING;
+          if (!mbar_wait(tid_empty_bar(slot), ((r / RING) & 1u) ^ 1u, abort_flag)) {
+            fail();
+            break;
           }
+          tid_ring[slot] = done ? -1 : (int)t;
+          mbar_arrive(tid_full_bar(slot));               // release: the index is visible to its readers
+          if (done) break;
+          ok = load_tile(0, t);
+        }
+      } else {
+        for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
+          const int qt = u % p.q_tiles, sp = u / p.q_tiles;
+          const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
+          for (int64_t t = t_begin; ok && t < t_end; ++t) ok = load_tile(qt, t);
         }
       }
       // drain: the last load issued into each stage has landed before the CTA may exit
@@ -329,34 +341,49 @@ __global__ void __launch_bounds__(kThreads, 1)
       // ---------------- MMA issuer ----------------
       uint32_t it = 0, tile_i = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-        const int sp = u / p.q_tiles;
-        const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
-        for (int64_t t = t_begin; ok && t < t_end; ++t, ++tile_i) {
-          const int b = tile_i & 1u;
-          if (!mbar_wait(tempty_bar(b), ((tile_i >> 1) & 1u) ^ 1u, abort_flag)) {
+      auto mma_tile = [&]() -> bool {
+        const int b = tile_i & 1u;
+        if (!mbar_wait(tempty_bar(b), ((tile_i >> 1) & 1u) ^ 1u, abort_flag)) {
+          fail();
+          return false;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem + (uint32_t)(b * BN);
+        for (int ks = 0; ks < p.k_steps; ++ks, ++it) {
+          const int s = it % STAGES;
+          if (!mbar_wait(full_bar(s), (it / STAGES) & 1u, abort_flag)) {
             fail();
-            ok = false;
-            break;
+            return false;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem + (uint32_t)(b * BN);
-          for (int ks = 0; ks < p.k_steps; ++ks, ++it) {
-            const int s = it % STAGES;
-            if (!mbar_wait(full_bar(s), (it / STAGES) & 1u, abort_flag)) {
-              fail();
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            const uint64_t ad = smem_desc(a_smem + s * A_BYTES);
-            const uint64_t bd = smem_desc(b_smem + s * B_BYTES);
+          const uint64_t ad = smem_desc(a_smem + s * A_BYTES);
+          const uint64_t bd = smem_desc(b_smem + s * B_BYTES);
 #pragma unroll
-            for (int kk = 0; kk < BK / 16; ++kk)
-              mma_bf16(d_tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), (ks | kk) != 0 ? 1u : 0u);
-            mma_commit(empty_bar(s));
+          for (int kk = 0; kk < BK / 16; ++kk)
+            mma_bf16(d_tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), (ks | kk) != 0 ? 1u : 0u);
+          mma_commit(empty_bar(s));
+        }
+        mma_commit(tfull_bar(b));
+        ++tile_i;
+        return true;
+      };
+      if (dyn) {
+        for (uint32_t r = 0; ok; ++r) {
+          const int slot = r % RING;
+          if (!mbar_wait(tid_full_bar(slot), (r / RING) & 1u, abort_flag)) {
+            fail();
+            break;
           }
-          if (ok) mma_commit(tfull_bar(b));
+          const int t = tid_ring[slot];
+          mbar_arrive(tid_empty_bar(slot));
+          if (t < 0) break;
+          ok = mma_tile();
+        }
+      } else {
+        for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
+          const int sp = u / p.q_tiles;
+          const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
+          for (int64_t t = t_begin; ok && t < t_end; ++t) ok = mma_tile();
         }
       }
       // drain: every MMA issued by this thread has completed before TMEM is freed
@@ -372,82 +399,107 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t tile_i = 0;
     bool ok = true;
     const unsigned full = 0xffffffffu;
-    for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-      const int qt = u % p.q_tiles, sp = u / p.q_tiles;
-      const int q = qt * BM + row;
-      const bool active = q < p.B;
-      const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
-      TopC<CPAD> top;
+    TopC<CPAD> top;
+    float best = -INFINITY;
+    // One finished accumulator: the 256 scores of key tile t for this thread's query row.
+    auto epi_tile = [&](int64_t t, bool active, int word) -> bool {
+      const int b = tile_i & 1u;
+      const uint32_t par = (tile_i >> 1) & 1u;
+      // every lane waits (each needs the barrier's acquire); the warp proceeds only if all lanes saw the phase
+      // complete, so the warp-collective tcgen05.ld below is never reached by part of a warp
+      const bool got = mbar_wait(tfull_bar(b), par, abort_flag);
+      if (!__all_sync(full, got)) {
+        if (lane == 0) fail();
+        return false;
+      }
+      tc_fence_after();
+      const int64_t j0 = t * BN;
+      const bool ragged = j0 + BN > p.n;
+#pragma unroll 1
+      for (int ch = 0; ch < BN / 32; ++ch) {
+        float v[32];
+        tmem_ld32(tmem + lane_addr + (uint32_t)(b * BN + ch * 32), v);
+        if constexpr (SIGN) {
+          // lane e keeps the word of key column jc + e: bit `lane` of it is this thread's hyperplane's sign
+          const int64_t jc = j0 + ch * 32;
+          uint32_t mine = 0;
+#pragma unroll
+          for (int e = 0; e < 32; ++e) {
+            const uint32_t w = __ballot_sync(full, v[e] >= 0.f);
+            if (lane == e) mine = w;
+          }
+          if (word < p.sig_words && jc + lane < p.n) p.sig[(jc + lane) * p.sig_words + word] = mine;
+        } else if (active) {
+          const int64_t jc = j0 + ch * 32;
+          if (ragged) {
+#pragma unroll
+            for (int e = 0; e < 32; ++e)
+              if (jc + e >= p.n) v[e] = -INFINITY;
+          }
+          float m = v[0];
+#pragma unroll
+          for (int e = 1; e < 32; ++e) m = fmaxf(m, v[e]);
+          best = fmaxf(best, m);
+          if (m >= top.thr) {
+            // rare path: stash the chunk in shared memory and insert the entries that clear the threshold
+            uint32_t mask = 0;
+#pragma unroll
+            for (int e = 0; e < 32; ++e) {
+              mask |= (v[e] >= top.thr ? 1u : 0u) << e;
+              my_stash[e * 129] = v[e];
+            }
+            while (mask) {
+              const int e = __ffs(mask) - 1;
+              mask &= mask - 1;
+              const float x = my_stash[e * 129];
+              if (x >= top.thr && jc + e < p.n) top.insert(x, (uint32_t)(jc + e), p.top_c);
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(tempty_bar(b));
+      ++tile_i;
+      return true;
+    };
+    auto write_partial = [&](int sp, int q) {
+      uint64_t* dst = p.part_cand + ((int64_t)sp * p.B + q) * p.top_c;
+#pragma unroll
+      for (int i = 0; i < CPAD; ++i)
+        if (i < p.top_c) dst[i] = i < top.count ? pack_cand(top.s[i], top.j[i]) : 0ull;
+      p.part_best[(int64_t)sp * p.B + q] = best;
+    };
+    if (dyn) {
+      const bool active = row < p.B;
       top.init(p.tau_c);
-      float best = -INFINITY;
-      const int word = (qt * BM + quad * 32) / 32;   // signature mode: this warp's word of every signature
-      for (int64_t t = t_begin; t < t_end; ++t, ++tile_i) {
-        const int b = tile_i & 1u;
-        const uint32_t par = (tile_i >> 1) & 1u;
-        // every lane waits (each needs the barrier's acquire); the warp proceeds only if all lanes saw the
-        // phase complete, so the warp-collective tcgen05.ld below is never reached by part of a warp
-        const bool got = mbar_wait(tfull_bar(b), par, abort_flag);
+      best = -INFINITY;
+      for (uint32_t r = 0; ok; ++r) {
+        const int slot = r % RING;
+        const bool got = mbar_wait(tid_full_bar(slot), (r / RING) & 1u, abort_flag);
         if (!__all_sync(full, got)) {
           if (lane == 0) fail();
           ok = false;
           break;
         }
-        tc_fence_after();
-        const int64_t j0 = t * BN;
-        const bool ragged = j0 + BN > p.n;
-#pragma unroll 1
-        for (int ch = 0; ch < BN / 32; ++ch) {
-          float v[32];
-          tmem_ld32(tmem + lane_addr + (uint32_t)(b * BN + ch * 32), v);
-          if constexpr (SIGN) {
-            // lane e keeps the word of key column jc + e: bit `lane` of it is this thread's hyperplane's sign
-            const int64_t jc = j0 + ch * 32;
-            uint32_t mine = 0;
-#pragma unroll
-            for (int e = 0; e < 32; ++e) {
-              const uint32_t w = __ballot_sync(full, v[e] >= 0.f);
-              if (lane == e) mine = w;
-            }
-            if (word < p.sig_words && jc + lane < p.n) p.sig[(jc + lane) * p.sig_words + word] = mine;
-          } else if (active) {
-            const int64_t jc = j0 + ch * 32;
-            if (ragged) {
-#pragma unroll
-              for (int e = 0; e < 32; ++e)
-                if (jc + e >= p.n) v[e] = -INFINITY;
-            }
-            float m = v[0];
-#pragma unroll
-            for (int e = 1; e < 32; ++e) m = fmaxf(m, v[e]);
-            best = fmaxf(best, m);
-            if (m >= top.thr) {
-              // rare path: stash the chunk in shared memory and insert the entries that clear the threshold
-              uint32_t mask = 0;
-#pragma unroll
-              for (int e = 0; e < 32; ++e) {
-                mask |= (v[e] >= top.thr ? 1u : 0u) << e;
-                my_stash[e * 129] = v[e];
-              }
-              while (mask) {
-                const int e = __ffs(mask) - 1;
-                mask &= mask - 1;
-                const float x = my_stash[e * 129];
-                if (x >= top.thr && jc + e < p.n) top.insert(x, (uint32_t)(jc + e), p.top_c);
-              }
-            }
-          }
-        }
-        tc_fence_before();
+        const int t = tid_ring[slot];
         __syncwarp();
-        if (lane == 0) mbar_arrive(tempty_bar(b));
+        if (lane == 0) mbar_arrive(tid_empty_bar(slot));
+        if (t < 0) break;
+        ok = epi_tile(t, active, 0);
       }
-      if (!ok) break;
-      if (active && !SIGN) {
-        uint64_t* dst = p.part_cand + ((int64_t)sp * p.B + q) * p.top_c;
-#pragma unroll
-        for (int i = 0; i < CPAD; ++i)
-          if (i < p.top_c) dst[i] = i < top.count ? pack_cand(top.s[i], top.j[i]) : 0ull;
-        p.part_best[(int64_t)sp * p.B + q] = best;
+      if (ok && active && !SIGN) write_partial(blockIdx.x, row);
+    } else {
+      for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
+        const int qt = u % p.q_tiles, sp = u / p.q_tiles;
+        const int q = qt * BM + row;
+        const bool active = q < p.B;
+        const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
+        const int word = (qt * BM + quad * 32) / 32;   // signature mode: this warp's word of every signature
+        top.init(p.tau_c);
+        best = -INFINITY;
+        for (int64_t t = t_begin; ok && t < t_end; ++t) ok = epi_tile(t, active, word);
+        if (ok && active && !SIGN) write_partial(sp, q);
       }
     }
   }
@@ -458,18 +510,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
   }
-}
-
-// Key boxes to prefetch into L2 ahead of the shared-memory ring. LACACHE_TC_PREFETCH overrides the default
-// (a tuning knob; any value gives the same results).
-int prefetch_distance() {
-  static int value = -1;
-  if (value < 0) {
-    const char* env = getenv("LACACHE_TC_PREFETCH");
-    int v = env ? atoi(env) : kDefaultPrefetch;
-    value = v < 0 ? 0 : (v > 64 ? 64 : v);
-  }
-  return value;
 }
 
 int gcd_int(int a, int b) {
@@ -527,7 +567,6 @@ cudaError_t launch_signatures(const __nv_bfloat16* rows, int64_t n, int d, const
   p.q_tiles = (bits + BM - 1) / BM;
   p.n_tiles = (n + BN - 1) / BN;
   p.k_steps = (d + BK - 1) / BK;
-  p.prefetch = 0;
   p.a_rows = bits >= BM ? BM : ((bits + 7) / 8) * 8;
   int s = num_sms / gcd_int(num_sms, p.q_tiles);
   if ((int64_t)s > p.n_tiles) s = (int)p.n_tiles;
@@ -556,7 +595,6 @@ cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int 
   p.q_tiles = (a.B + BM - 1) / BM;
   p.n_tiles = (a.n + BN - 1) / BN;
   p.k_steps = (a.d + BK - 1) / BK;
-  p.prefetch = prefetch_distance();
   // A batch of at most 128 queries is loaded as a box of B rows (rounded up to 8) rather than 128: boxes that
   // are mostly out of bounds stream measurably slower. The MMA still computes 128 rows; rows past B hold stale
   // shared memory and their TMEM lanes are never read.
@@ -565,13 +603,18 @@ cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int 
   if (!encode_rows(encode, &tq, a.q, a.d, a.B, (uint32_t)p.a_rows) ||
       !encode_rows(encode, &tk, a.keys, a.d, a.n, (uint32_t)BN))
     return cudaErrorInvalidValue;
-  // splits such that q_tiles * splits is a multiple of the SM count (whole waves of units)
+  // splits such that q_tiles * splits is a multiple of the SM count (whole waves of units); one query tile with
+  // a tile counter: a dynamic schedule with one split per CTA
   int s = num_sms / gcd_int(num_sms, p.q_tiles);
   if ((int64_t)s > p.n_tiles) s = (int)p.n_tiles;
   if (s > max_splits) s = max_splits;
   if (s < 1) s = 1;
   p.splits = s;
   p.units = p.q_tiles * s;
+  if (p.q_tiles == 1 && a.tile_ctr) {
+    p.tile_ctr = a.tile_ctr;
+    p.tile_ctr_next = a.tile_ctr_next;
+  }
   p.part_cand = a.part_cand;
   p.part_best = a.part_best;
   p.dev_status = a.dev_status;
