@@ -13,7 +13,9 @@ from .lookup import (CHECK_BOTH, CHECK_EMB, CHECK_TOKENS, HIT, MISS_KEY, REJECT,
 from .serve import ServeLoop
 from .calibrate import calibrate, nearest_rank, pair_similarities
 from .lsh import hamming, lookup_lsh, projections, signatures
+from .speculative import accepted_prefix
 
 __all__ = ["round_to_bf16", "widen", "CHECK_BOTH", "CHECK_EMB", "CHECK_TOKENS", "HIT", "MISS_KEY", "REJECT",
            "KeyCheck", "Params", "Result", "Store", "decide", "lookahead", "lookup", "passes", "ServeLoop",
-           "calibrate", "nearest_rank", "pair_similarities", "hamming", "lookup_lsh", "projections", "signatures"]
+           "calibrate", "nearest_rank", "pair_similarities", "hamming", "lookup_lsh", "projections", "signatures",
+           "accepted_prefix"]
