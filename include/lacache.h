@@ -237,6 +237,15 @@ lacache_status lacache_calibrate(int64_t n, int32_t d, const void* x_dev, const 
                                  void* cuda_stream);
 size_t lacache_calibrate_workspace_bytes(void);
 
+/* Reuse of the lookahead prefix on a miss (section 3.3, "Speculative Decoding"). A query that is not served has
+ * its k draft tokens f_k(x) verified by the target model in one forward pass: from the first token on, draft token
+ * t is accepted if P_f(t) >= P_g(t), and the first rejection hands decoding to the target model. Given
+ * p_target_dev and p_draft_dev ([B x k] floats: each model's probability of each draft token), writes
+ * accepted_dev[q] = the number of leading accepted tokens, or -1 where status_dev[q] == LACACHE_HIT (a served query
+ * decodes nothing). status_dev may be NULL (every query verified). Asynchronous on cuda_stream. */
+lacache_status lacache_verify_draft(int32_t B, int32_t k, const float* p_target_dev, const float* p_draft_dev,
+                                    const uint8_t* status_dev, int32_t* accepted_dev, void* cuda_stream);
+
 /* Static description of a status code. */
 const char* lacache_status_string(lacache_status s);
 

@@ -22,7 +22,7 @@ LACACHE_MAX_MODELS = 8
 
 EXPORTS = ["lacache_create", "lacache_create_ensemble", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
            "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
-           "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_enable_lsh", "lacache_read_signatures", "lacache_calibrate", "lacache_calibrate_workspace_bytes",
+           "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_enable_lsh", "lacache_read_signatures", "lacache_calibrate", "lacache_calibrate_workspace_bytes", "lacache_verify_draft",
            "lacache_lookup_noalloc",
            "lacache_status_string"]
 
@@ -86,6 +86,7 @@ def load() -> ctypes.CDLL:
         "lacache_read_signatures": ([vp, i64, i64, vp, vp], i32),
         "lacache_calibrate": ([i64, i32, vp, vp, ctypes.c_double, ctypes.c_float, vp, vp, vp, vp], i32),
         "lacache_calibrate_workspace_bytes": ([], ctypes.c_size_t),
+        "lacache_verify_draft": ([i32, i32, vp, vp, vp, vp, vp], i32),
         "lacache_lookup_noalloc": ([ctypes.POINTER(lacache_config), i64, vp, vp, vp, i32, vp, vp, vp,
                                     ctypes.POINTER(lacache_result), vp], i32),
         "lacache_status_string": ([i32], ctypes.c_char_p),
@@ -244,6 +245,13 @@ def lacache_calibrate(x, y, percentile: float, cap: float, sims, result, workspa
     _check("lacache_calibrate", load().lacache_calibrate(int(x.shape[0]), int(x.shape[1]), _ptr(x), _ptr(y),
                                                          float(percentile), float(cap), _ptr(sims), _ptr(result),
                                                          _ptr(workspace), _stream(cuda_stream)))
+
+
+def lacache_verify_draft(p_target, p_draft, status, accepted, cuda_stream=None) -> None:
+    """Accepted draft-prefix length per query (P_f >= P_g from the first token on); -1 for served queries."""
+    B, k = int(p_target.shape[0]), int(p_target.shape[1])
+    _check("lacache_verify_draft", load().lacache_verify_draft(B, k, _ptr(p_target), _ptr(p_draft), _ptr(status),
+                                                               _ptr(accepted), _stream(cuda_stream)))
 
 
 def lacache_lookup_noalloc(cfg: lacache_config, key, prefix, ids, q_emb, q_prefix, q_ids, out: dict,

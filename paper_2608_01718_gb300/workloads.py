@@ -299,3 +299,13 @@ def lsh_radius(tau_c: float, bits: int, z: float = 4.0) -> int:
     theta = math.acos(max(-1.0, min(1.0, tau_c)))
     p = theta / math.pi
     return min(bits, int(math.ceil(bits * p + z * math.sqrt(bits * p * (1 - p)))))
+
+
+def draft_probabilities(batch: int, k: int, seed: int = 20260801, device="cpu"):
+    """Stand-ins for the target's and the draft's probabilities of each of the k draft tokens, [batch x k] fp32:
+    correlated uniforms, so that acceptance runs of every length occur."""
+    g = torch.Generator(device=device)
+    g.manual_seed(sub_seed(seed, f"draft/{batch}/{k}", 0))
+    pg = torch.rand((batch, k), generator=g, device=device)
+    pf = (pg + 0.2 * torch.randn((batch, k), generator=g, device=device) + 0.3).clamp(0.0, 1.0)
+    return pf.contiguous(), pg.contiguous()

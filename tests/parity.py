@@ -92,6 +92,12 @@ class Report:
             setattr(self, f.name, getattr(self, f.name) + getattr(other, f.name))
 
 
+def log_report(name: str, rep: Report) -> None:
+    """One line per parity case (visible with pytest -s): what was compared and what fell in the margin band."""
+    print(f"PARITY {name}: queries={rep.queries} exact={rep.exact} band={rep.band} literal_band={rep.literal_band} "
+          f"hits={rep.hits} rejects={rep.rejects} misses={rep.misses} near_ties={rep.near_ties}", flush=True)
+
+
 def _close(a, b, tol=TOL) -> bool:
     if np.isnan(a) and np.isnan(b):
         return True

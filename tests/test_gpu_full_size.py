@@ -14,8 +14,8 @@ from paper_2608_01718_gb300 import build
 from paper_2608_01718_gb300 import lacache as L
 from paper_2608_01718_gb300 import workloads as wl
 
-from parity import (TOL, StreamedOracle, compare, fill, new_cache, oracle_queries, oracle_store, params,
-                    stratified_sample)
+from parity import (TOL, Report, StreamedOracle, compare, fill, log_report, new_cache, oracle_queries, oracle_store,
+                    params, stratified_sample)
 
 pytestmark = [pytest.mark.gpu, pytest.mark.slow]
 
@@ -42,6 +42,7 @@ def _check_streamed(w, per_class):
         g = {k: v.cpu().numpy() for k, v in out.items()}
     res = so.result()
     rep = compare(g, res, p, rows=sample, pair_scores=so.pair_scores)
+    log_report(f"{w.name} full size, sampled", rep)
     assert rep.exact + rep.band == len(sample)
     assert rep.band <= max(1, len(sample) // 50)
     assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
@@ -75,6 +76,7 @@ def test_serve_loop_thousand_steps():
     del st
     origin = {}          # appended entry id -> (step, query index) of the query it holds
     hits_checked = 0
+    replayed = Report()
     with new_cache(w, L.LACACHE_STAGE1_TENSOR, capacity=capacity) as cache:
         fill(cache, w)
         for step in range(w.steps):
@@ -99,11 +101,15 @@ def test_serve_loop_thousand_steps():
                 g = {k: v.cpu().numpy() for k, v in out.items()}
                 res, ofirst, om = loop.step(oracle_queries(q))
                 rep = compare(g, res, p)
+                replayed.add(rep)
                 assert rep.band == 0 and (ofirst, om) == (first, m)
             if step % 97 == 0:
                 hits_checked += _check_hits(w, p, q, out, origin)
         assert cache.size > w.n + 100 * w.steps
         assert hits_checked > 100
+    log_report(f"{w.name} oracle-replayed steps 0-{replay - 1}", replayed)
+    print(f"PARITY {w.name}: {w.steps} steps, final size {w.n + len(origin)}, HITs checked {hits_checked}",
+          flush=True)
 
 
 def _check_hits(w, p, q, out, origin):

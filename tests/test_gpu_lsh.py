@@ -12,7 +12,7 @@ from paper_2608_01718_gb300 import build
 from paper_2608_01718_gb300 import lacache as L
 from paper_2608_01718_gb300 import workloads as wl
 
-from parity import compare, fill, gpu_lookup, new_cache, oracle_queries, oracle_store, params
+from parity import compare, fill, gpu_lookup, log_report, new_cache, oracle_queries, oracle_store, params
 
 pytestmark = pytest.mark.gpu
 
@@ -68,6 +68,7 @@ def test_lsh_lookup_matches_the_oracle(bits):
     keep = np.nonzero(~amb)[0]
     sub = oracle.Result(**{f: getattr(res, f)[keep] for f in res.__dataclass_fields__})
     rep = compare(g, sub, p, rows=keep)
+    log_report(f"lsh bits={bits} radius={radius} ({w.batch - len(keep)} queries with ambiguous bits)", rep)
     assert rep.exact + rep.band == len(keep) and len(keep) >= w.batch - 2
     assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
     # at this radius the index keeps every near-duplicate's target: the decisions equal the exact lookup's

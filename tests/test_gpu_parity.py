@@ -15,8 +15,8 @@ from paper_2608_01718_gb300 import build
 from paper_2608_01718_gb300 import lacache as L
 from paper_2608_01718_gb300 import workloads as wl
 
-from parity import (TOL, Report, compare, fill, gpu_lookup, new_cache, oracle_queries, oracle_store, pair_scores_fn,
-                    params)
+from parity import (TOL, Report, compare, fill, gpu_lookup, log_report, new_cache, oracle_queries, oracle_store,
+                    pair_scores_fn, params)
 
 pytestmark = pytest.mark.gpu
 
@@ -46,6 +46,7 @@ def run_parity(w, stage1, check_mode=oracle.CHECK_EMB, token_match_min=None, ste
             p = params(w, check_mode, token_match_min)
             res = oracle.lookup(st, oq, p)
             rep.add(compare(g, res, p, pair_scores=pair_scores_fn(st, oq)))
+    log_report(f"{w.name} n={w.n} B={w.batch} stage1={stage1} mode={check_mode}", rep)
     return rep
 
 
@@ -111,6 +112,7 @@ def test_ensemble_full_size_rejects_prefix_mimics():
     oq = oracle_queries(q)
     p = params(w)
     rep = compare(g, oracle.lookup(st, oq, p), p, pair_scores=pair_scores_fn(st, oq))
+    log_report(f"{w.name} full size", rep)
     assert rep.exact + rep.band == w.batch and rep.band <= 1
     cls = q["class"].numpy()
     assert np.all(g["status"][cls == wl.MIMIC] == L.LACACHE_REJECT)
