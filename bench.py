@@ -32,7 +32,7 @@ sys.path.insert(0, ROOT)
 METRIC = "lookups/sec at 1 GB300 (N entries, batch B, k) + % of HBM or bf16 roofline"
 UNIT = "queries/s"
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "simt": "stage1_simt.cu", "lsh": "lsh.cu"}
+STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "tensor-pair": "stage1_tensor.cu", "simt": "stage1_simt.cu", "lsh": "lsh.cu"}
 
 
 def parse_args():
@@ -47,6 +47,8 @@ def parse_args():
     ap.add_argument("--batches", type=int, default=8, help="distinct query batches cycled through")
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--entries", type=int, default=0,
+                    help="store size override: a smaller case of the workload (profiling captures)")
     return ap.parse_args()
 
 
@@ -286,7 +288,8 @@ def run_ours(args, w):
         step(i)
     torch.cuda.synchronize()
     cache.sync()
-    kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_SIMT: "simt",
+    kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_TENSOR_PAIR: "tensor-pair",
+                   L.LACACHE_STAGE1_SIMT: "simt",
                    L.LACACHE_STAGE1_LSH: "lsh"}[cache.last_launch()[1]]
     if world > 1:
         dist.barrier()
@@ -443,6 +446,8 @@ def main():
     if args.workload in CALIBRATION:
         return run_calibration(args)
     w = wl.WORKLOADS[args.workload]
+    if args.entries:
+        w = w.scaled(n=args.entries)
     if args.impl == "reference":
         return run_reference(args, w)
     return run_ours(args, w)

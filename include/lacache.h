@@ -62,7 +62,10 @@ typedef enum {
   LACACHE_STAGE1_AUTO = 0,
   LACACHE_STAGE1_TENSOR = 1, /* tcgen05 tensor-core scan (TMA-fed, TMEM accumulators) */
   LACACHE_STAGE1_SIMT = 2,   /* CUDA-core FFMA scan */
-  LACACHE_STAGE1_LSH = 3     /* SimHash index, then the exact key check (requires lacache_enable_lsh) */
+  LACACHE_STAGE1_LSH = 3,    /* SimHash index, then the exact key check (requires lacache_enable_lsh) */
+  LACACHE_STAGE1_TENSOR_PAIR = 4 /* reported by lacache_last_launch only, not a configuration value: the tensor
+                                    scan on two-CTA clusters (one M=256 MMA per pair of SMs), chosen for batches of
+                                    more than 128 queries */
 } lacache_stage1;
 
 /* Ensemble of m lookahead checks (section 3.4, "Analysis"; Figure 6): every entry and query carries one k-token
@@ -183,7 +186,8 @@ lacache_status lacache_size(const lacache_t* h, int64_t* n);
  * previous lacache_sync (the status word is then cleared). */
 lacache_status lacache_sync(lacache_t* h);
 
-/* Number of stage-1 partial lists the last lookup used, and which stage-1 kernel it ran (lacache_stage1). */
+/* Number of stage-1 partial lists the last lookup used, and which stage-1 kernel it ran (lacache_stage1; a
+ * tensor-core lookup reports LACACHE_STAGE1_TENSOR or LACACHE_STAGE1_TENSOR_PAIR). */
 lacache_status lacache_last_launch(const lacache_t* h, int32_t* n_splits, int32_t* stage1_kernel);
 
 /* Stage timing (measurement). lacache_stage_timing(h, m) with m > 0 makes the next m lookups record CUDA events

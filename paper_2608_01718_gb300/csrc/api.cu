@@ -240,8 +240,10 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
       // launch has completed before this one touches memory)
       a.tile_ctr = h->tile_ctr + (h->tc_launches & 1);
       a.tile_ctr_next = h->tile_ctr + ((h->tc_launches + 1) & 1);
-      e = lc::launch_stage1_tensor(a, h->encode, h->num_sms, h->max_splits, st, &splits);
+      bool paired = false;
+      e = lc::launch_stage1_tensor(a, h->encode, h->num_sms, h->max_splits, st, &splits, &paired);
       if (e == cudaSuccess) ++h->tc_launches;
+      if (paired) kernel = LACACHE_STAGE1_TENSOR_PAIR;
     } else if (kernel == LACACHE_STAGE1_LSH) {
       e = lc::launch_signatures(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, h->dev_status, h->encode, h->num_sms,
                                 st);

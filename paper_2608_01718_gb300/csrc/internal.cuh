@@ -98,8 +98,9 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
 // Launchers (host). Each returns the CUDA error of the launch. `splits` is the number of partial lists written.
 cudaError_t launch_stage1_simt(const Stage1Args& a, int num_sms, int max_splits, cudaStream_t st, int* splits);
 // Encodes its own TMA descriptors for a.q and a.keys with `encode`.
+// *paired (if not null) is set when the batch ran on CTA pairs.
 cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int num_sms, int max_splits,
-                                 cudaStream_t st, int* splits);
+                                 cudaStream_t st, int* splits, bool* paired = nullptr);
 cudaError_t launch_stage2(const Stage2Args& a, cudaStream_t st);
 
 // SimHash signatures of n rows ([n x d] bf16) against `bits` hyperplanes ([bits x d] bf16), bits a multiple of 32:

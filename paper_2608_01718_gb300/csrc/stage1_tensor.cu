@@ -15,6 +15,13 @@
 //   warps 2..5  epilogue: thread = query row (TMEM lane); reads its 256 scores with tcgen05.ld, keeps a sorted
 //               top_c of (score, id) in registers with the threshold max(tau_c, current c-th best), and finally
 //               writes the unit's partial list. Double-buffered accumulators overlap it with the next tile's MMAs.
+// Batches of more than one query tile run as CTA pairs (a two-CTA cluster on the two SMs of a TPC): one
+// tcgen05.mma.cta_group::2 of M=256 (two query tiles, one per SM), N=256, K=16 per step. Each SM loads its own
+// 128x64 query box and HALF of the key box (128 keys); the pair's tensor cores exchange the key halves, and each
+// SM's TMEM receives its own 128 query rows x 256 keys. Per SM and k-step that is 32 KB of TMA writes and of MMA
+// operand reads instead of 48 KB, and each key tile is read once per pair of query tiles. The leader CTA (rank 0)
+// issues the MMAs; both CTAs' loads complete on the leader's full barrier, its commits arrive on both CTAs'
+// empty and tmem_full barriers, and both CTAs' epilogues release an accumulator on the leader's tmem_empty.
 // Every mbarrier wait is bounded: on a timeout the CTA records LACACHE_ERR_DEVICE_TIMEOUT in the status word, the
 // other roles see an abort flag and stop, in-flight copies and MMAs are drained, TMEM is freed and the CTA exits.
 #include <cuda.h>
@@ -28,23 +35,31 @@ namespace {
 constexpr int BM = 128;                     // queries per tile (TMEM lanes)
 constexpr int BN = 256;                     // keys per tile (accumulator columns)
 constexpr int BK = 64;                      // bf16 per k-step = one 128-byte swizzled row
-constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;        // 16 KB
-constexpr int B_BYTES = BN * BK * 2;        // 32 KB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int TMEM_COLS = 2 * BN;           // two accumulators
 constexpr int kThreads = 192;
 constexpr int kEpiWarps = 4;
 constexpr long long kWaitCycles = 2000000000LL;   // about one second of SM clock
 constexpr int RING = 4;                             // tile-index ring of the dynamic schedule
-constexpr int kBarriers = 2 * STAGES + 5 + 2 * RING;  // full, empty, tmem_full x2, tmem_empty x2, drain, ring
 constexpr size_t kStashBytes = 32 * 129 * 4;          // epilogue's rare-path chunk stash
-constexpr size_t kSmemBytes = 1024 + (size_t)STAGES * STAGE_BYTES + kBarriers * 8 + 16 + RING * 4 + kStashBytes;
 
-// tcgen05 instruction descriptor, kind::f16: D f32 (bits 4-5 = 1), A bf16 (bits 7-9 = 1), B bf16 (bits 10-12 =
-// 1), A and B K-major (bits 15, 16 = 0), N >> 3 in bits 17-22, M >> 4 in bits 24-28.
-constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-                            ((uint32_t)(BM >> 4) << 24);
+// Per-CTA geometry. Single CTA: the whole 256-key box per stage, 4 stages. CTA pair: half the key box, so 6
+// stages fit in the same shared memory.
+template <bool PAIR>
+struct Geo {
+  static constexpr int kStages = PAIR ? 6 : 4;
+  static constexpr int kBRows = PAIR ? BN / 2 : BN;        // key rows this CTA loads per tile
+  static constexpr int kBBytes = kBRows * BK * 2;
+  static constexpr int kStageBytes = A_BYTES + kBBytes;
+  // full, empty, tmem_full x2, tmem_empty x2, drain, ring full/empty
+  static constexpr int kBarriers = 2 * kStages + 5 + 2 * RING;
+  static constexpr size_t kSmem = 1024 + (size_t)kStages * kStageBytes + kBarriers * 8 + 16 + RING * 4 + kStashBytes;
+  // tcgen05 instruction descriptor, kind::f16: D f32 (bits 4-5 = 1), A bf16 (bits 7-9 = 1), B bf16 (bits 10-12
+  // = 1), A and B K-major (bits 15, 16 = 0), N >> 3 in bits 17-22, M >> 4 in bits 24-28 (M = 256 for the pair).
+  static constexpr uint32_t kIdesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+                                     ((uint32_t)((PAIR ? 2 * BM : BM) >> 4) << 24);
+};
+static_assert(Geo<false>::kSmem <= 227 * 1024 && Geo<true>::kSmem <= 227 * 1024, "shared memory budget");
 
 struct TcParams {
   int64_t n;
@@ -53,6 +68,7 @@ struct TcParams {
   float tau_c;
   int top_c;
   int q_tiles;
+  int pairs;      // CTA-pair schedule: query-tile pairs (ceil(q_tiles / 2)); units are (pair, split)
   int splits;
   int units;
   int64_t n_tiles;
@@ -92,9 +108,8 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-// Wait for the phase of the given parity to complete; false after about a second, or when another role aborted.
-__device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const volatile uint32_t* abort_flag) {
-  if (mbar_try_wait(bar, parity)) return true;
+// Slow path of mbar_wait: poll until the phase completes, about a second passes, or another role aborts.
+__device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, const volatile uint32_t* abort_flag) {
   const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -103,11 +118,53 @@ __device__ __noinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const vola
   }
 }
 
+// Wait for the phase of the given parity to complete; false after about a second, or when another role aborted.
+// The first probe is inline: on the MMA issuer's path the phase has usually completed already, and an
+// out-of-line call per k-step costs measurable tensor-pipe time (about a sixth of the MMA rate at N = 256).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const volatile uint32_t* abort_flag) {
+  return mbar_try_wait(bar, parity) || mbar_wait_slow(bar, parity, abort_flag);
+}
+
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
   asm volatile(
       "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];"
       ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
       : "memory");
+}
+// CTA-pair form: the destination is this CTA's shared memory, the mbarrier may be the peer's (the leader's).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap* map, uint32_t bar, int x, int y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3}], [%4];"
+      ::"r"(dst), "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_id_x() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ uint32_t cluster_count_x() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+  return r;
+}
+// Address of the same shared-memory variable in the cluster CTA of the given rank.
+__device__ __forceinline__ uint32_t map_to_rank(uint32_t addr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
 __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
@@ -116,28 +173,59 @@ __device__ __forceinline__ void tma_prefetch_desc(const CUtensorMap* map) {
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
+// TMEM allocation: one warp of the CTA (cta_group::1), or one warp of each CTA of the pair collectively
+// (cta_group::2: the same columns in both SMs).
+template <bool PAIR>
 __device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
-               : "memory");
+  if constexpr (PAIR)
+    asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+                 : "memory");
+  else
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+                 : "memory");
 }
+template <bool PAIR>
 __device__ __forceinline__ void tmem_relinquish() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  if constexpr (PAIR)
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+  else
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
 }
+template <bool PAIR>
 __device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+  if constexpr (PAIR)
+    asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+  else
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
 }
 
+template <bool PAIR>
 __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t accumulate) {
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "setp.ne.b32 p, %4, 0;\n\t"
-      "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
-      ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(kIdesc), "r"(accumulate)
-      : "memory");
+  if constexpr (PAIR)
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(Geo<true>::kIdesc), "r"(accumulate)
+        : "memory");
+  else
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}"
+        ::"r"(d_tmem), "l"(a_desc), "l"(b_desc), "r"(Geo<false>::kIdesc), "r"(accumulate)
+        : "memory");
 }
-__device__ __forceinline__ void mma_commit(uint32_t bar) {
-  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-               : "memory");
+// Arrives once on `bar` when every MMA this thread issued so far has completed. The pair form arrives on the
+// barrier at the same offset in each CTA of `cta_mask`.
+template <bool PAIR>
+__device__ __forceinline__ void mma_commit(uint32_t bar, uint16_t cta_mask) {
+  if constexpr (PAIR)
+    asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;"
+                 ::"r"(bar), "h"(cta_mask) : "memory");
+  else
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
 }
 
 // Shared-memory matrix descriptor of a K-major operand tile written by TMA with 128-byte swizzle: rows of 128 B,
@@ -214,40 +302,44 @@ struct TopC {
 // SIGN = false: the key check (threshold + top-c partial lists). SIGN = true: the same GEMM with random hyperplanes
 // in place of the queries, and an epilogue that writes SimHash signatures: bit h of row j's signature is set iff
 // <r_h, row_j> >= 0; each warp's 32 hyperplanes form one 32-bit word, packed with a ballot per key column.
-template <int CPAD, bool SIGN>
+// PAIR = true: launched as two-CTA clusters, static schedule over (query-tile pair, split) units.
+template <int CPAD, bool SIGN, bool PAIR>
 __global__ void __launch_bounds__(kThreads, 1)
     stage1_tensor_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
                          const TcParams p) {
+  using G = Geo<PAIR>;
+  constexpr int S = G::kStages;
   extern __shared__ unsigned char smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   unsigned char* gbase = smem_raw + (base - raw);
   const uint32_t a_smem = base;
-  const uint32_t b_smem = base + STAGES * A_BYTES;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(gbase + (size_t)STAGES * STAGE_BYTES);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + kBarriers);
+  const uint32_t b_smem = base + S * A_BYTES;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(gbase + (size_t)S * G::kStageBytes);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + G::kBarriers);
   volatile int* tid_ring = reinterpret_cast<volatile int*>(tmem_slot + 4);
   float* stash = reinterpret_cast<float*>(tmem_slot + 4 + RING);
   volatile uint32_t* abort_flag = tmem_slot + 1;
   const uint32_t bar0 = smem_u32(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
-  auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
-  auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
-  auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
-  const uint32_t drain_bar = bar0 + 8u * (2 * STAGES + 4);
-  auto tid_full_bar = [&](int r) { return bar0 + 8u * (2 * STAGES + 5 + r); };
-  auto tid_empty_bar = [&](int r) { return bar0 + 8u * (2 * STAGES + 5 + RING + r); };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (S + s); };
+  auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * S + b); };
+  auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * S + 2 + b); };
+  const uint32_t drain_bar = bar0 + 8u * (2 * S + 4);
+  auto tid_full_bar = [&](int r) { return bar0 + 8u * (2 * S + 5 + r); };
+  auto tid_empty_bar = [&](int r) { return bar0 + 8u * (2 * S + 5 + RING + r); };
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = PAIR ? cluster_rank() : 0u;   // 0: leader (issues the MMAs)
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), 1);
+    for (int s = 0; s < S; ++s) {
+      mbar_init(full_bar(s), 1);    // the (leader's) producer's arrive; both CTAs' bytes complete it
+      mbar_init(empty_bar(s), 1);   // the (leader's) MMA commit
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull_bar(b), 1);
-      mbar_init(tempty_bar(b), kEpiWarps);
+      mbar_init(tempty_bar(b), (PAIR ? 2 : 1) * kEpiWarps);   // the epilogue warps of both CTAs of a pair
     }
     mbar_init(drain_bar, 1);
     for (int r = 0; r < RING; ++r) {
@@ -262,9 +354,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tmap_q);
     tma_prefetch_desc(&tmap_k);
   }
+  // A pair: both CTAs' barriers are initialised, and both CTAs are running, before either touches the other's
+  // shared memory or allocates the pair's TMEM.
+  if constexpr (PAIR) cluster_sync();
   if (warp == 1) {
-    tmem_alloc(smem_u32(tmem_slot), TMEM_COLS);
-    tmem_relinquish();
+    tmem_alloc<PAIR>(smem_u32(tmem_slot), TMEM_COLS);
+    tmem_relinquish<PAIR>();
   }
   tc_fence_before();
   __syncthreads();
@@ -278,14 +373,23 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   auto fail = [&]() {
     *abort_flag = 1u;
+    if constexpr (PAIR) {   // the peer stops too
+      const uint32_t peer = map_to_rank(smem_u32((const void*)abort_flag), rank ^ 1u);
+      asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(peer), "r"(1u) : "memory");
+    }
     atomicOr(p.dev_status, kDevTimeout);
   };
 
   // Dynamic schedule (one query tile): the producer claims key tiles from a global counter and hands their
   // indices to the MMA issuer and the epilogue through a small ring; a CTA's claims increase, so ids still arrive
-  // in increasing order. Static schedule: units (query tile, split of the key tiles) in a fixed order.
-  const bool dyn = p.tile_ctr != nullptr;
+  // in increasing order. Static schedule: units (query tile, split of the key tiles) in a fixed order; for a
+  // pair, units (pair of query tiles, split) and this CTA takes the pair's tile of its rank.
+  const bool dyn = !PAIR && p.tile_ctr != nullptr;
   if (dyn && threadIdx.x == 0 && blockIdx.x == 0) *p.tile_ctr_next = 0;   // for the next launch (see TcParams)
+  const int unit0 = PAIR ? (int)cluster_id_x() : (int)blockIdx.x;
+  const int ustep = PAIR ? (int)cluster_count_x() : (int)gridDim.x;
+  const int per_split = PAIR ? p.pairs : p.q_tiles;
+  auto unit_qt = [&](int u) { return PAIR ? 2 * (u % p.pairs) + (int)rank : u % p.q_tiles; };
 
   if (warp == 0) {
     if (lane == 0) {
@@ -295,16 +399,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       const uint32_t withheld = (p.inject_stall && blockIdx.x == 0) ? 1u : 0xFFFFFFFFu;
       auto load_tile = [&](int qt, int64_t t) -> bool {
         for (int ks = 0; ks < p.k_steps; ++ks, ++it) {
-          const int s = it % STAGES;
-          const uint32_t ph = (it / STAGES) & 1u;
+          const int s = it % S;
+          const uint32_t ph = (it / S) & 1u;
           if (!mbar_wait(empty_bar(s), ph ^ 1u, abort_flag)) {
             fail();
             return false;
           }
           if (it == withheld) continue;   // nothing arrives on this stage: its consumer's wait runs out
-          mbar_expect_tx(full_bar(s), (uint32_t)(p.a_rows * BK * 2 + B_BYTES));
-          tma_load_2d(a_smem + s * A_BYTES, &tmap_q, full_bar(s), ks * BK, qt * BM);
-          tma_load_2d(b_smem + s * B_BYTES, &tmap_k, full_bar(s), ks * BK, (int)(t * BN));
+          if constexpr (PAIR) {
+            // both CTAs' boxes complete the leader's full barrier, which expects the bytes of all four. A box
+            // that would lie wholly out of bounds (the odd query tile's partner, the upper half of a last key
+            // tile of at most 128 keys) is replaced by the leader's box: the epilogue never reads those rows
+            // (queries >= B) or columns (ids >= n).
+            const uint32_t lead_full = map_to_rank(full_bar(s), 0);
+            if (rank == 0) mbar_expect_tx(full_bar(s), (uint32_t)(2 * G::kStageBytes));
+            const int qy = (qt < p.q_tiles ? qt : qt - 1) * BM;
+            const int64_t ky = t * BN + (int64_t)rank * G::kBRows;
+            tma_load_2d_pair(a_smem + s * A_BYTES, &tmap_q, lead_full, ks * BK, qy);
+            tma_load_2d_pair(b_smem + s * G::kBBytes, &tmap_k, lead_full, ks * BK, (int)(ky < p.n ? ky : t * BN));
+          } else {
+            mbar_expect_tx(full_bar(s), (uint32_t)(p.a_rows * BK * 2 + G::kBBytes));
+            tma_load_2d(a_smem + s * A_BYTES, &tmap_q, full_bar(s), ks * BK, qt * BM);
+            tma_load_2d(b_smem + s * G::kBBytes, &tmap_k, full_bar(s), ks * BK, (int)(t * BN));
+          }
         }
         return true;
       };
@@ -325,19 +442,28 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = load_tile(0, t);
         }
       } else {
-        for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-          const int qt = u % p.q_tiles, sp = u / p.q_tiles;
+        for (int u = unit0; ok && u < p.units; u += ustep) {
+          const int qt = unit_qt(u), sp = u / per_split;
           const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
           for (int64_t t = t_begin; ok && t < t_end; ++t) ok = load_tile(qt, t);
         }
       }
-      // drain: the last load issued into each stage has landed before the CTA may exit
-      const uint32_t first = it > (uint32_t)STAGES ? it - STAGES : 0u;
-      for (uint32_t i = first; i < it; ++i)
-        if (i != withheld && !mbar_wait(full_bar(i % STAGES), (i / STAGES) & 1u, nullptr)) fail();
+      // drain: the last load issued into each stage has landed before the CTA may exit. A pair's loads complete
+      // on the leader's barrier, so the peer waits instead for the MMA commits that free its stages (each
+      // follows the MMAs that read them, which waited for the data).
+      const uint32_t first = it > (uint32_t)S ? it - S : 0u;
+      for (uint32_t i = first; i < it; ++i) {
+        if (i == withheld) continue;
+        const bool landed = (PAIR && rank != 0) ? mbar_wait(empty_bar(i % S), (i / S) & 1u, nullptr)
+                                                : mbar_wait(full_bar(i % S), (i / S) & 1u, nullptr);
+        if (!landed) {
+          fail();
+          break;
+        }
+      }
     }
   } else if (warp == 1) {
-    if (lane == 0) {
+    if (lane == 0 && rank == 0) {
       // ---------------- MMA issuer ----------------
       uint32_t it = 0, tile_i = 0;
       bool ok = true;
@@ -350,20 +476,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         const uint32_t d_tmem = tmem + (uint32_t)(b * BN);
         for (int ks = 0; ks < p.k_steps; ++ks, ++it) {
-          const int s = it % STAGES;
-          if (!mbar_wait(full_bar(s), (it / STAGES) & 1u, abort_flag)) {
+          const int s = it % S;
+          if (!mbar_wait(full_bar(s), (it / S) & 1u, abort_flag)) {
             fail();
             return false;
           }
           tc_fence_after();
           const uint64_t ad = smem_desc(a_smem + s * A_BYTES);
-          const uint64_t bd = smem_desc(b_smem + s * B_BYTES);
+          const uint64_t bd = smem_desc(b_smem + s * G::kBBytes);
 #pragma unroll
           for (int kk = 0; kk < BK / 16; ++kk)
-            mma_bf16(d_tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), (ks | kk) != 0 ? 1u : 0u);
-          mma_commit(empty_bar(s));
+            mma_bf16<PAIR>(d_tmem, ad + (uint64_t)(kk * 2), bd + (uint64_t)(kk * 2), (ks | kk) != 0 ? 1u : 0u);
+          mma_commit<PAIR>(empty_bar(s), 3);
         }
-        mma_commit(tfull_bar(b));
+        mma_commit<PAIR>(tfull_bar(b), 3);
         ++tile_i;
         return true;
       };
@@ -380,15 +506,24 @@ __global__ void __launch_bounds__(kThreads, 1)
           ok = mma_tile();
         }
       } else {
-        for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-          const int sp = u / p.q_tiles;
+        for (int u = unit0; ok && u < p.units; u += ustep) {
+          const int sp = u / per_split;
           const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
           for (int64_t t = t_begin; ok && t < t_end; ++t) ok = mma_tile();
         }
       }
       // drain: every MMA issued by this thread has completed before TMEM is freed
-      mma_commit(drain_bar);
+      mma_commit<PAIR>(drain_bar, 1);
       if (!mbar_wait(drain_bar, 0, nullptr)) fail();
+      // a pair: the peer's epilogue releases of the last accumulators (remote arrivals on this CTA's barriers)
+      // have landed before the leader may exit
+      if (PAIR && ok) {
+        for (uint32_t i = tile_i > 2u ? tile_i - 2u : 0u; i < tile_i; ++i)
+          if (!mbar_wait(tempty_bar(i & 1u), (i >> 1) & 1u, abort_flag)) {
+            fail();
+            break;
+          }
+      }
     }
   } else {
     // ---------------- epilogue ----------------
@@ -459,7 +594,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(tempty_bar(b));
+      if (lane == 0) {
+        if constexpr (PAIR)
+          mbar_arrive_cluster(map_to_rank(tempty_bar(b), 0));
+        else
+          mbar_arrive(tempty_bar(b));
+      }
       ++tile_i;
       return true;
     };
@@ -490,8 +630,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (ok && active && !SIGN) write_partial(blockIdx.x, row);
     } else {
-      for (int u = blockIdx.x; ok && u < p.units; u += gridDim.x) {
-        const int qt = u % p.q_tiles, sp = u / p.q_tiles;
+      for (int u = unit0; ok && u < p.units; u += ustep) {
+        const int qt = unit_qt(u), sp = u / per_split;
         const int q = qt * BM + row;
         const bool active = q < p.B;
         const int64_t t_begin = p.n_tiles * sp / p.splits, t_end = p.n_tiles * (sp + 1) / p.splits;
@@ -506,9 +646,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
+  // a pair: neither CTA frees the pair's TMEM or exits while the other may still read its accumulators or
+  // receive the other's barrier arrivals
+  if constexpr (PAIR) cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, TMEM_COLS);
+    tmem_dealloc<PAIR>(tmem, TMEM_COLS);
   }
 }
 
@@ -521,24 +664,52 @@ int gcd_int(int a, int b) {
   return a;
 }
 
-template <int CPAD, bool SIGN = false>
-cudaError_t launch_cpad(const CUtensorMap* tq, const CUtensorMap* tk, const TcParams& p, int grid, cudaStream_t st) {
-  cudaError_t e = cudaFuncSetAttribute(stage1_tensor_kernel<CPAD, SIGN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)kSmemBytes);
-  if (e != cudaSuccess) return e;
+template <int CPAD, bool SIGN, bool PAIR>
+cudaLaunchConfig_t launch_config(cudaLaunchAttribute (&attr)[2], int grid, cudaStream_t st) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(grid);
   cfg.blockDim = dim3(kThreads);
-  cfg.dynamicSmemBytes = kSmemBytes;
+  cfg.dynamicSmemBytes = Geo<PAIR>::kSmem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[1].id = cudaLaunchAttributeClusterDimension;
+  attr[1].val.clusterDim.x = PAIR ? 2 : 1;
+  attr[1].val.clusterDim.y = 1;
+  attr[1].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, stage1_tensor_kernel<CPAD, SIGN>, *tq, *tk, p);
+  cfg.numAttrs = PAIR ? 2 : 1;
+  return cfg;
+}
+
+template <int CPAD, bool SIGN, bool PAIR>
+cudaError_t launch_cpad(const CUtensorMap* tq, const CUtensorMap* tk, const TcParams& p, int grid, cudaStream_t st) {
+  cudaError_t e = cudaFuncSetAttribute(stage1_tensor_kernel<CPAD, SIGN, PAIR>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)Geo<PAIR>::kSmem);
+  if (e != cudaSuccess) return e;
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = launch_config<CPAD, SIGN, PAIR>(attr, grid, st);
+  e = cudaLaunchKernelEx(&cfg, stage1_tensor_kernel<CPAD, SIGN, PAIR>, *tq, *tk, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
+}
+
+// CTA pairs of this kernel that can be resident at once on the current device (0: none, or not supported).
+template <int CPAD>
+int max_pair_clusters(cudaStream_t st) {
+  if (cudaFuncSetAttribute(stage1_tensor_kernel<CPAD, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)Geo<true>::kSmem) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  cudaLaunchAttribute attr[2];
+  cudaLaunchConfig_t cfg = launch_config<CPAD, false, true>(attr, 2, st);
+  int clusters = 0;
+  if (cudaOccupancyMaxActiveClusters(&clusters, stage1_tensor_kernel<CPAD, false, true>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return clusters;
 }
 
 bool encode_rows(EncodeTiledFn encode, CUtensorMap* m, const void* base, int64_t d, int64_t rows,
@@ -550,6 +721,68 @@ bool encode_rows(EncodeTiledFn encode, CUtensorMap* m, const void* base, int64_t
   return encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Key check of a batch of at least two query tiles on CTA pairs; false if no pair can be resident (the caller
+// then uses single CTAs).
+template <int CPAD>
+bool launch_pairs(TcParams p, const Stage1Args& a, EncodeTiledFn encode, int max_splits, cudaStream_t st,
+                  int* splits, cudaError_t* err) {
+  static int clusters = -1;   // per process: the device model does not change under a running process
+  if (clusters < 0) clusters = max_pair_clusters<CPAD>(st);
+  if (clusters < 1) return false;
+  p.pairs = (p.q_tiles + 1) / 2;
+  p.a_rows = BM;
+  CUtensorMap tq, tk;
+  if (!encode_rows(encode, &tq, a.q, a.d, a.B, (uint32_t)BM) ||
+      !encode_rows(encode, &tk, a.keys, a.d, a.n, (uint32_t)Geo<true>::kBRows)) {
+    *err = cudaErrorInvalidValue;
+    return true;
+  }
+  // whole waves of units over the resident pairs
+  int s = clusters / gcd_int(clusters, p.pairs);
+  if ((int64_t)s > p.n_tiles) s = (int)p.n_tiles;
+  if (s > max_splits) s = max_splits;
+  if (s < 1) s = 1;
+  p.splits = s;
+  p.units = p.pairs * s;
+  *splits = s;
+  const int grid = 2 * (p.units < clusters ? p.units : clusters);
+  *err = launch_cpad<CPAD, false, true>(&tq, &tk, p, grid, st);
+  return true;
+}
+
+template <int CPAD>
+cudaError_t launch_key_check(TcParams p, const Stage1Args& a, EncodeTiledFn encode, int num_sms, int max_splits,
+                             cudaStream_t st, int* splits, bool* paired) {
+  cudaError_t err = cudaSuccess;
+  if (p.q_tiles >= 2 && !p.inject_stall && launch_pairs<CPAD>(p, a, encode, max_splits, st, splits, &err)) {
+    if (paired) *paired = true;
+    return err;
+  }
+  // A batch of at most 128 queries is loaded as a box of B rows (rounded up to 8) rather than 128: boxes that
+  // are mostly out of bounds stream measurably slower. The MMA still computes 128 rows; rows past B hold stale
+  // shared memory and their TMEM lanes are never read.
+  p.a_rows = a.B >= BM ? BM : ((a.B + 7) / 8) * 8;
+  CUtensorMap tq, tk;
+  if (!encode_rows(encode, &tq, a.q, a.d, a.B, (uint32_t)p.a_rows) ||
+      !encode_rows(encode, &tk, a.keys, a.d, a.n, (uint32_t)BN))
+    return cudaErrorInvalidValue;
+  // splits such that q_tiles * splits is a multiple of the SM count (whole waves of units); one query tile with
+  // a tile counter: a dynamic schedule with one split per CTA
+  int s = num_sms / gcd_int(num_sms, p.q_tiles);
+  if ((int64_t)s > p.n_tiles) s = (int)p.n_tiles;
+  if (s > max_splits) s = max_splits;
+  if (s < 1) s = 1;
+  p.splits = s;
+  p.units = p.q_tiles * s;
+  if (p.q_tiles == 1 && a.tile_ctr) {
+    p.tile_ctr = a.tile_ctr;
+    p.tile_ctr_next = a.tile_ctr_next;
+  }
+  *splits = s;
+  const int grid = p.units < num_sms ? p.units : num_sms;
+  return launch_cpad<CPAD, false, false>(&tq, &tk, p, grid, st);
 }
 
 }  // namespace
@@ -581,11 +814,12 @@ cudaError_t launch_signatures(const __nv_bfloat16* rows, int64_t n, int d, const
       !encode_rows(encode, &tk, rows, d, n, (uint32_t)BN))
     return cudaErrorInvalidValue;
   const int grid = p.units < num_sms ? p.units : num_sms;
-  return launch_cpad<4, true>(&tq, &tk, p, grid, st);
+  return launch_cpad<4, true, false>(&tq, &tk, p, grid, st);
 }
 
 cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int num_sms, int max_splits,
-                                 cudaStream_t st, int* splits) {
+                                 cudaStream_t st, int* splits, bool* paired) {
+  if (paired) *paired = false;
   TcParams p{};
   p.n = a.n;
   p.d = a.d;
@@ -595,36 +829,14 @@ cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int 
   p.q_tiles = (a.B + BM - 1) / BM;
   p.n_tiles = (a.n + BN - 1) / BN;
   p.k_steps = (a.d + BK - 1) / BK;
-  // A batch of at most 128 queries is loaded as a box of B rows (rounded up to 8) rather than 128: boxes that
-  // are mostly out of bounds stream measurably slower. The MMA still computes 128 rows; rows past B hold stale
-  // shared memory and their TMEM lanes are never read.
-  p.a_rows = a.B >= BM ? BM : ((a.B + 7) / 8) * 8;
-  CUtensorMap tq, tk;
-  if (!encode_rows(encode, &tq, a.q, a.d, a.B, (uint32_t)p.a_rows) ||
-      !encode_rows(encode, &tk, a.keys, a.d, a.n, (uint32_t)BN))
-    return cudaErrorInvalidValue;
-  // splits such that q_tiles * splits is a multiple of the SM count (whole waves of units); one query tile with
-  // a tile counter: a dynamic schedule with one split per CTA
-  int s = num_sms / gcd_int(num_sms, p.q_tiles);
-  if ((int64_t)s > p.n_tiles) s = (int)p.n_tiles;
-  if (s > max_splits) s = max_splits;
-  if (s < 1) s = 1;
-  p.splits = s;
-  p.units = p.q_tiles * s;
-  if (p.q_tiles == 1 && a.tile_ctr) {
-    p.tile_ctr = a.tile_ctr;
-    p.tile_ctr_next = a.tile_ctr_next;
-  }
   p.part_cand = a.part_cand;
   p.part_best = a.part_best;
   p.dev_status = a.dev_status;
   p.inject_stall = a.inject_stall;
-  *splits = s;
-  const int grid = p.units < num_sms ? p.units : num_sms;
-  if (a.top_c <= 4) return launch_cpad<4>(&tq, &tk, p, grid, st);
-  if (a.top_c <= 8) return launch_cpad<8>(&tq, &tk, p, grid, st);
-  if (a.top_c <= 16) return launch_cpad<16>(&tq, &tk, p, grid, st);
-  return launch_cpad<32>(&tq, &tk, p, grid, st);
+  if (a.top_c <= 4) return launch_key_check<4>(p, a, encode, num_sms, max_splits, st, splits, paired);
+  if (a.top_c <= 8) return launch_key_check<8>(p, a, encode, num_sms, max_splits, st, splits, paired);
+  if (a.top_c <= 16) return launch_key_check<16>(p, a, encode, num_sms, max_splits, st, splits, paired);
+  return launch_key_check<32>(p, a, encode, num_sms, max_splits, st, splits, paired);
 }
 
 }  // namespace lc

@@ -39,6 +39,8 @@ def _check_streamed(w, per_class):
         out = cache.lookup(q["emb"], q["prefix"], q["ids"])
         torch.cuda.synchronize()
         cache.sync()
+        # batches of more than one query tile run on CTA pairs
+        assert cache.last_launch()[1] == (L.LACACHE_STAGE1_TENSOR_PAIR if w.batch > 128 else L.LACACHE_STAGE1_TENSOR)
         g = {k: v.cpu().numpy() for k, v in out.items()}
     res = so.result()
     rep = compare(g, res, p, rows=sample, pair_scores=so.pair_scores)
