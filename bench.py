@@ -345,7 +345,7 @@ def run_ours(args, w):
     peaks, peak_src = load_peaks()
     s1_bytes, s2_bytes, flops = algorithmic(w, w.batch)
     t1_avg_s = t1_ms / max(1, timed) / 1e3
-    traffic = kernel_traffic(kernel_name, w.name)
+    traffic = None if args.entries else kernel_traffic(kernel_name, w.name)
     value = job["value"]
     # the stage-1 kernel is bound by HBM below the ridge (flops per byte of the measured peaks), else by the
     # tensor pipe; a kernel timed back to back for over a second is compared with the sustained bf16 peak
