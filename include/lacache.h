@@ -18,7 +18,7 @@
  *  - Pointers named *_dev are CUDA device pointers (cudaMalloc or equivalent) on the handle's device. Pointers
  *    named *_host are host pointers (page-locked memory is fastest). The caller owns every input and output
  *    buffer; the handle owns the device store and its scratch.
- *  - Embedding pointers must be 16-byte aligned (TMA reads them).
+ *  - Device embedding pointers must be 16-byte aligned (TMA reads them). Host pointers may have any alignment.
  *  - `cuda_stream` is a cudaStream_t (NULL = the legacy default stream). Device calls are asynchronous on it;
  *    argument errors are reported synchronously and leave the cache unchanged.
  *  - Device-side faults of the library's own kernels (a bounded wait that ran out) do not abort the process:
@@ -144,9 +144,12 @@ lacache_status lacache_insert(lacache_t* h, int64_t n, const void* key_dev, cons
 lacache_status lacache_lookup(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
                               const int32_t* q_ids_dev, const lacache_result* out, void* cuda_stream);
 
-/* lacache_lookup for host-resident queries and results: copies the inputs into the handle's device staging,
- * runs the same kernels, copies the results back into *out_host (host pointers) and synchronizes cuda_stream
- * before returning. */
+/* lacache_lookup for host-resident queries and results (any host memory: pageable or pinned, any alignment).
+ * The inputs reach the handle's device staging in one of two ways. An array in pinned memory that the device can
+ * map is read by the device directly, one gather kernel covering all such arrays. Any other array is copied by
+ * DMA. The same kernels then run. Their results go straight into the handle's mapped pinned staging, or through
+ * one device-to-host copy where the device cannot map it. The call synchronizes cuda_stream, copies the results
+ * into *out_host (host pointers) and returns. */
 lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_host, const void* q_prefix_host,
                                    const int32_t* q_ids_host, const lacache_result* out_host, void* cuda_stream);
 

@@ -7,6 +7,8 @@
 
 #include <new>
 
+#include <algorithm>
+
 #include "internal.cuh"
 
 struct lacache {
@@ -27,7 +29,8 @@ struct lacache {
   int32_t* append_count_host;  // pinned
   unsigned char* stage_in;   // device staging for lookup_host inputs
   unsigned char* stage_out;  // device staging for lookup_host results
-  unsigned char* stage_host; // pinned host copy of stage_out
+  unsigned char* stage_host; // pinned host staging of lookup_host results (mapped: the kernels write it directly)
+  unsigned char* stage_host_dev; // device address of stage_host, or nullptr if the device cannot map it
   int last_splits;
   int last_kernel;
   lc::EncodeTiledFn encode;
@@ -126,6 +129,44 @@ __global__ void append_rows_kernel(const uint4* __restrict__ q_emb, const uint4*
   for (int i = threadIdx.x; i < kv; i += blockDim.x) key[row * kv + i] = q_emb[(int64_t)q * kv + i];
   for (int i = threadIdx.x; i < pv; i += blockDim.x) pre[row * pv + i] = q_pre[(int64_t)q * pv + i];
   for (int i = threadIdx.x; i < k; i += blockDim.x) ids[row * k + i] = q_ids[(int64_t)q * k + i];
+}
+
+// lookup_host's inputs, read by the device straight from mapped pinned host memory (NVLink-C2C on Grace) into the
+// device staging: one launch for the three arrays instead of one DMA copy each. Segments with zero bytes are
+// skipped; 16-byte vectors where both ends are aligned, bytes otherwise. Lets the stage-1 grid (a programmatic
+// dependent) start its set-up at once; that grid reads nothing before this one has completed.
+struct GatherSeg {
+  const unsigned char* src;
+  unsigned char* dst;
+  size_t bytes;
+};
+struct GatherArgs {
+  GatherSeg seg[3];
+};
+__global__ void gather_host_kernel(GatherArgs g) {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const size_t tid = blockIdx.x * (size_t)blockDim.x + threadIdx.x, nth = (size_t)gridDim.x * blockDim.x;
+  for (int s = 0; s < 3; ++s) {
+    const GatherSeg e = g.seg[s];
+    const bool vec = (((uintptr_t)e.src | (uintptr_t)e.dst) & 15u) == 0;
+    const size_t nv = vec ? e.bytes / 16 : 0;
+    const uint4* sv = reinterpret_cast<const uint4*>(e.src);
+    uint4* dv = reinterpret_cast<uint4*>(e.dst);
+    for (size_t i = tid; i < nv; i += nth) dv[i] = sv[i];
+    for (size_t i = nv * 16 + tid; i < e.bytes; i += nth) e.dst[i] = e.src[i];
+  }
+}
+
+// The address through which the current device can read host pointer p, or nullptr when it has none (pageable
+// memory, or pinned memory not mapped for this device). Asked of the driver on every call, never cached: a
+// device access through a stale answer would fault.
+const void* mapped_device_pointer(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
 }
 
 size_t stage_in_bytes(const lacache_config& c, int pd) {
@@ -369,7 +410,7 @@ lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_
             cudaMalloc(&h->stage_in, stage_in_bytes(c, pd)) == cudaSuccess &&
             cudaMalloc(&h->stage_out, stage_out_bytes(c, ens->m)) == cudaSuccess &&
             cudaMallocHost(&h->append_count_host, 4) == cudaSuccess &&
-            cudaMallocHost(&h->stage_host, stage_out_bytes(c, ens->m)) == cudaSuccess &&
+            cudaHostAlloc((void**)&h->stage_host, stage_out_bytes(c, ens->m), cudaHostAllocMapped) == cudaSuccess &&
             cudaMemset(h->dev_status, 0, 4) == cudaSuccess &&
             cudaMemset(h->part_cand, 0, (size_t)h->max_splits * c.max_batch * c.top_c * 8) == cudaSuccess &&
             cudaDeviceSynchronize() == cudaSuccess;
@@ -378,6 +419,10 @@ lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_
     free_all(h);
     delete h;
     return LACACHE_ERR_OOM;
+  }
+  if (cudaHostGetDevicePointer((void**)&h->stage_host_dev, h->stage_host, 0) != cudaSuccess) {
+    cudaGetLastError();
+    h->stage_host_dev = nullptr;   // results then come back with one device-to-host copy
   }
   void* fn = nullptr;
   cudaDriverEntryPointQueryResult q;
@@ -454,21 +499,41 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
   unsigned char* q_emb = h->stage_in;
   unsigned char* q_pre = q_emb + (size_t)c.max_batch * c.d * 2;
   int32_t* q_ids = reinterpret_cast<int32_t*>(q_pre + (size_t)c.max_batch * h->pd * 2);
-  cudaError_t e = cudaMemcpyAsync(q_emb, q_emb_host, (size_t)B * c.d * 2, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(q_pre, q_prefix_host, (size_t)B * h->pd * 2, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(q_ids, q_ids_host, (size_t)B * c.k * 4, cudaMemcpyHostToDevice, st);
-  if (e != cudaSuccess) return LACACHE_ERR_CUDA;
+  // Inputs: arrays in mapped pinned memory are gathered by one kernel; any other array is copied by DMA.
+  const void* src[3] = {q_emb_host, q_prefix_host, q_ids_host};
+  unsigned char* dst[3] = {q_emb, q_pre, reinterpret_cast<unsigned char*>(q_ids)};
+  const size_t nbytes[3] = {(size_t)B * c.d * 2, (size_t)B * h->pd * 2, (size_t)B * c.k * 4};
+  GatherArgs g{};
+  size_t gathered = 0;
+  for (int i = 0; i < 3; ++i) {
+    const void* dev_src = mapped_device_pointer(src[i]);
+    if (dev_src) {
+      g.seg[i] = GatherSeg{static_cast<const unsigned char*>(dev_src), dst[i], nbytes[i]};
+      gathered += nbytes[i];
+    } else if (cudaMemcpyAsync(dst[i], src[i], nbytes[i], cudaMemcpyHostToDevice, st) != cudaSuccess) {
+      return LACACHE_ERR_CUDA;
+    }
+  }
+  if (gathered) {
+    const size_t vec = (gathered + 15) / 16;
+    const int grid = (int)std::min<size_t>((vec + 255) / 256, (size_t)2 * h->num_sms);
+    gather_host_kernel<<<grid, 256, 0, st>>>(g);
+    if (cudaGetLastError() != cudaSuccess) return LACACHE_ERR_CUDA;
+  }
   const bool cand = out_host->cand_id || out_host->cand_score || out_host->cand_prefix_score ||
                     out_host->cand_matches;
   const bool scores = out_host->prefix_scores != nullptr;
   size_t bytes = 0;
-  lacache_result dev = staged_result(h->stage_out, B, c.top_c, h->ens.m, cand, scores, &bytes);
+  // Results: written by the kernels straight into the mapped pinned staging when the device can map it.
+  unsigned char* out_stage = h->stage_host_dev ? h->stage_host_dev : h->stage_out;
+  lacache_result dev = staged_result(out_stage, B, c.top_c, h->ens.m, cand, scores, &bytes);
   lacache_result host = staged_result(h->stage_host, B, c.top_c, h->ens.m, cand, scores, &bytes);
   lacache_status s = run_lookup(h, B, q_emb, q_pre, q_ids, dev, st);
   if (s != LACACHE_OK) return s;
-  if (cudaMemcpyAsync(h->stage_host, h->stage_out, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess ||
-      cudaStreamSynchronize(st) != cudaSuccess)
+  if (!h->stage_host_dev &&
+      cudaMemcpyAsync(h->stage_host, h->stage_out, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess)
     return LACACHE_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return LACACHE_ERR_CUDA;
   const size_t b4 = (size_t)B * 4, bc4 = (size_t)B * c.top_c * 4;
   struct Copy {
     void* dst;

@@ -192,6 +192,39 @@ def test_host_buffer_lookup_matches_device_lookup(stage1):
             assert np.array_equal(v.numpy(), g[k], equal_nan=True), k
 
 
+def _host_copy(t, kind, offset=0):
+    """A host copy of tensor t: pinned, pageable, or pinned at `offset` bytes past a 16-byte boundary."""
+    if kind == "pageable":
+        return t.cpu().clone()
+    raw = torch.empty(t.numel() * t.element_size() + offset, dtype=torch.uint8).pin_memory()
+    v = raw[offset:].view(t.dtype).view(t.shape)
+    v.copy_(t.cpu())
+    return v
+
+
+@pytest.mark.parametrize("kinds", [("pageable", "pageable", "pageable"), ("pinned+2", "pinned+6", "pinned+4"),
+                                   ("pinned", "pageable", "pinned+4")], ids=["pageable", "misaligned", "mixed"])
+def test_host_buffer_lookup_any_host_memory(kinds):
+    # inputs in mapped pinned memory are gathered by a kernel, others copied by DMA; results written to the
+    # library's mapped staging are copied into any host arrays. B = 300 also covers the CTA-pair kernel.
+    w = wl.WORKLOADS["serve-2m"].scaled(n=12_050, batch=300, clusters=120)
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+        fill(cache, w)
+        q = wl.batch(w, 0, device="cuda")
+        g = gpu_lookup(cache, q)
+        hq = {}
+        for key, kind in zip(("emb", "prefix", "ids"), kinds):
+            off = int(kind.split("+")[1]) if "+" in kind else 0
+            hq[key] = _host_copy(q[key], "pageable" if kind == "pageable" else "pinned", off)
+            assert (hq[key].data_ptr() % 16 == 0) == (off == 0)
+        out = L.alloc_result(w.batch, w.top_c, "cpu", pinned=kinds[0] != "pageable")
+        for _ in range(2):   # twice: the second call reuses the staging
+            L.lacache_lookup_host(cache.h, hq["emb"], hq["prefix"], hq["ids"], out)
+            for k, v in out.items():
+                assert np.array_equal(v.numpy(), g[k], equal_nan=True), k
+        assert cache.last_launch()[1] == L.LACACHE_STAGE1_TENSOR_PAIR
+
+
 @pytest.mark.parametrize("stage1", PATHS)
 def test_serve_loop_appends_misses_like_the_oracle(stage1):
     w = wl.WORKLOADS["serve-2m"].scaled(n=20_000, batch=64, clusters=200)
