@@ -3,7 +3,7 @@
 // One CTA (8 warps) per query:
 //  1. merge the stage-1 partial lists (splits x top_c packed candidates) into C_q, the top_c candidates by
 //     (key score desc, entry id asc): every thread keeps a sorted top-c of the entries it reads (loads issued
-//     four at a time), each warp reduces its lanes' lists by top_c rounds of a warp-wide max, and warp 0 merges
+//     eight at a time), each warp reduces its lanes' lists by top_c rounds of a warp-wide max, and warp 0 merges
 //     the eight warp lists the same way;
 //  2. the candidates are checked in parallel, one warp per candidate: r = <p_q, P_j> (the prefix-embedding cosine
 //     sim(f_k(x), f_k(x'))) in fp32, each lane's 8-element chunks in order, then a butterfly sum (every lane ends
@@ -25,13 +25,14 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// Warp-wide maximum of a packed candidate, as two 32-bit warp reductions: the largest high word (score order),
+// then the largest low word (~id) among the lanes that hold it. Unsigned 64-bit order is (high, low)
+// lexicographic, so this is the 64-bit maximum.
 __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const uint64_t other = __shfl_xor_sync(kFull, v, o);
-    v = other > v ? other : v;
-  }
-  return v;
+  const uint32_t hi = (uint32_t)(v >> 32), lo = (uint32_t)v;
+  const uint32_t mhi = __reduce_max_sync(kFull, hi);
+  const uint32_t mlo = __reduce_max_sync(kFull, hi == mhi ? lo : 0u);
+  return ((uint64_t)mhi << 32) | mlo;
 }
 
 __device__ __forceinline__ float dot8(const uint4& u, const uint4& v, float acc) {
@@ -93,10 +94,11 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
 #pragma unroll
   for (int i = 0; i < CPAD; ++i) loc[i] = 0;
   const int total = a.splits * C;
-  for (int e0 = threadIdx.x; e0 < total; e0 += 4 * kThreads) {
-    uint64_t x[4];
+  constexpr int U = CPAD <= 16 ? 8 : 4;   // loads in flight per thread (one pass for 152 splits x 8)
+  for (int e0 = threadIdx.x; e0 < total; e0 += U * kThreads) {
+    uint64_t x[U];
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < U; ++u) {
       const int e = e0 + u * kThreads;
       x[u] = 0;
       if (e < total) {
@@ -105,20 +107,24 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
       }
     }
 #pragma unroll
-    for (int u = 0; u < 4; ++u) {
+    for (int u = 0; u < U; ++u) {
       if (x[u] != 0 && (int64_t)cand_id(x[u]) >= a.n) x[u] = 0;   // never gather outside the store
       keep(loc, x[u]);
     }
   }
-  // 1c. per-warp top-c
+  // 1c. per-warp top-c (rounds stop at the first empty maximum: every later one is empty too)
   for (int r = 0; r < C; ++r) {
     const uint64_t m = warp_max_u64(loc[0]);
-    if (loc[0] == m && m != 0) {
+    if (lane == 0) warp_top[warp][r] = m;
+    if (m == 0) {
+      for (int i = r + 1 + lane; i < C; i += 32) warp_top[warp][i] = 0;
+      break;
+    }
+    if (loc[0] == m) {
 #pragma unroll
       for (int i = 0; i < CPAD - 1; ++i) loc[i] = loc[i + 1];
       loc[CPAD - 1] = 0;
     }
-    if (lane == 0) warp_top[warp][r] = m;
   }
   __syncthreads();
   // 1d. warp 0 merges the eight warp lists: lane l < kWarps walks list l
