@@ -47,6 +47,10 @@ def parse_args():
     ap.add_argument("--batches", type=int, default=8, help="distinct query batches cycled through")
     ap.add_argument("--e2e-steps", type=int, default=500)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--mode", choices=["replicas", "shard"], default="replicas",
+                    help="replicas: every rank serves its own batches against a full copy of the store (weak "
+                         "scaling); shard: the store is split by entry range across the ranks, every rank serves "
+                         "the same batches, one all-gather and a merge per lookup (strong scaling)")
     ap.add_argument("--entries", type=int, default=0,
                     help="store size override: a smaller case of the workload (profiling captures)")
     return ap.parse_args()
@@ -380,17 +384,166 @@ def run_ours(args, w):
         "clocks": clock,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        # a bounded sample: as many store rows as take about 15 s of oracle time (all of them if fewer)
-        probe = min(w.n, 8192)
-        store, oq = oracle_sample(w, probe, 0, "cuda")
-        per_row = time_oracle(store, oq, w) / probe
-        rows = int(min(w.n, max(probe, 15.0 / per_row)))
-        store, oq = oracle_sample(w, rows, 0, "cuda")
-        t = time_oracle(store, oq, w)
-        line["cpu_baseline"] = {
-            "value": w.batch / (t * w.n / rows), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
+        line["cpu_baseline"] = cpu_baseline(w)
+    cache.close()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def cpu_baseline(w) -> dict:
+    """The oracle on the host cores over a bounded sample: as many store rows as take about 15 s of oracle time
+    (all of them if fewer), scaled to the full store."""
+    probe = min(w.n, 8192)
+    store, oq = oracle_sample(w, probe, 0, "cuda")
+    per_row = time_oracle(store, oq, w) / probe
+    rows = int(min(w.n, max(probe, 15.0 / per_row)))
+    store, oq = oracle_sample(w, rows, 0, "cuda")
+    t = time_oracle(store, oq, w)
+    return {"value": w.batch / (t * w.n / rows), "unit": UNIT, "cores": cpu_threads(), "kind": "oracle",
             "sample": f"oracle lookup of the {w.batch}-query batch against the first {rows} of the {w.n} store rows "
                       f"({t:.1f} s), scaled to the full store by N/rows (the oracle is linear in N)"}
+
+
+def run_sharded(args, w):
+    """Entry-range sharding: rank r holds store rows [N r / world, N (r + 1) / world); every rank looks up the same
+    batches; per lookup, the rank's own lookup, one all-gather of the candidate records and the merge
+    (paper_2608_01718_gb300.sharded). Strong scaling: the job serves B queries per step whatever the world size."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_01718_gb300 import build, sharded
+    from paper_2608_01718_gb300 import lacache as L
+    from paper_2608_01718_gb300 import workloads as wl
+
+    rank, local_rank, world = rank_info()
+    torch.cuda.set_device(local_rank)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+    build.build()
+    a, b = w.n * rank // world, w.n * (rank + 1) // world
+    models = len(w.prefix_dims) if w.prefix_dims is not None else 1
+    cache = L.LaCache(w.d, w.k, max(1, b - a), w.tau_c, w.tau_a, w.top_c, max_batch=w.batch, device=local_rank,
+                      prefix_dims=w.prefix_dims, tau_a_models=w.tau_a_models)
+    dtype = L.LACACHE_F32 if w.key_dtype == "f32" else L.LACACHE_BF16
+    off = 0
+    for ch in wl.iter_store(w, "cuda"):
+        n = ch["key"].shape[0]
+        lo, hi = max(a, off), min(b, off + n)
+        if lo < hi:
+            cache.insert(ch["key"][lo - off:hi - off], ch["prefix"][lo - off:hi - off], ch["ids"][lo - off:hi - off],
+                         dtype)
+        off += n
+        del ch
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    stream = torch.cuda.current_stream()
+    scratch = L.alloc_result(w.batch, w.top_c, "cuda", candidates=False)
+
+    def local_lookup(q, rec):
+        L.lacache_lookup(cache.h, q["emb"], q["prefix"], q["ids"], {**scratch, **rec}, stream)
+
+    def merge(shards, out):
+        L.lacache_merge_shards(shards, w.top_c, models, out, stream)
+
+    lk = sharded.ShardedLookup(w.batch, w.top_c, models, a, "cuda", local_lookup, merge)
+    nb = args.batches
+    batches = [wl.batch(w, step=i, device="cuda") for i in range(nb)]
+    outs = [L.alloc_result(w.batch, w.top_c, "cuda", candidates=False, models=models if models > 1 else 0)
+            for _ in range(nb)]
+
+    def step(i):
+        lk(batches[i % nb], outs[i % nb])
+
+    for i in range(max(3, args.warmup)):
+        step(i)
+    torch.cuda.synchronize()
+    cache.sync()
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    clocks = ClockSampler(torch.cuda.current_device())
+    clocks.start()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for i in range(args.steps):
+        step(i)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clock = clocks.stop()
+    cache.sync()
+    elapsed_ms = ev0.elapsed_time(ev1)
+    L.lacache_stage_timing(cache.h, args.steps)
+    for i in range(args.steps):
+        step(i)
+    t1_ms, t2_ms, timed = L.lacache_stage_times(cache.h)
+    L.lacache_stage_timing(cache.h, 0)
+
+    # end to end: pinned host batch -> device, the sharded lookup, the decisions back to pinned host memory
+    hq = [{k: batches[i][k].cpu().pin_memory() for k in ("emb", "prefix", "ids")} for i in range(nb)]
+    dq = [{k: torch.empty_like(batches[i][k]) for k in ("emb", "prefix", "ids")} for i in range(nb)]
+    keys = ("entry_id", "status", "key_score", "prefix_score", "token_matches", "n_cand")
+    hout = [{k: torch.empty_like(outs[i][k], device="cpu").pin_memory() for k in keys} for i in range(nb)]
+
+    def e2e_step(i):
+        j = i % nb
+        for k in dq[j]:
+            dq[j][k].copy_(hq[j][k], non_blocking=True)
+        lk(dq[j], outs[j])
+        for k in keys:
+            hout[j][k].copy_(outs[j][k], non_blocking=True)
+        stream.synchronize()
+
+    for i in range(max(3, args.warmup)):
+        e2e_step(i)
+    if world > 1:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for i in range(args.e2e_steps):
+        e2e_step(i)
+    e2e_s = time.perf_counter() - t0
+    times = torch.tensor([elapsed_ms, e2e_s], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(times, op=dist.ReduceOp.MAX)
+    elapsed_ms, e2e_s = float(times[0]), float(times[1])
+
+    peaks, peak_src = load_peaks()
+    local = w.scaled(n=max(1, b - a))
+    s1_bytes, _, flops = algorithmic(local, w.batch)
+    t1_avg_s = t1_ms / max(1, timed) / 1e3
+    ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    if flops / s1_bytes < ridge:
+        roof = {"bound": "hbm", "achieved": s1_bytes / t1_avg_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "peak_source": f"{peak_src} (copy bandwidth)"}
+    else:
+        roof = {"bound": "tensor", "achieved": flops / t1_avg_s / 1e12, "peak": peaks["bf16_tflops"],
+                "unit": "TFLOP/s", "peak_source": f"{peak_src} (burst bf16 dense)"}
+    roof["frac"] = roof["achieved"] / roof["peak"]
+    kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_TENSOR_PAIR: "tensor-pair",
+                   L.LACACHE_STAGE1_SIMT: "simt", L.LACACHE_STAGE1_LSH: "lsh"}[cache.last_launch()[1]]
+    line = {
+        "metric": METRIC, "value": w.batch * args.steps / (elapsed_ms / 1e3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps,
+        "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": workload_config(w) | {"parallelism": f"entry-shards{world}", "shard_entries": b - a},
+        "stage1_kernel": kernel_name,
+        "roofline": roof | {"traffic": None, "kernel": f"stage1_{kernel_name} (one shard)",
+                            "algorithmic_bytes_per_launch": s1_bytes, "algorithmic_flops_per_launch": flops,
+                            "avg_launch_ms": t1_avg_s * 1e3},
+        "stage_ms": {"stage1": t1_ms / max(1, timed), "stage2": t2_ms / max(1, timed), "timed_lookups": timed},
+        "e2e": {"value": w.batch * args.e2e_steps / e2e_s, "unit": UNIT,
+                "h2d_bytes_per_step": w.batch * (2 * w.d + 2 * w.pd + w.k * 4),
+                "d2h_bytes_per_step": w.batch * (4 + 1 + 4 + 4 + 4 + 4), "steps": args.e2e_steps,
+                "api": "paper_2608_01718_gb300.sharded.ShardedLookup (pinned host buffers, synchronous per step)"},
+        "gpu_launches": 3 * args.steps,
+        "clocks": clock,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w)
     cache.close()
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -450,6 +603,8 @@ def main():
         w = w.scaled(n=args.entries)
     if args.impl == "reference":
         return run_reference(args, w)
+    if args.mode == "shard":
+        return run_sharded(args, w)
     return run_ours(args, w)
 
 

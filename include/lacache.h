@@ -113,6 +113,9 @@ typedef struct {
   int32_t* cand_matches;      /* optional [B x top_c]: their token matches, -1 padded */
   float* prefix_scores;       /* optional [B x m]: every model's lookahead score for the candidate of prefix_score
                                  (prefix_score is model 0's); NaN on MISS_KEY */
+  uint8_t* cand_pass;         /* optional [B x top_c]: 1 if the candidate passes the lookahead check under the
+                                 handle's check mode (every model of an ensemble), 0 otherwise and as padding */
+  float* cand_prefix_scores;  /* optional [B x top_c x m]: every model's lookahead score per candidate, NaN padded */
 } lacache_result;
 
 /* Create a cache on cfg->device with an empty store of cfg->capacity entries. Allocates the store
@@ -255,6 +258,41 @@ lacache_status lacache_verify_draft(int32_t B, int32_t k, const float* p_target_
 
 /* Static description of a status code. */
 const char* lacache_status_string(lacache_status s);
+
+/* Entry-range sharding (one store split across GPUs by row ranges; a multi-GPU form of the lookup). Each GPU
+ * holds global entries [id_base, id_base + n) in its own handle and runs lacache_lookup on the same batch with the
+ * candidate outputs (cand_id, cand_score, cand_prefix_score, cand_matches, cand_pass, and cand_prefix_scores for
+ * an ensemble). The shards' outputs are then exchanged, for instance by one all-gather, and merged here into the
+ * result of one lookup over the whole store.
+ *
+ * The merge is exact. The key check is per entry, so A_q is the union of the shards' sets. Every member of the
+ * global candidate list C_q is among its own shard's first top_c, so C_q is the first top_c of the shards' lists
+ * by (key score desc, global id asc). A candidate's lookahead result depends only on its own row. The served
+ * entry is the first passing member of C_q. key_score on a miss is the maximum over the shards. All shards must
+ * use the same top_c, thresholds and check mode.
+ *
+ * A shard's outputs as the merge reads them: device pointers on the current device, laid out as lacache_lookup
+ * writes them. */
+typedef struct {
+  const int32_t* cand_id;            /* [B x top_c] local ids, -1 padded */
+  const float* cand_score;           /* [B x top_c] */
+  const float* cand_prefix_score;    /* [B x top_c] */
+  const int32_t* cand_matches;       /* [B x top_c] */
+  const uint8_t* cand_pass;          /* [B x top_c] */
+  const float* cand_prefix_scores;   /* [B x top_c x m]; may be NULL when m == 1 (cand_prefix_score is used) */
+  const float* key_score;            /* [B] */
+  const int32_t* n_cand;             /* [B] */
+  int64_t id_base;                   /* global id of the shard's entry 0; bases increase with the shard index */
+} lacache_shard_result;
+
+#define LACACHE_MAX_SHARDS 16
+
+/* Merge the outputs of G shards (1..LACACHE_MAX_SHARDS; shards is a host array) for a batch of B queries into
+ * *out (device pointers; the same fields and optional fields as a lookup; entry and candidate ids are global and
+ * must fit in int32). m is the number of lookahead models (1 without an ensemble). Runs on the current device,
+ * asynchronously on cuda_stream. */
+lacache_status lacache_merge_shards(int32_t G, const lacache_shard_result* shards, int32_t B, int32_t top_c,
+                                    int32_t m, const lacache_result* out, void* cuda_stream);
 
 #ifdef __cplusplus
 }

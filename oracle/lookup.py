@@ -98,6 +98,8 @@ class Result:
     cand_prefix_score: np.ndarray  # f64 [B, c]; r, NaN padded
     cand_matches: np.ndarray      # int32 [B, c]; m, -1 padded
     prefix_scores: np.ndarray     # f64 [B, models]; every model's r for the candidate of prefix_score
+    cand_pass: np.ndarray         # bool [B, c]; each candidate passes the lookahead check (False padded)
+    cand_prefix_scores: np.ndarray  # f64 [B, c, models]; every model's r per candidate, NaN padded
     margin: np.ndarray            # f64 [B]; decision margin: smallest score change altering status/entry_id
     list_margin: np.ndarray       # f64 [B]; smallest score change altering C_q or its order
     literal_margin: np.ndarray    # f64 [B]; min(|max_j s - tau_c|, s_(1) - s_(2))
@@ -211,6 +213,7 @@ def decide(kc: KeyCheck, q_prefix_bits, q_ids, params: Params,
         cand_id=np.full((B, c), -1, np.int32), cand_score=np.full((B, c), np.nan),
         cand_prefix_score=np.full((B, c), np.nan), cand_matches=np.full((B, c), -1, np.int32),
         prefix_scores=np.full((B, n_models), np.nan),
+        cand_pass=np.zeros((B, c), bool), cand_prefix_scores=np.full((B, c, n_models), np.nan),
         margin=np.full(B, np.inf), list_margin=np.full(B, np.inf), literal_margin=np.full(B, np.inf),
         next_id=np.full(B, -1, np.int32), next_score=np.full(B, np.nan))
 
@@ -231,6 +234,8 @@ def decide(kc: KeyCheck, q_prefix_bits, q_ids, params: Params,
             r = rm[:, 0]                              # model 0: the reported prefix score
             res.cand_prefix_score[b, :nc] = r
             res.cand_matches[b, :nc] = m
+            res.cand_pass[b, :nc] = ok
+            res.cand_prefix_scores[b, :nc] = rm
             hits = np.nonzero(ok)[0]
             shown = int(hits[0]) if hits.size else 0
             if hits.size:

@@ -173,14 +173,15 @@ size_t stage_in_bytes(const lacache_config& c, int pd) {
   return (size_t)c.max_batch * ((size_t)2 * c.d + (size_t)2 * pd + (size_t)4 * c.k);
 }
 size_t stage_out_bytes(const lacache_config& c, int m) {
-  // five [B] 4-byte arrays, four [B x top_c] 4-byte arrays, one [B x m] 4-byte array, one [B] byte array, each
-  // rounded up to 16 bytes
-  return (size_t)c.max_batch * (21 + (size_t)c.top_c * 16 + (size_t)m * 4) + 11 * 16;
+  // five [B] 4-byte arrays, one [B] byte array, four [B x top_c] 4-byte arrays, one [B x top_c] byte array, one
+  // [B x m] and one [B x top_c x m] 4-byte array, each rounded up to 16 bytes
+  const size_t cm = (size_t)c.top_c * m;
+  return (size_t)c.max_batch * (21 + (size_t)c.top_c * 17 + (size_t)m * 4 + cm * 4) + 13 * 16;
 }
 
-// Layout of the results of lookup_host in the device staging buffer (and in its pinned host copy): the arrays of
-// a B-query batch packed back to back, each 16-byte aligned, so that one copy brings them all back.
-lacache_result staged_result(unsigned char* base, int B, int top_c, int m, bool cand, bool scores,
+// Layout of the results of lookup_host in the staging buffer: the arrays of a B-query batch packed back to back,
+// each 16-byte aligned; an optional array is present iff `want` asks for it.
+lacache_result staged_result(unsigned char* base, int B, int top_c, int m, const lacache_result& want,
                              size_t* bytes) {
   unsigned char* p = base;
   auto take = [&](size_t n) {
@@ -196,11 +197,13 @@ lacache_result staged_result(unsigned char* base, int B, int top_c, int m, bool 
   r.token_matches = (int32_t*)take(b * 4);
   r.n_cand = (int32_t*)take(b * 4);
   r.status = (uint8_t*)take(b);
-  r.cand_id = cand ? (int32_t*)take(bc * 4) : nullptr;
-  r.cand_score = cand ? (float*)take(bc * 4) : nullptr;
-  r.cand_prefix_score = cand ? (float*)take(bc * 4) : nullptr;
-  r.cand_matches = cand ? (int32_t*)take(bc * 4) : nullptr;
-  r.prefix_scores = scores ? (float*)take(b * m * 4) : nullptr;
+  r.cand_id = want.cand_id ? (int32_t*)take(bc * 4) : nullptr;
+  r.cand_score = want.cand_score ? (float*)take(bc * 4) : nullptr;
+  r.cand_prefix_score = want.cand_prefix_score ? (float*)take(bc * 4) : nullptr;
+  r.cand_matches = want.cand_matches ? (int32_t*)take(bc * 4) : nullptr;
+  r.prefix_scores = want.prefix_scores ? (float*)take(b * m * 4) : nullptr;
+  r.cand_pass = want.cand_pass ? (uint8_t*)take(bc) : nullptr;
+  r.cand_prefix_scores = want.cand_prefix_scores ? (float*)take(bc * m * 4) : nullptr;
   *bytes = (size_t)(p - base);
   return r;
 }
@@ -520,14 +523,11 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
     gather_host_kernel<<<grid, 256, 0, st>>>(g);
     if (cudaGetLastError() != cudaSuccess) return LACACHE_ERR_CUDA;
   }
-  const bool cand = out_host->cand_id || out_host->cand_score || out_host->cand_prefix_score ||
-                    out_host->cand_matches;
-  const bool scores = out_host->prefix_scores != nullptr;
   size_t bytes = 0;
   // Results: written by the kernels straight into the mapped pinned staging when the device can map it.
   unsigned char* out_stage = h->stage_host_dev ? h->stage_host_dev : h->stage_out;
-  lacache_result dev = staged_result(out_stage, B, c.top_c, h->ens.m, cand, scores, &bytes);
-  lacache_result host = staged_result(h->stage_host, B, c.top_c, h->ens.m, cand, scores, &bytes);
+  lacache_result dev = staged_result(out_stage, B, c.top_c, h->ens.m, *out_host, &bytes);
+  lacache_result host = staged_result(h->stage_host, B, c.top_c, h->ens.m, *out_host, &bytes);
   lacache_status s = run_lookup(h, B, q_emb, q_pre, q_ids, dev, st);
   if (s != LACACHE_OK) return s;
   if (!h->stage_host_dev &&
@@ -546,6 +546,8 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
       {out_host->cand_id, host.cand_id, bc4},          {out_host->cand_score, host.cand_score, bc4},
       {out_host->cand_prefix_score, host.cand_prefix_score, bc4}, {out_host->cand_matches, host.cand_matches, bc4},
       {out_host->prefix_scores, host.prefix_scores, b4 * h->ens.m},
+      {out_host->cand_pass, host.cand_pass, (size_t)B * c.top_c},
+      {out_host->cand_prefix_scores, host.cand_prefix_scores, bc4 * h->ens.m},
   };
   for (const Copy& cp : copies)
     if (cp.dst && cp.src) memcpy(cp.dst, cp.src, cp.bytes);

@@ -176,6 +176,16 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
   }
   __syncthreads();
 
+  // candidate i passes the lookahead check under the check mode
+  const int tmin = a.token_match_min > 0 ? a.token_match_min : k;
+  auto passes = [&](int i) {
+    const bool emb_ok = cand_emb_ok[i] != 0;
+    const bool tok_ok = cand_m[i] >= tmin;
+    return a.check_mode == LACACHE_CHECK_EMB ? emb_ok
+           : a.check_mode == LACACHE_CHECK_TOKENS ? tok_ok
+                                                  : (emb_ok && tok_ok);
+  };
+
   // optional per-candidate outputs
   const float qnan = __int_as_float(0x7fc00000);
   for (int i = threadIdx.x; i < C; i += kThreads) {
@@ -185,20 +195,16 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
     if (a.out.cand_score) a.out.cand_score[o] = v ? cand_score(cand[i]) : qnan;
     if (a.out.cand_prefix_score) a.out.cand_prefix_score[o] = v ? cand_rm[i][0] : qnan;
     if (a.out.cand_matches) a.out.cand_matches[o] = v ? cand_m[i] : -1;
+    if (a.out.cand_pass) a.out.cand_pass[o] = v && passes(i) ? 1 : 0;
+    if (a.out.cand_prefix_scores)
+      for (int h = 0; h < a.m; ++h) a.out.cand_prefix_scores[o * a.m + h] = v ? cand_rm[i][h] : qnan;
   }
 
   // 3. decision: the first candidate, in C_q order, that passes
   if (threadIdx.x == 0) {
-    const int tmin = a.token_match_min > 0 ? a.token_match_min : k;
     int served = -1;
-    for (int i = 0; i < n_cand && served < 0; ++i) {
-      const bool emb_ok = cand_emb_ok[i] != 0;
-      const bool tok_ok = cand_m[i] >= tmin;
-      const bool pass = a.check_mode == LACACHE_CHECK_EMB ? emb_ok
-                        : a.check_mode == LACACHE_CHECK_TOKENS ? tok_ok
-                                                               : (emb_ok && tok_ok);
-      if (pass) served = i;
-    }
+    for (int i = 0; i < n_cand && served < 0; ++i)
+      if (passes(i)) served = i;
     const int shown = served >= 0 ? served : 0;   // the candidate whose scores are reported
     if (served >= 0) {
       a.out.status[q] = LACACHE_HIT;

@@ -20,11 +20,12 @@ LACACHE_STAGE1_TENSOR_PAIR = 4   # reported by lacache_last_launch only
 LACACHE_MISS_KEY, LACACHE_HIT, LACACHE_REJECT = 0, 1, 2
 
 LACACHE_MAX_MODELS = 8
+LACACHE_MAX_SHARDS = 16
 
 EXPORTS = ["lacache_create", "lacache_create_ensemble", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
            "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
            "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_enable_lsh", "lacache_read_signatures", "lacache_calibrate", "lacache_calibrate_workspace_bytes", "lacache_verify_draft",
-           "lacache_lookup_noalloc",
+           "lacache_lookup_noalloc", "lacache_merge_shards",
            "lacache_status_string"]
 
 
@@ -43,7 +44,14 @@ class lacache_ensemble(ctypes.Structure):
 class lacache_result(ctypes.Structure):
     _fields_ = [(name, ctypes.c_void_p) for name in
                 ("entry_id", "status", "key_score", "prefix_score", "token_matches", "n_cand",
-                 "cand_id", "cand_score", "cand_prefix_score", "cand_matches", "prefix_scores")]
+                 "cand_id", "cand_score", "cand_prefix_score", "cand_matches", "prefix_scores", "cand_pass",
+                 "cand_prefix_scores")]
+
+
+class lacache_shard_result(ctypes.Structure):
+    _fields_ = [(name, ctypes.c_void_p) for name in
+                ("cand_id", "cand_score", "cand_prefix_score", "cand_matches", "cand_pass", "cand_prefix_scores",
+                 "key_score", "n_cand")] + [("id_base", ctypes.c_int64)]
 
 
 class LacacheError(RuntimeError):
@@ -90,6 +98,8 @@ def load() -> ctypes.CDLL:
         "lacache_verify_draft": ([i32, i32, vp, vp, vp, vp, vp], i32),
         "lacache_lookup_noalloc": ([ctypes.POINTER(lacache_config), i64, vp, vp, vp, i32, vp, vp, vp,
                                     ctypes.POINTER(lacache_result), vp], i32),
+        "lacache_merge_shards": ([i32, ctypes.POINTER(lacache_shard_result), i32, i32, i32,
+                                  ctypes.POINTER(lacache_result), vp], i32),
         "lacache_status_string": ([i32], ctypes.c_char_p),
     }
     for name, (args, res) in sig.items():
@@ -174,6 +184,19 @@ def lacache_lookup(h: int, q_emb, q_prefix, q_ids, out: dict, cuda_stream=None) 
     res = _result_struct(out)
     _check("lacache_lookup", load().lacache_lookup(h, int(q_emb.shape[0]), _ptr(q_emb), _ptr(q_prefix),
                                                    _ptr(q_ids), ctypes.byref(res), _stream(cuda_stream)))
+
+
+def lacache_merge_shards(shards: list, top_c: int, models: int, out: dict, cuda_stream=None) -> None:
+    """Merge entry-range shards' lookup outputs (``shards``: one (outputs dict, id_base) per shard, outputs as
+    alloc_result(candidates=True) writes them) into ``out``, the whole-store result."""
+    arr = (lacache_shard_result * len(shards))()
+    for g, (o, base) in enumerate(shards):
+        arr[g] = lacache_shard_result(*[_ptr(o.get(name)) for name, _ in lacache_shard_result._fields_[:-1]],
+                                      int(base))
+    res = _result_struct(out)
+    B = int(out["status"].shape[0])
+    _check("lacache_merge_shards", load().lacache_merge_shards(len(shards), arr, B, top_c, models, ctypes.byref(res),
+                                                               _stream(cuda_stream)))
 
 
 def lacache_lookup_host(h: int, q_emb, q_prefix, q_ids, out: dict, cuda_stream=None) -> None:
@@ -267,7 +290,9 @@ def lacache_lookup_noalloc(cfg: lacache_config, key, prefix, ids, q_emb, q_prefi
 
 def alloc_result(batch: int, top_c: int, device, candidates: bool = True, pinned: bool = False,
                  models: int = 0) -> dict:
-    """Output buffers of one lookup: device tensors (or pinned host tensors with ``device="cpu"``)."""
+    """Output buffers of one lookup: device tensors (or pinned host tensors with ``device="cpu"``). ``candidates``
+    adds the per-candidate arrays (with their pass bits); ``models`` > 0 adds every model's lookahead scores, for
+    the shown candidate and, with ``candidates``, per candidate."""
     import torch
     kw = {"device": device}
     if pinned:
@@ -282,9 +307,12 @@ def alloc_result(batch: int, top_c: int, device, candidates: bool = True, pinned
         out.update({"cand_id": torch.empty((batch, top_c), dtype=torch.int32, **kw),
                     "cand_score": torch.empty((batch, top_c), dtype=torch.float32, **kw),
                     "cand_prefix_score": torch.empty((batch, top_c), dtype=torch.float32, **kw),
-                    "cand_matches": torch.empty((batch, top_c), dtype=torch.int32, **kw)})
+                    "cand_matches": torch.empty((batch, top_c), dtype=torch.int32, **kw),
+                    "cand_pass": torch.empty((batch, top_c), dtype=torch.uint8, **kw)})
     if models:
         out["prefix_scores"] = torch.empty((batch, models), dtype=torch.float32, **kw)
+        if candidates:
+            out["cand_prefix_scores"] = torch.empty((batch, top_c, models), dtype=torch.float32, **kw)
     return out
 
 

@@ -141,7 +141,7 @@ def compare(gpu: dict, res: oracle.Result, p: oracle.Params, rows=None, pair_sco
         if res.list_margin[b] >= TOL:
             assert gpu["n_cand"][g] == res.n_cand[b], f"{msg}: n_cand {gpu['n_cand'][g]} vs {res.n_cand[b]}"
         if "cand_id" in gpu:
-            _compare_candidates(gpu, res, g, b, rep, msg)
+            _compare_candidates(gpu, res, g, b, rep, msg, p)
         rep.exact += 1
         rep.hits += st == oracle.HIT
         rep.rejects += st == oracle.REJECT
@@ -159,7 +159,15 @@ def pair_scores_fn(store: oracle.Store, oq: dict):
     return f
 
 
-def _compare_candidates(gpu, res, g, b, rep, msg):
+def _pass_settled(res, b, i, p) -> bool:
+    """Candidate i's pass bit is not within the tolerance of flipping (every threshold it uses is clear)."""
+    if p.check_mode == oracle.CHECK_TOKENS:
+        return True
+    taus = p.tau_a_models if p.prefix_dims is not None else (p.tau_a,)
+    return all(abs(res.cand_prefix_scores[b, i, h] - t) >= TOL for h, t in enumerate(taus))
+
+
+def _compare_candidates(gpu, res, g, b, rep, msg, p):
     nc = int(res.n_cand[b])
     c = res.cand_id.shape[1]
     ng = int(gpu["n_cand"][g])
@@ -177,12 +185,20 @@ def _compare_candidates(gpu, res, g, b, rep, msg):
             assert gid == o_ids[i], f"{msg}: candidate {i} id {gid} vs {o_ids[i]}"
             assert _close(gpu["cand_prefix_score"][g, i], res.cand_prefix_score[b, i]), f"{msg}: cand r {i}"
             assert gpu["cand_matches"][g, i] == res.cand_matches[b, i], f"{msg}: cand m {i}"
+            if "cand_pass" in gpu and _pass_settled(res, b, i, p):
+                assert bool(gpu["cand_pass"][g, i]) == bool(res.cand_pass[b, i]), f"{msg}: cand pass {i}"
+            if "cand_prefix_scores" in gpu:
+                for h in range(res.cand_prefix_scores.shape[2]):
+                    assert _close(gpu["cand_prefix_scores"][g, i, h], res.cand_prefix_scores[b, i, h]), \
+                        f"{msg}: cand {i} model {h} score"
         else:
             rep.near_ties += 1
             pos = [k for k, j in enumerate(o_ids) if j == gid]
             assert pos and abs(o_scores[pos[0]] - gs) <= TOL, f"{msg}: tied candidate {gid} not in oracle order"
     for i in range(ng, c):
         assert gpu["cand_id"][g, i] == -1 and np.isnan(gpu["cand_score"][g, i])
+        if "cand_pass" in gpu:
+            assert gpu["cand_pass"][g, i] == 0
 
 
 class StreamedOracle:

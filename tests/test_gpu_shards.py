@@ -1,0 +1,106 @@
+"""Entry-range sharding on one GPU: a store cut into G row ranges, one handle per range, each handle's lookup
+written into its rank's slice of one gathered buffer (as the all-gather of paper_2608_01718_gb300.sharded leaves
+it), then lacache_merge_shards. The merge must reproduce a single whole-store handle's lookup bit for bit, every
+field including the candidate lists. A row's fp32 scores do not depend on which handle or tile holds it. The
+merge must also match the oracle. The shard handles run one after another: no kernel waits on another."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_01718_gb300 import build, sharded
+from paper_2608_01718_gb300 import lacache as L
+from paper_2608_01718_gb300 import workloads as wl
+from parity import compare, log_report, new_cache, oracle_queries, oracle_store, params, fill
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    build.build()
+    L.load()
+
+
+def fill_range(cache, w, a, b):
+    """Insert store rows [a, b) of the workload."""
+    dtype = L.LACACHE_F32 if w.key_dtype == "f32" else L.LACACHE_BF16
+    off = 0
+    for ch in wl.iter_store(w, "cuda"):
+        n = ch["key"].shape[0]
+        lo, hi = max(a, off), min(b, off + n)
+        if lo < hi:
+            cache.insert(ch["key"][lo - off:hi - off], ch["prefix"][lo - off:hi - off], ch["ids"][lo - off:hi - off],
+                         dtype)
+        off += n
+    torch.cuda.synchronize()
+
+
+CASES = {
+    "tiny-2": (wl.WORKLOADS["tiny-4k"], (0, 2048, 4096), L.LACACHE_STAGE1_TENSOR, oracle.CHECK_EMB),
+    "tiny-empty-simt": (wl.WORKLOADS["tiny-4k"], (0, 700, 700, 2901, 4096), L.LACACHE_STAGE1_SIMT, oracle.CHECK_EMB),
+    "tiny-16": (wl.WORKLOADS["tiny-4k"], tuple(range(0, 4097, 256)), L.LACACHE_STAGE1_TENSOR, oracle.CHECK_EMB),
+    "tiny-tokens": (wl.WORKLOADS["tiny-4k"].scaled(n=3000, k=4, vocab=3, batch=48), (0, 1100, 3000),
+                    L.LACACHE_STAGE1_TENSOR, oracle.CHECK_TOKENS),
+    "mid-4": (wl.WORKLOADS["mid-1m"].scaled(n=70_000), (0, 9000, 30_000, 51_234, 70_000), L.LACACHE_STAGE1_TENSOR,
+              oracle.CHECK_EMB),
+    "pairs-3": (wl.WORKLOADS["serve-2m"].scaled(n=12_050, batch=300, clusters=120), (0, 4000, 8000, 12_050),
+                L.LACACHE_STAGE1_TENSOR, oracle.CHECK_EMB),
+    "ensemble-2": (wl.WORKLOADS["ensemble-1m"].scaled(n=20_000, batch=48), (0, 7777, 20_000), L.LACACHE_STAGE1_TENSOR,
+                   oracle.CHECK_EMB),
+}
+
+
+@pytest.mark.parametrize("case", list(CASES))
+def test_merged_shards_equal_the_whole_store_lookup(case):
+    w, cuts, stage1, mode = CASES[case]
+    models = len(w.prefix_dims) if w.prefix_dims is not None else 1
+    B, c = w.batch, w.top_c
+    q = wl.batch(w, 0, device="cuda")
+    with new_cache(w, stage1, check_mode=mode) as whole:
+        fill(whole, w)
+        ref = alloc = L.alloc_result(B, c, "cuda", candidates=True, models=models if models > 1 else 0)
+        whole.lookup(q["emb"], q["prefix"], q["ids"], out=alloc)
+        torch.cuda.synchronize()
+        whole.sync()
+    G = len(cuts) - 1
+    gathered = torch.zeros((G, sharded.record_bytes(B, c, models)), dtype=torch.uint8, device="cuda")
+    shards = []
+    for g, (a, b) in enumerate(zip(cuts, cuts[1:])):
+        with new_cache(w, stage1, check_mode=mode, capacity=max(1, b - a)) as part:
+            fill_range(part, w, a, b)
+            rec = sharded.views(gathered[g], B, c, models)
+            out = {**L.alloc_result(B, c, "cuda", candidates=False), **rec}
+            part.lookup(q["emb"], q["prefix"], q["ids"], out=out)
+            torch.cuda.synchronize()
+            part.sync()
+        shards.append((rec, a))
+    merged = L.alloc_result(B, c, "cuda", candidates=True, models=models if models > 1 else 0)
+    L.lacache_merge_shards(shards, c, models, merged)
+    torch.cuda.synchronize()
+    got = {k: v.cpu().numpy() for k, v in merged.items()}
+    want = {k: v.cpu().numpy() for k, v in ref.items()}
+    assert got.keys() == want.keys()
+    for k in want:
+        assert np.array_equal(got[k], want[k], equal_nan=True), k
+    # and against the oracle, as every lookup is
+    p = params(w, mode)
+    res = oracle.lookup(oracle_store(w), oracle_queries(q), p)
+    rep = compare(got, res, p)
+    log_report(f"{case}: {G} shards merged, n={w.n} B={B}", rep)
+    assert rep.exact + rep.band == B
+    assert len({int(s) for s in got["status"]}) >= 2
+
+
+def test_merge_rejects_bad_arguments():
+    B, c = 4, 2
+    rec = sharded.views(torch.zeros(sharded.record_bytes(B, c, 1), dtype=torch.uint8, device="cuda"), B, c, 1)
+    out = L.alloc_result(B, c, "cuda")
+    no_models = {k: v for k, v in rec.items() if k != "cand_prefix_scores"}
+    for shards, models in [([], 1), ([(rec, 0)] * 17, 1), ([(rec, 10), (rec, 5)], 1), ([(no_models, 0)], 2),
+                           ([(rec, -1)], 1), ([(rec, 0)], 9)]:
+        with pytest.raises(L.LacacheError) as e:
+            L.lacache_merge_shards(shards, c, models, out)
+        assert e.value.status == L.LACACHE_ERR_INVALID_ARG

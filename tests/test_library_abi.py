@@ -39,11 +39,13 @@ def test_status_strings(lib):
 
 
 def test_struct_layouts_match_the_header():
-    # lacache_config: 2 x int32, int64, 2 x float, 6 x int32 = 48 bytes; lacache_result: 11 pointers;
+    # lacache_config: 2 x int32, int64, 2 x float, 6 x int32 = 48 bytes; lacache_result: 13 pointers;
+    # lacache_shard_result: 8 pointers and an int64;
     # lacache_ensemble: int32 + 8 int32 + 8 float
     assert ctypes.sizeof(lacache.lacache_config) == 48
     assert lacache.lacache_config.capacity.offset == 8
-    assert ctypes.sizeof(lacache.lacache_result) == 88
+    assert ctypes.sizeof(lacache.lacache_result) == 104
+    assert ctypes.sizeof(lacache.lacache_shard_result) == 72
     assert ctypes.sizeof(lacache.lacache_ensemble) == 68
 
 
