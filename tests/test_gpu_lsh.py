@@ -51,7 +51,7 @@ def test_signatures_match_the_oracle(bits):
     assert amb.mean() < 1e-3
 
 
-@pytest.mark.parametrize("bits", [128, 256])
+@pytest.mark.parametrize("bits", [128, 256, 512])
 def test_lsh_lookup_matches_the_oracle(bits):
     w = wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=40)
     radius = wl.lsh_radius(w.tau_c, bits)
