@@ -27,6 +27,8 @@
 #include <cuda.h>
 #include <string.h>
 
+#include <atomic>
+
 #include "internal.cuh"
 
 namespace lc {
@@ -42,6 +44,7 @@ constexpr int kEpiWarps = 4;
 constexpr long long kWaitCycles = 2000000000LL;   // about one second of SM clock
 constexpr int RING = 4;                             // tile-index ring of the dynamic schedule
 constexpr size_t kStashBytes = 32 * 129 * 4;          // epilogue's rare-path chunk stash
+constexpr int kMaxDeviceSlots = 64;                   // devices whose CTA-pair capacity is cached
 
 // Per-CTA geometry. Single CTA: the whole 256-key box per stage, 4 stages. CTA pair: half the key box, so 6
 // stages fit in the same shared memory.
@@ -728,8 +731,18 @@ bool encode_rows(EncodeTiledFn encode, CUtensorMap* m, const void* base, int64_t
 template <int CPAD>
 bool launch_pairs(TcParams p, const Stage1Args& a, EncodeTiledFn encode, int max_splits, cudaStream_t st,
                   int* splits, cudaError_t* err) {
-  static int clusters = -1;   // per process: the device model does not change under a running process
-  if (clusters < 0) clusters = max_pair_clusters<CPAD>(st);
+  // per device and kernel instance, asked once (an idempotent query: concurrent first calls store the same value)
+  static std::atomic<int> cache[kMaxDeviceSlots];
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDeviceSlots) {
+    cudaGetLastError();
+    return false;
+  }
+  int clusters = cache[dev].load(std::memory_order_relaxed);
+  if (clusters == 0) {
+    clusters = max_pair_clusters<CPAD>(st);
+    cache[dev].store(clusters < 1 ? -1 : clusters, std::memory_order_relaxed);
+  }
   if (clusters < 1) return false;
   p.pairs = (p.q_tiles + 1) / 2;
   p.a_rows = BM;
