@@ -769,7 +769,7 @@ template <int CPAD>
 cudaError_t launch_key_check(TcParams p, const Stage1Args& a, EncodeTiledFn encode, int num_sms, int max_splits,
                              cudaStream_t st, int* splits, bool* paired) {
   cudaError_t err = cudaSuccess;
-  if (p.q_tiles >= 2 && !p.inject_stall && launch_pairs<CPAD>(p, a, encode, max_splits, st, splits, &err)) {
+  if (p.q_tiles >= 2 && launch_pairs<CPAD>(p, a, encode, max_splits, st, splits, &err)) {
     if (paired) *paired = true;
     return err;
   }

@@ -3,7 +3,9 @@
 lacache_inject_stall makes the tensor kernel's first CTA withhold one TMA load (no copy is issued). The MMA
 issuer's bounded wait then runs out (about a second). The kernel records the timeout in the status word, drains
 and exits, and lacache_sync reports LACACHE_ERR_DEVICE_TIMEOUT. The context must stay usable: the next lookup
-matches the one taken before the injection.
+matches the one taken before the injection. With B = 256 the batch runs on CTA pairs: the withholding CTA is the
+leader of the first pair, whose abort also stops its peer; both CTAs still meet at the cluster barrier before
+freeing the pair's TMEM.
 """
 import pytest
 import torch
@@ -23,8 +25,9 @@ def library():
     L.load()
 
 
-def test_stage1_wait_timeout_is_reported_and_the_context_stays_usable():
-    w = wl.WORKLOADS["mid-1m"].scaled(n=40_000)
+@pytest.mark.parametrize("batch", [32, 256], ids=["single-cta", "cta-pairs"])
+def test_stage1_wait_timeout_is_reported_and_the_context_stays_usable(batch):
+    w = wl.WORKLOADS["mid-1m"].scaled(n=40_000, batch=batch)
     with L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch,
                    stage1=L.LACACHE_STAGE1_TENSOR) as cache:
         for ch in wl.iter_store(w, "cuda"):
@@ -34,6 +37,7 @@ def test_stage1_wait_timeout_is_reported_and_the_context_stays_usable():
         cache.sync()
         L.lacache_inject_stall(cache.h, 1)
         cache.lookup(q["emb"], q["prefix"], q["ids"])
+        assert cache.last_launch()[1] == (L.LACACHE_STAGE1_TENSOR_PAIR if batch > 128 else L.LACACHE_STAGE1_TENSOR)
         with pytest.raises(L.LacacheError) as e:
             cache.sync()
         assert e.value.status == L.LACACHE_ERR_DEVICE_TIMEOUT
