@@ -3,6 +3,7 @@ compute calls are made here)."""
 import ctypes
 import os
 import re
+import subprocess
 
 import pytest
 
@@ -20,6 +21,22 @@ def lib():
 def declared_functions():
     text = open(HEADER).read()
     return sorted(set(re.findall(r"^\s*(?:lacache_status|const char\*|size_t)\s+(lacache_\w+)\s*\(", text, re.M)))
+
+
+def test_header_is_strict_c99(tmp_path):
+    src = tmp_path / "uses_header.c"
+    src.write_text('#include "lacache.h"\nint main(void) { return lacache_status_string(LACACHE_OK) == 0; }\n')
+    res = subprocess.run(["gcc", "-std=c99", "-Wall", "-Wextra", "-Wpedantic", "-Werror", "-fsyntax-only",
+                          "-I", os.path.dirname(HEADER), str(src)], capture_output=True, text=True)
+    assert res.returncode == 0, res.stderr
+
+
+def test_c_client_compiles_against_the_header(tmp_path):
+    client = os.path.join(os.path.dirname(os.path.abspath(__file__)), "c_client", "lookup_client.c")
+    cuda_inc = os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "include")
+    res = subprocess.run(["gcc", "-std=c99", "-Wall", "-Wextra", "-Werror", "-fsyntax-only", "-I",
+                          os.path.dirname(HEADER), "-I", cuda_inc, client], capture_output=True, text=True)
+    assert res.returncode == 0, res.stderr
 
 
 def test_header_declares_the_binding_names():
