@@ -382,6 +382,7 @@ def run_ours(args, w):
                 "api": "lacache_lookup_host (pinned host buffers, synchronous)"},
         "gpu_launches": (3 if lsh else 2) * args.steps,
         "clocks": clock,
+        "decisions": decision_rates(w, batches[0], outs[0]),
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w)
@@ -391,6 +392,28 @@ def run_ours(args, w):
     if world > 1:
         dist.destroy_process_group()
     return 0
+
+
+def decision_rates(w, q: dict, out: dict) -> dict:
+    """The paper's hit metrics (section 4.1) on one looked-up batch, from the generator's query classes: the
+    benign hit rate (near-duplicates served their own target), the attack hit rate (collision and mimic queries
+    served anything), and the attack hit rate a key check alone would give (those with a candidate above tau_c),
+    which the lookahead check brings down."""
+    import numpy as np
+
+    from paper_2608_01718_gb300 import lacache as L
+    from paper_2608_01718_gb300 import workloads as wl
+    cls, tgt = q["class"].cpu().numpy(), q["target"].cpu().numpy()
+    status, entry = out["status"].cpu().numpy(), out["entry_id"].cpu().numpy()
+    n_cand = out["n_cand"].cpu().numpy()
+    near = cls == wl.NEAR
+    attack = (cls == wl.COLLISION) | (cls == wl.MIMIC)
+    rate = lambda m: float(np.mean(m)) if m.size else None
+    return {"queries": int(len(cls)), "near_duplicate": int(near.sum()), "attack": int(attack.sum()),
+            "benign_hit_rate": rate((status[near] == L.LACACHE_HIT) & (entry[near] == tgt[near])),
+            "attack_hit_rate": rate(status[attack] == L.LACACHE_HIT),
+            "attack_hit_rate_key_check_only": rate(n_cand[attack] > 0),
+            "random_hit_rate": rate(status[cls == wl.RANDOM] == L.LACACHE_HIT)}
 
 
 def cpu_baseline(w) -> dict:
@@ -541,6 +564,7 @@ def run_sharded(args, w):
                 "api": "paper_2608_01718_gb300.sharded.ShardedLookup (pinned host buffers, synchronous per step)"},
         "gpu_launches": 3 * args.steps,
         "clocks": clock,
+        "decisions": decision_rates(w, batches[0], outs[0]),
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(w)

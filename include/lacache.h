@@ -44,7 +44,8 @@ typedef enum {
   LACACHE_ERR_OOM = 3,            /* device allocation failed at create */
   LACACHE_ERR_CUDA = 4,           /* a CUDA runtime call failed */
   LACACHE_ERR_DEVICE_TIMEOUT = 5, /* a kernel's bounded wait ran out (reported by lacache_sync) */
-  LACACHE_ERR_UNSUPPORTED = 6     /* valid but unsupported configuration (e.g. top_c > 32, d % 8 != 0) */
+  LACACHE_ERR_UNSUPPORTED = 6,    /* valid but unsupported configuration (e.g. top_c > 32, d % 8 != 0) */
+  LACACHE_ERR_IO = 7              /* a file could not be opened, read or written, or is not a saved cache */
 } lacache_status;
 
 /* How stage 2 decides that candidate x' passes the lookahead check (Algorithm 1; section 4.1). */
@@ -191,6 +192,37 @@ lacache_status lacache_size(const lacache_t* h, int64_t* n);
 /* Synchronize the handle's device and report any device-side status set by the library's kernels since the
  * previous lacache_sync (the status word is then cleared). */
 lacache_status lacache_sync(lacache_t* h);
+
+/* Persistence of a cache across processes. lacache_save writes the handle's configuration (lacache_config and the
+ * lacache_ensemble of its lookahead checks) and its valid entries to `path`: an 8-byte magic "LACACHE1", a format
+ * version, the two structs and the entry count, then the key rows [n x d] bf16, the prefix rows [n x prefix row]
+ * bf16 and the token ids [n x k] int32, all little-endian. It synchronizes the handle's device first, so every
+ * insert and append issued before the call is saved. A SimHash index is not saved: enable it again after loading.
+ * lacache_load creates a new handle on `device` from such a file, with the saved configuration; capacity > 0
+ * replaces the saved capacity (it must hold the saved entries, else LACACHE_ERR_CAPACITY). Entry ids are kept.
+ * A file that cannot be read, or is not a saved cache, gives LACACHE_ERR_IO before any device is touched. */
+lacache_status lacache_save(lacache_t* h, const char* path);
+/* The handle's configuration and lookahead checks, as created or loaded (either pointer may be NULL). */
+lacache_status lacache_get_config(const lacache_t* h, lacache_config* cfg, lacache_ensemble* ens);
+lacache_status lacache_load(const char* path, int32_t device, int64_t capacity, lacache_t** out);
+
+/* Decision counters of a handle (section 4.1's hit metrics count these outcomes): lookups and queries looked up,
+ * and of those queries the HITs, lookahead rejections (REJECT) and key misses (MISS_KEY); entries inserted and
+ * misses appended. */
+typedef struct {
+  int64_t lookups;
+  int64_t queries;
+  int64_t hits;
+  int64_t rejects;
+  int64_t key_misses;
+  int64_t inserted;
+  int64_t appended;
+} lacache_stats;
+
+/* The counters since create or the last reset (reset != 0 zeroes them after reading). Synchronizes the handle's
+ * device: every lookup issued before the call is counted. Lookups through lacache_lookup_noalloc have no handle
+ * and are not counted. */
+lacache_status lacache_get_stats(lacache_t* h, lacache_stats* out, int32_t reset);
 
 /* Number of stage-1 partial lists the last lookup used, and which stage-1 kernel it ran (lacache_stage1; a
  * tensor-core lookup reports LACACHE_STAGE1_TENSOR or LACACHE_STAGE1_TENSOR_PAIR). */

@@ -2,6 +2,7 @@
 // update of the serve loop, and the dispatch of a lookup to the stage-1 and stage-2 kernels.
 #include <cuda.h>
 #include <math.h>
+#include <stdio.h>
 #include <stdlib.h>
 #include <string.h>
 
@@ -37,6 +38,8 @@ struct lacache {
   int inject_stall;          // lookups left that withhold one stage-1 load (failure-detection tests)
   int* tile_ctr;             // two tile counters of the dynamic stage-1 schedule, used alternately
   int64_t tc_launches;       // tensor stage-1 launches so far (selects the counter)
+  unsigned long long* counters;  // device: decisions [hits, rejects, key misses] (stage 2 adds per query)
+  int64_t lookups, queries, inserted, appended;   // host-side counters
   int lsh_bits;              // SimHash index: signature bits (0 = no index)
   int lsh_radius;
   uint32_t* sig;             // [capacity x lsh_bits/32] entry signatures
@@ -246,6 +249,7 @@ void free_all(lacache* h) {
   cudaFree(h->append_dst);
   cudaFree(h->append_count);
   cudaFree(h->tile_ctr);
+  cudaFree(h->counters);
   cudaFree(h->stage_in);
   cudaFree(h->stage_out);
   if (h->append_count_host) cudaFreeHost(h->append_count_host);
@@ -321,11 +325,14 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
   b.q_prefix = reinterpret_cast<const __nv_bfloat16*>(q_prefix);
   b.q_ids = q_ids;
   b.out = out;
+  b.counters = h->counters;
   if (ev && cudaEventRecord(ev[1], st) != cudaSuccess) return LACACHE_ERR_CUDA;
   if (lc::launch_stage2(b, st) != cudaSuccess) return LACACHE_ERR_CUDA;
   if (ev && cudaEventRecord(ev[2], st) != cudaSuccess) return LACACHE_ERR_CUDA;
   h->last_splits = splits;
   h->last_kernel = kernel;
+  ++h->lookups;
+  h->queries += B;
   return LACACHE_OK;
 }
 
@@ -346,6 +353,7 @@ const char* lacache_status_string(lacache_status s) {
     case LACACHE_ERR_CUDA: return "CUDA error";
     case LACACHE_ERR_DEVICE_TIMEOUT: return "device wait timed out";
     case LACACHE_ERR_UNSUPPORTED: return "unsupported configuration";
+    case LACACHE_ERR_IO: return "i/o error";
   }
   return "unknown status";
 }
@@ -409,6 +417,8 @@ lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_
             cudaMalloc(&h->append_dst, (size_t)c.max_batch * 4) == cudaSuccess &&
             cudaMalloc(&h->append_count, 4) == cudaSuccess &&
             cudaMalloc(&h->tile_ctr, 2 * sizeof(int)) == cudaSuccess &&
+            cudaMalloc(&h->counters, 3 * sizeof(unsigned long long)) == cudaSuccess &&
+            cudaMemset(h->counters, 0, 3 * sizeof(unsigned long long)) == cudaSuccess &&
             cudaMemset(h->tile_ctr, 0, 2 * sizeof(int)) == cudaSuccess &&
             cudaMalloc(&h->stage_in, stage_in_bytes(c, pd)) == cudaSuccess &&
             cudaMalloc(&h->stage_out, stage_out_bytes(c, ens->m)) == cudaSuccess &&
@@ -448,6 +458,7 @@ lacache_status lacache_destroy(lacache_t* h) {
 
 lacache_status lacache_insert(lacache_t* h, int64_t n, const void* key_dev, const void* prefix_dev,
                               const int32_t* ids_dev, int32_t dtype, int64_t* first_id, void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_insert");
   if (!h || n < 0) return LACACHE_ERR_INVALID_ARG;
   if (dtype != LACACHE_BF16 && dtype != LACACHE_F32) return LACACHE_ERR_INVALID_ARG;
   if (n > 0 && (!key_dev || !prefix_dev || !ids_dev)) return LACACHE_ERR_INVALID_ARG;
@@ -478,11 +489,13 @@ lacache_status lacache_insert(lacache_t* h, int64_t n, const void* key_dev, cons
   if (e == cudaSuccess) e = sign_rows(h, h->n, n, st);
   if (e != cudaSuccess) return LACACHE_ERR_CUDA;
   h->n += n;
+  h->inserted += n;
   return LACACHE_OK;
 }
 
 lacache_status lacache_lookup(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
                               const int32_t* q_ids_dev, const lacache_result* out, void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_lookup");
   if (!h || B < 1 || B > h->cfg.max_batch) return LACACHE_ERR_INVALID_ARG;
   if (!q_emb_dev || !q_prefix_dev || !q_ids_dev || !result_ok(out)) return LACACHE_ERR_INVALID_ARG;
   if (!aligned16(q_emb_dev) || !aligned16(q_prefix_dev)) return LACACHE_ERR_INVALID_ARG;
@@ -493,6 +506,7 @@ lacache_status lacache_lookup(lacache_t* h, int32_t B, const void* q_emb_dev, co
 
 lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_host, const void* q_prefix_host,
                                    const int32_t* q_ids_host, const lacache_result* out_host, void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_lookup_host");
   if (!h || B < 1 || B > h->cfg.max_batch) return LACACHE_ERR_INVALID_ARG;
   if (!q_emb_host || !q_prefix_host || !q_ids_host || !result_ok(out_host)) return LACACHE_ERR_INVALID_ARG;
   DeviceGuard guard(h->cfg.device);
@@ -557,6 +571,7 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
 lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
                                      const int32_t* q_ids_dev, const uint8_t* status_dev, int64_t* first_id,
                                      int64_t* n_appended, void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_append_misses");
   if (!h || B < 1 || B > h->cfg.max_batch) return LACACHE_ERR_INVALID_ARG;
   if (!q_emb_dev || !q_prefix_dev || !q_ids_dev || !status_dev) return LACACHE_ERR_INVALID_ARG;
   if (!aligned16(q_emb_dev) || !aligned16(q_prefix_dev)) return LACACHE_ERR_INVALID_ARG;
@@ -579,11 +594,13 @@ lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_
   if (first_id) *first_id = h->n;
   if (n_appended) *n_appended = m;
   h->n += m;
+  h->appended += m;
   return LACACHE_OK;
 }
 
 lacache_status lacache_enable_lsh(lacache_t* h, int32_t bits, int32_t radius, const void* hyperplanes_dev,
                                   void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_enable_lsh");
   if (!h || !hyperplanes_dev || ((uintptr_t)hyperplanes_dev & 15u)) return LACACHE_ERR_INVALID_ARG;
   if (bits != 128 && bits != 256 && bits != 512) return LACACHE_ERR_UNSUPPORTED;
   if (radius < 0 || radius > bits) return LACACHE_ERR_INVALID_ARG;
@@ -700,6 +717,155 @@ lacache_status lacache_stage_times(lacache_t* h, double* stage1_ms, double* stag
 lacache_status lacache_inject_stall(lacache_t* h, int32_t lookups) {
   if (!h || lookups < 0) return LACACHE_ERR_INVALID_ARG;
   h->inject_stall = lookups;
+  return LACACHE_OK;
+}
+
+}  // extern "C"
+
+namespace {
+
+// Saved-cache file header (little-endian, fixed-width fields; padding is written as zeros).
+constexpr char kFileMagic[8] = {'L', 'A', 'C', 'A', 'C', 'H', 'E', '1'};
+constexpr uint32_t kFileVersion = 1;
+struct FileHeader {
+  char magic[8];
+  uint32_t version;
+  uint32_t header_bytes;
+  lacache_config cfg;
+  lacache_ensemble ens;
+  int64_t n;
+};
+constexpr size_t kIoChunk = (size_t)64 << 20;   // bytes per staged copy
+
+// Copies `bytes` between a device array and a file through a pinned staging buffer of at most kIoChunk bytes.
+bool copy_out(FILE* f, const void* dev, size_t bytes, unsigned char* stage) {
+  for (size_t off = 0; off < bytes; off += kIoChunk) {
+    const size_t len = bytes - off < kIoChunk ? bytes - off : kIoChunk;
+    if (cudaMemcpy(stage, static_cast<const unsigned char*>(dev) + off, len, cudaMemcpyDeviceToHost) != cudaSuccess ||
+        fwrite(stage, 1, len, f) != len)
+      return false;
+  }
+  return true;
+}
+bool copy_in(FILE* f, void* dev, size_t bytes, unsigned char* stage) {
+  for (size_t off = 0; off < bytes; off += kIoChunk) {
+    const size_t len = bytes - off < kIoChunk ? bytes - off : kIoChunk;
+    if (fread(stage, 1, len, f) != len ||
+        cudaMemcpy(static_cast<unsigned char*>(dev) + off, stage, len, cudaMemcpyHostToDevice) != cudaSuccess)
+      return false;
+  }
+  return true;
+}
+
+}  // namespace
+
+extern "C" {
+
+lacache_status lacache_save(lacache_t* h, const char* path) {
+  lc::NvtxRange nvtx("lacache_save");
+  if (!h || !path) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok() || cudaDeviceSynchronize() != cudaSuccess) return LACACHE_ERR_CUDA;
+  FileHeader hdr;
+  memset(&hdr, 0, sizeof hdr);
+  memcpy(hdr.magic, kFileMagic, sizeof kFileMagic);
+  hdr.version = kFileVersion;
+  hdr.header_bytes = (uint32_t)sizeof hdr;
+  hdr.cfg = h->cfg;
+  hdr.ens = h->ens;
+  hdr.n = h->n;
+  FILE* f = fopen(path, "wb");
+  if (!f) return LACACHE_ERR_IO;
+  const size_t n = (size_t)h->n;
+  const size_t sizes[3] = {n * h->cfg.d * 2, n * h->pd * 2, n * h->cfg.k * 4};
+  unsigned char* stage = nullptr;
+  lacache_status s = LACACHE_OK;
+  if (cudaMallocHost(&stage, kIoChunk) != cudaSuccess) {
+    cudaGetLastError();
+    s = LACACHE_ERR_OOM;
+  } else if (fwrite(&hdr, 1, sizeof hdr, f) != sizeof hdr || !copy_out(f, h->key, sizes[0], stage) ||
+             !copy_out(f, h->prefix, sizes[1], stage) || !copy_out(f, h->ids, sizes[2], stage)) {
+    s = LACACHE_ERR_IO;
+  }
+  if (stage) cudaFreeHost(stage);
+  if (fclose(f) != 0 && s == LACACHE_OK) s = LACACHE_ERR_IO;
+  return s;
+}
+
+lacache_status lacache_get_config(const lacache_t* h, lacache_config* cfg, lacache_ensemble* ens) {
+  if (!h) return LACACHE_ERR_INVALID_ARG;
+  if (cfg) *cfg = h->cfg;
+  if (ens) *ens = h->ens;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_load(const char* path, int32_t device, int64_t capacity, lacache_t** out) {
+  lc::NvtxRange nvtx("lacache_load");
+  if (!out) return LACACHE_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!path || capacity < 0) return LACACHE_ERR_INVALID_ARG;
+  FILE* f = fopen(path, "rb");
+  if (!f) return LACACHE_ERR_IO;
+  FileHeader hdr;
+  if (fread(&hdr, 1, sizeof hdr, f) != sizeof hdr || memcmp(hdr.magic, kFileMagic, sizeof kFileMagic) != 0 ||
+      hdr.version != kFileVersion || hdr.header_bytes != sizeof hdr || hdr.n < 0) {
+    fclose(f);
+    return LACACHE_ERR_IO;
+  }
+  lacache_config cfg = hdr.cfg;
+  cfg.device = device;
+  if (capacity > 0) cfg.capacity = capacity;
+  if (cfg.capacity < hdr.n) {
+    fclose(f);
+    return LACACHE_ERR_CAPACITY;
+  }
+  lacache_t* h = nullptr;
+  lacache_status s = lacache_create_ensemble(&cfg, &hdr.ens, &h);
+  if (s != LACACHE_OK) {
+    fclose(f);
+    return s;
+  }
+  DeviceGuard guard(h->cfg.device);
+  const size_t n = (size_t)hdr.n;
+  const size_t sizes[3] = {n * h->cfg.d * 2, n * h->pd * 2, n * h->cfg.k * 4};
+  unsigned char* stage = nullptr;
+  if (!guard.ok() || cudaMallocHost(&stage, kIoChunk) != cudaSuccess) {
+    cudaGetLastError();
+    s = LACACHE_ERR_OOM;
+  } else if (!copy_in(f, h->key, sizes[0], stage) || !copy_in(f, h->prefix, sizes[1], stage) ||
+             !copy_in(f, h->ids, sizes[2], stage)) {
+    s = LACACHE_ERR_IO;
+  }
+  if (stage) cudaFreeHost(stage);
+  fclose(f);
+  if (s != LACACHE_OK) {
+    lacache_destroy(h);
+    return s;
+  }
+  h->n = hdr.n;
+  *out = h;
+  return LACACHE_OK;
+}
+
+lacache_status lacache_get_stats(lacache_t* h, lacache_stats* out, int32_t reset) {
+  if (!h || !out) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  unsigned long long d[3];
+  if (cudaDeviceSynchronize() != cudaSuccess ||
+      cudaMemcpy(d, h->counters, sizeof d, cudaMemcpyDeviceToHost) != cudaSuccess)
+    return LACACHE_ERR_CUDA;
+  out->lookups = h->lookups;
+  out->queries = h->queries;
+  out->hits = (int64_t)d[0];
+  out->rejects = (int64_t)d[1];
+  out->key_misses = (int64_t)d[2];
+  out->inserted = h->inserted;
+  out->appended = h->appended;
+  if (reset) {
+    if (cudaMemset(h->counters, 0, sizeof d) != cudaSuccess) return LACACHE_ERR_CUDA;
+    h->lookups = h->queries = h->inserted = h->appended = 0;
+  }
   return LACACHE_OK;
 }
 

@@ -169,6 +169,7 @@ extern "C" size_t lacache_calibrate_workspace_bytes(void) { return lc::calibrate
 extern "C" lacache_status lacache_calibrate(int64_t n, int32_t d, const void* x_dev, const void* y_dev,
                                             double percentile, float cap, float* sims_dev, float* result_dev,
                                             void* workspace_dev, void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_calibrate");
   if (n < 1 || n > (int64_t)INT32_MAX || d <= 0 || !x_dev || !y_dev || !sims_dev || !result_dev || !workspace_dev)
     return LACACHE_ERR_INVALID_ARG;
   if (!(percentile >= 0.0 && percentile <= 100.0) || isnan(cap)) return LACACHE_ERR_INVALID_ARG;

@@ -7,9 +7,21 @@
 #include <stdint.h>
 #include <string.h>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "lacache.h"
 
 namespace lc {
+
+// An NVTX range over the enclosing scope: each public call appears by name on a profiler's timeline (a no-op when
+// no tool is attached).
+class NvtxRange {
+ public:
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 constexpr int kMaxTopC = 32;
 constexpr int kMaxD = 8192;
@@ -88,6 +100,7 @@ struct Stage2Args {
   const __nv_bfloat16* q_prefix; // [B x pd]
   const int32_t* q_ids;          // [B x k]
   lacache_result out;            // device pointers
+  unsigned long long* counters;  // decision counters [hits, rejects, key misses], or nullptr
 };
 
 // cuTensorMapEncodeTiled, obtained from the driver at run time.

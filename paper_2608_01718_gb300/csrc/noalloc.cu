@@ -71,6 +71,7 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
                                                  const void* q_emb_dev, const void* q_prefix_dev,
                                                  const int32_t* q_ids_dev, const lacache_result* out,
                                                  void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_lookup_noalloc");
   if (!cfg || !out || n < 0 || B < 1) return LACACHE_ERR_INVALID_ARG;
   const lacache_config c = *cfg;
   if (c.d <= 0 || c.k <= 0 || c.top_c <= 0 || isnan(c.tau_c) || isnan(c.tau_a)) return LACACHE_ERR_INVALID_ARG;

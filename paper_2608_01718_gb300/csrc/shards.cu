@@ -140,6 +140,7 @@ __global__ void __launch_bounds__(kWarps * 32) merge_shards_kernel(const __grid_
 extern "C" lacache_status lacache_merge_shards(int32_t G, const lacache_shard_result* shards, int32_t B,
                                                int32_t top_c, int32_t m, const lacache_result* out,
                                                void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_merge_shards");
   if (G < 1 || G > LACACHE_MAX_SHARDS || !shards || B < 1 || top_c < 1 || top_c > lc::kMaxTopC || m < 1 ||
       m > LACACHE_MAX_MODELS || !out)
     return LACACHE_ERR_INVALID_ARG;

@@ -37,6 +37,7 @@ __global__ void __launch_bounds__(kVerifyWarps * 32)
 extern "C" lacache_status lacache_verify_draft(int32_t B, int32_t k, const float* p_target_dev,
                                                const float* p_draft_dev, const uint8_t* status_dev,
                                                int32_t* accepted_dev, void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_verify_draft");
   if (B < 1 || k < 1 || k > lc::kMaxK || !p_target_dev || !p_draft_dev || !accepted_dev)
     return LACACHE_ERR_INVALID_ARG;
   const int blocks = (B + lc::kVerifyWarps - 1) / lc::kVerifyWarps;

@@ -220,6 +220,7 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
     if (a.out.prefix_scores)
       for (int h = 0; h < a.m; ++h) a.out.prefix_scores[(int64_t)q * a.m + h] = n_cand ? cand_rm[shown][h] : qnan;
     a.out.n_cand[q] = n_cand;
+    if (a.counters) atomicAdd(a.counters + (served >= 0 ? 0 : n_cand ? 1 : 2), 1ull);
   }
 }
 

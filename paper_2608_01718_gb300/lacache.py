@@ -12,7 +12,7 @@ import os
 LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_build", "liblacache.so")
 
 LACACHE_OK, LACACHE_ERR_INVALID_ARG, LACACHE_ERR_CAPACITY, LACACHE_ERR_OOM = 0, 1, 2, 3
-LACACHE_ERR_CUDA, LACACHE_ERR_DEVICE_TIMEOUT, LACACHE_ERR_UNSUPPORTED = 4, 5, 6
+LACACHE_ERR_CUDA, LACACHE_ERR_DEVICE_TIMEOUT, LACACHE_ERR_UNSUPPORTED, LACACHE_ERR_IO = 4, 5, 6, 7
 LACACHE_CHECK_EMB, LACACHE_CHECK_TOKENS, LACACHE_CHECK_BOTH = 0, 1, 2
 LACACHE_BF16, LACACHE_F32 = 0, 1
 LACACHE_STAGE1_AUTO, LACACHE_STAGE1_TENSOR, LACACHE_STAGE1_SIMT, LACACHE_STAGE1_LSH = 0, 1, 2, 3
@@ -25,7 +25,8 @@ LACACHE_MAX_SHARDS = 16
 EXPORTS = ["lacache_create", "lacache_create_ensemble", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
            "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
            "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_enable_lsh", "lacache_read_signatures", "lacache_calibrate", "lacache_calibrate_workspace_bytes", "lacache_verify_draft",
-           "lacache_lookup_noalloc", "lacache_merge_shards",
+           "lacache_lookup_noalloc", "lacache_merge_shards", "lacache_get_stats", "lacache_save", "lacache_load",
+           "lacache_get_config",
            "lacache_status_string"]
 
 
@@ -46,6 +47,11 @@ class lacache_result(ctypes.Structure):
                 ("entry_id", "status", "key_score", "prefix_score", "token_matches", "n_cand",
                  "cand_id", "cand_score", "cand_prefix_score", "cand_matches", "prefix_scores", "cand_pass",
                  "cand_prefix_scores")]
+
+
+class lacache_stats(ctypes.Structure):
+    _fields_ = [(name, ctypes.c_int64) for name in
+                ("lookups", "queries", "hits", "rejects", "key_misses", "inserted", "appended")]
 
 
 class lacache_shard_result(ctypes.Structure):
@@ -98,6 +104,10 @@ def load() -> ctypes.CDLL:
         "lacache_verify_draft": ([i32, i32, vp, vp, vp, vp, vp], i32),
         "lacache_lookup_noalloc": ([ctypes.POINTER(lacache_config), i64, vp, vp, vp, i32, vp, vp, vp,
                                     ctypes.POINTER(lacache_result), vp], i32),
+        "lacache_get_stats": ([vp, ctypes.POINTER(lacache_stats), i32], i32),
+        "lacache_save": ([vp, ctypes.c_char_p], i32),
+        "lacache_load": ([ctypes.c_char_p, i32, i64, ctypes.POINTER(vp)], i32),
+        "lacache_get_config": ([vp, ctypes.POINTER(lacache_config), ctypes.POINTER(lacache_ensemble)], i32),
         "lacache_merge_shards": ([i32, ctypes.POINTER(lacache_shard_result), i32, i32, i32,
                                   ctypes.POINTER(lacache_result), vp], i32),
         "lacache_status_string": ([i32], ctypes.c_char_p),
@@ -184,6 +194,32 @@ def lacache_lookup(h: int, q_emb, q_prefix, q_ids, out: dict, cuda_stream=None) 
     res = _result_struct(out)
     _check("lacache_lookup", load().lacache_lookup(h, int(q_emb.shape[0]), _ptr(q_emb), _ptr(q_prefix),
                                                    _ptr(q_ids), ctypes.byref(res), _stream(cuda_stream)))
+
+
+def lacache_get_stats(h: int, reset: bool = False) -> dict:
+    """The handle's decision counters (synchronizes its device); reset zeroes them after reading."""
+    st = lacache_stats()
+    _check("lacache_get_stats", load().lacache_get_stats(h, ctypes.byref(st), int(reset)))
+    return {name: int(getattr(st, name)) for name, _ in lacache_stats._fields_}
+
+
+def lacache_save(h: int, path: str) -> None:
+    """Write the cache (configuration and valid entries) to ``path``."""
+    _check("lacache_save", load().lacache_save(h, os.fsencode(path)))
+
+
+def lacache_load(path: str, device: int = 0, capacity: int = 0) -> int:
+    """A new handle on ``device`` from a saved cache; capacity > 0 replaces the saved capacity."""
+    h = ctypes.c_void_p()
+    _check("lacache_load", load().lacache_load(os.fsencode(path), device, capacity, ctypes.byref(h)))
+    return h.value
+
+
+def lacache_get_config(h: int) -> tuple:
+    """(lacache_config, lacache_ensemble) of a handle."""
+    cfg, ens = lacache_config(), lacache_ensemble()
+    _check("lacache_get_config", load().lacache_get_config(h, ctypes.byref(cfg), ctypes.byref(ens)))
+    return cfg, ens
 
 
 def lacache_merge_shards(shards: list, top_c: int, models: int, out: dict, cuda_stream=None) -> None:
@@ -333,6 +369,19 @@ class LaCache:
             self.models = len(prefix_dims)
             self.h = lacache_create_ensemble(self.cfg, make_ensemble(prefix_dims, tau_a_models))
 
+    @classmethod
+    def load(cls, path: str, device: int = 0, capacity: int = 0) -> "LaCache":
+        """A cache saved with save(), on ``device``."""
+        obj = cls.__new__(cls)
+        obj.h = lacache_load(path, device, capacity)
+        obj.cfg, ens = lacache_get_config(obj.h)
+        obj.device = device
+        obj.models = int(ens.m)
+        return obj
+
+    def save(self, path: str) -> None:
+        lacache_save(self.h, path)
+
     def close(self) -> None:
         if self.h:
             lacache_destroy(self.h)
@@ -359,6 +408,9 @@ class LaCache:
             out = alloc_result(q_emb.shape[0], self.cfg.top_c, q_emb.device, candidates, models=self.models)
         lacache_lookup(self.h, q_emb, q_prefix, q_ids, out, cuda_stream)
         return out
+
+    def stats(self, reset: bool = False) -> dict:
+        return lacache_get_stats(self.h, reset)
 
     def append_misses(self, q_emb, q_prefix, q_ids, status, cuda_stream=None) -> tuple[int, int]:
         return lacache_append_misses(self.h, q_emb, q_prefix, q_ids, status, cuda_stream)

@@ -282,3 +282,24 @@ def test_mid_cache_full_size(stage1):
     rep = run_parity(wl.WORKLOADS["mid-1m"], stage1)
     assert rep.exact + rep.band == 32 and rep.band <= 1
     assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
+
+
+def test_decision_counters_match_the_outputs():
+    w = wl.WORKLOADS["tiny-4k"]
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR, capacity=w.n + 2 * w.batch) as cache:
+        fill(cache, w)
+        assert cache.stats(reset=True)["inserted"] == w.n
+        want = {"hits": 0, "rejects": 0, "key_misses": 0}
+        for step in range(3):
+            q = wl.batch(w, step, device="cuda")
+            out = cache.lookup(q["emb"], q["prefix"], q["ids"])
+            st = out["status"].cpu().numpy()
+            want["hits"] += int((st == L.LACACHE_HIT).sum())
+            want["rejects"] += int((st == L.LACACHE_REJECT).sum())
+            want["key_misses"] += int((st == L.LACACHE_MISS_KEY).sum())
+        _, appended = cache.append_misses(q["emb"], q["prefix"], q["ids"], out["status"])
+        got = cache.stats(reset=True)
+        assert got["lookups"] == 3 and got["queries"] == 3 * w.batch and got["inserted"] == 0
+        assert {k: got[k] for k in want} == want and got["appended"] == appended
+        assert min(want.values()) > 0
+        assert cache.stats() == {k: 0 for k in got}

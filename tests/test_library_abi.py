@@ -51,6 +51,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 def test_status_strings(lib):
     assert lacache.status_string(lacache.LACACHE_OK) == "ok"
+    assert lacache.status_string(lacache.LACACHE_ERR_IO) == "i/o error"
     assert lacache.status_string(lacache.LACACHE_ERR_CAPACITY) == "capacity exceeded"
     assert lacache.status_string(99) == "unknown status"
 
@@ -63,6 +64,7 @@ def test_struct_layouts_match_the_header():
     assert lacache.lacache_config.capacity.offset == 8
     assert ctypes.sizeof(lacache.lacache_result) == 104
     assert ctypes.sizeof(lacache.lacache_shard_result) == 72
+    assert ctypes.sizeof(lacache.lacache_stats) == 56
     assert ctypes.sizeof(lacache.lacache_ensemble) == 68
 
 
@@ -105,3 +107,17 @@ def test_invalid_configs_are_rejected_before_touching_a_device(lib, field, value
     h = ctypes.c_void_p(1)
     assert lib.lacache_create(ctypes.byref(cfg), ctypes.byref(h)) == status
     assert h.value is None
+
+
+def test_load_rejects_what_is_not_a_saved_cache_before_touching_a_device(lib, tmp_path):
+    h = ctypes.c_void_p(1)
+    missing = str(tmp_path / "missing.lacache").encode()
+    assert lib.lacache_load(missing, 0, 0, ctypes.byref(h)) == lacache.LACACHE_ERR_IO and h.value is None
+    bad = tmp_path / "bad.lacache"
+    bad.write_bytes(b"NOTACACHE" + bytes(200))
+    assert lib.lacache_load(str(bad).encode(), 0, 0, ctypes.byref(h)) == lacache.LACACHE_ERR_IO
+    short = tmp_path / "short.lacache"
+    short.write_bytes(b"LACACHE1" + bytes(10))          # magic, then a truncated header
+    assert lib.lacache_load(str(short).encode(), 0, 0, ctypes.byref(h)) == lacache.LACACHE_ERR_IO
+    assert lib.lacache_load(str(short).encode(), 0, -1, ctypes.byref(h)) == lacache.LACACHE_ERR_INVALID_ARG
+    assert lib.lacache_save(None, b"x") == lacache.LACACHE_ERR_INVALID_ARG
