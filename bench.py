@@ -354,7 +354,16 @@ def run_ours(args, w):
     # the stage-1 kernel is bound by HBM below the ridge (flops per byte of the measured peaks), else by the
     # tensor pipe; a kernel timed back to back for over a second is compared with the sustained bf16 peak
     ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
-    if flops / s1_bytes < ridge:
+    if lsh:
+        # the SimHash scan is bound by integer popcounts: B x N x (bits / 32) per lookup, against 16 per clock
+        # per SM (the CUDA arithmetic-throughput table's population-count rate) x SMs x the maximum SM clock
+        sms = torch.cuda.get_device_properties(local_rank).multi_processor_count
+        popc = w.batch * w.n * (lsh["bits"] // 32)
+        roof = {"bound": "alu", "achieved": popc / t1_avg_s / 1e12,
+                "peak": 16 * sms * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12, "unit": "Tpopc/s",
+                "peak_source": f"derived: 16 popcounts/clock/SM x {sms} SMs x max SM clock",
+                "algorithmic_popcounts_per_launch": popc}
+    elif flops / s1_bytes < ridge:
         roof = {"bound": "hbm", "achieved": s1_bytes / t1_avg_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "peak_source": f"{peak_src} (copy bandwidth)"}
     else:
