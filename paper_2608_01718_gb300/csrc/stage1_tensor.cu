@@ -4,9 +4,11 @@
 //
 //   D[m][n] = sum_k Q[qt*128 + m][k] * K[t*256 + n][k]      (bf16 operands, fp32 accumulation in TMEM)
 //
-// Layout of the work: units are (query tile of 128, split of the key tiles); a persistent grid walks them with
-// the query tile varying fastest, so the CTAs that run at the same time stream the same key range and share it
-// through L2. Each CTA:
+// Layout of the work. One query tile (B <= 128): a dynamic schedule, in which CTAs claim 256-key tiles from a
+// global counter (one split per CTA), which balances the tail. Several query tiles: units are (query tile of
+// 128, split of the key tiles), walked by a persistent grid with the query tile varying fastest, so the CTAs that
+// run at the same time stream the same key range and share it through L2; more than one query tile runs on CTA
+// pairs (below). Each CTA:
 //   warp 0      TMA producer: per k-step, one 128x64 query box and one 256x64 key box (128-byte swizzle) into a
 //               4-stage shared-memory ring (mbarrier full/empty pairs);
 //   warp 1      MMA issuer: allocates 512 TMEM columns (two 128x256 fp32 accumulators) and issues
