@@ -82,19 +82,21 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
   // The next lookup's stage 1 may be scheduled now; it too waits for this grid before touching memory.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  // 1a. best key score over all entries (max over the splits' maxima)
-  float best = -INFINITY;
-  for (int s = threadIdx.x; s < a.splits; s += kThreads) best = fmaxf(best, a.part_best[(int64_t)s * a.B + q]);
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(kFull, best, o));
-  if (lane == 0) warp_best[warp] = best;
-
-  // 1b. thread-local top-c of the partial entries
+  // 1a + 1b. The splits' best scores and their partial lists, loaded together (one memory round trip for the
+  // common case of at most 2 x kThreads splits and U x kThreads list entries); then the maximum of the best
+  // scores, and every thread's sorted top-c of the entries it read.
   uint64_t loc[CPAD];
 #pragma unroll
   for (int i = 0; i < CPAD; ++i) loc[i] = 0;
   const int total = a.splits * C;
   constexpr int U = CPAD <= 16 ? 8 : 4;   // loads in flight per thread (one pass for 152 splits x 8)
+  float best = -INFINITY;
+  {
+    const int s0 = threadIdx.x, s1 = threadIdx.x + kThreads;
+    const float b0 = s0 < a.splits ? a.part_best[(int64_t)s0 * a.B + q] : -INFINITY;
+    const float b1 = s1 < a.splits ? a.part_best[(int64_t)s1 * a.B + q] : -INFINITY;
+    best = fmaxf(b0, b1);
+  }
   for (int e0 = threadIdx.x; e0 < total; e0 += U * kThreads) {
     uint64_t x[U];
 #pragma unroll
@@ -112,6 +114,10 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
       keep(loc, x[u]);
     }
   }
+  for (int s = threadIdx.x + 2 * kThreads; s < a.splits; s += kThreads) best = fmaxf(best, a.part_best[(int64_t)s * a.B + q]);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(kFull, best, o));
+  if (lane == 0) warp_best[warp] = best;
   // 1c. per-warp top-c (rounds stop at the first empty maximum: every later one is empty too)
   for (int r = 0; r < C; ++r) {
     const uint64_t m = warp_max_u64(loc[0]);
@@ -156,6 +162,10 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
   for (int i = warp; i < n_cand; i += kWarps) {
     const uint32_t j = cand_id(cand[i]);
     const uint4* pj = reinterpret_cast<const uint4*>(a.prefix + (int64_t)j * pd);
+    const int32_t* tj = a.ids + (int64_t)j * k;
+    // the first 32 token ids of both prefixes, loaded with the prefix rows below rather than after them
+    const bool tl = lane < k;
+    const int32_t tq0 = tl ? __ldg(tq + lane) : 0, tj0 = tl ? __ldg(tj + lane) : 0;
     int emb_ok = 1;
     for (int h = 0; h < a.m; ++h) {
       float acc = 0.f;
@@ -165,9 +175,8 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
       emb_ok &= r >= a.tau_m[h] ? 1 : 0;
       if (lane == 0) cand_rm[i][h] = r;
     }
-    int eq = 0;
-    const int32_t* tj = a.ids + (int64_t)j * k;
-    for (int t = lane; t < k; t += 32) eq += (__ldg(tq + t) == __ldg(tj + t)) ? 1 : 0;
+    int eq = tl && tq0 == tj0 ? 1 : 0;
+    for (int t = lane + 32; t < k; t += 32) eq += (__ldg(tq + t) == __ldg(tj + t)) ? 1 : 0;
     const int m = __reduce_add_sync(kFull, eq);
     if (lane == 0) {
       cand_emb_ok[i] = emb_ok;
