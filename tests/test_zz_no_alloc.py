@@ -45,9 +45,10 @@ def _same(a: dict, b: dict):
         assert np.all(both_nan | (np.abs(x - y) <= TOL) | (x == y)), name
 
 
+@pytest.mark.parametrize("batch", [96, 256], ids=["one-tile", "cta-pairs"])
 @pytest.mark.parametrize("stage1", [L.LACACHE_STAGE1_TENSOR, L.LACACHE_STAGE1_SIMT], ids=["tensor", "simt"])
-def test_noalloc_lookup_matches_the_handle_lookup(stage1):
-    w = wl.WORKLOADS["mid-1m"].scaled(n=50_000, batch=96)
+def test_noalloc_lookup_matches_the_handle_lookup(stage1, batch):
+    w = wl.WORKLOADS["mid-1m"].scaled(n=50_000, batch=batch)
     key, pre, ids = _rows(w)
     with L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch, stage1=stage1) as cache:
         cache.insert(key, pre, ids)
