@@ -303,3 +303,14 @@ def test_decision_counters_match_the_outputs():
         assert {k: got[k] for k in want} == want and got["appended"] == appended
         assert min(want.values()) > 0
         assert cache.stats() == {k: 0 for k in got}
+
+
+@pytest.mark.parametrize("top_c", [1, 2, 16, 32])
+@pytest.mark.parametrize("batch", [40, 200], ids=["single-cta", "cta-pairs"])
+def test_candidate_list_sizes(top_c, batch):
+    # every epilogue list size of the tensor kernel (4, 8, 16, 32 slots), on one query tile and on CTA pairs;
+    # top_c = 1 and 2 also make the candidate cut bind for most near-duplicates and collisions
+    w = wl.WORKLOADS["serve-2m"].scaled(n=20_000, batch=batch, clusters=150, top_c=top_c)
+    rep = run_parity(w, L.LACACHE_STAGE1_TENSOR)
+    assert rep.exact + rep.band == w.batch and rep.band <= 2
+    assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
