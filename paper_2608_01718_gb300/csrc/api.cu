@@ -36,8 +36,7 @@ struct lacache {
   int last_kernel;
   lc::EncodeTiledFn encode;
   int inject_stall;          // lookups left that withhold one stage-1 load (failure-detection tests)
-  int* tile_ctr;             // two tile counters of the dynamic stage-1 schedule, used alternately
-  int64_t tc_launches;       // tensor stage-1 launches so far (selects the counter)
+  int* tile_ctr;             // [next tile, CTAs done] of the dynamic stage-1 schedule (each launch leaves them zero)
   unsigned long long* counters;  // device: decisions [hits, rejects, key misses] (stage 2 adds per query)
   int64_t lookups, queries, inserted, appended;   // host-side counters
   int lsh_bits;              // SimHash index: signature bits (0 = no index)
@@ -284,13 +283,11 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
     cudaError_t e;
     if (kernel == LACACHE_STAGE1_TENSOR) {
       if (!h->encode) return LACACHE_ERR_CUDA;
-      // launch i claims tiles from counter i % 2 and zeroes counter (i + 1) % 2, which served launch i - 1 (that
-      // launch has completed before this one touches memory)
-      a.tile_ctr = h->tile_ctr + (h->tc_launches & 1);
-      a.tile_ctr_next = h->tile_ctr + ((h->tc_launches + 1) & 1);
+      // the kernel leaves the schedule's counters zero for the next launch (the previous one has completed
+      // before this one touches memory)
+      a.tile_ctr = h->tile_ctr;
       bool paired = false;
       e = lc::launch_stage1_tensor(a, h->encode, h->num_sms, h->max_splits, st, &splits, &paired);
-      if (e == cudaSuccess) ++h->tc_launches;
       if (paired) kernel = LACACHE_STAGE1_TENSOR_PAIR;
     } else if (kernel == LACACHE_STAGE1_LSH) {
       e = lc::launch_signatures(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, h->dev_status, h->encode, h->num_sms,

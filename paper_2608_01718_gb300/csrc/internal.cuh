@@ -77,8 +77,9 @@ struct Stage1Args {
   float* part_best;
   unsigned int* dev_status;
   int inject_stall;           // test support: CTA 0 of the tensor kernel withholds one load (see lacache.h)
-  int* tile_ctr;              // tensor kernel, one query tile: dynamic tile schedule on this zeroed counter
-  int* tile_ctr_next;         // the counter the next launch will use; zeroed by this launch (nullptr: static)
+  int* tile_ctr;              // tensor kernel, one query tile: dynamic tile schedule on these two counters
+                              // [next tile, CTAs done], zero at launch and zero again when the grid ends
+                              // (nullptr: static schedule)
 };
 
 struct Stage2Args {

@@ -80,8 +80,7 @@ struct TcParams {
   int k_steps;
   int a_rows;     // rows of the query box: B rounded up to 8 when B <= 128, else 128
   int inject_stall;  // test support: CTA 0 withholds its second load, so its MMA issuer's bounded wait runs out
-  int* tile_ctr;      // dynamic schedule: tile counter to claim from (nullptr: static schedule)
-  int* tile_ctr_next; // the other counter, zeroed here for the next launch (it served the previous one)
+  int* tile_ctr;      // dynamic schedule: [next tile, CTAs done], zero at launch and left zero (nullptr: static)
   uint32_t* sig;     // signature mode: [n x sig_words] output words
   int sig_words;
   uint64_t* part_cand;
@@ -390,7 +389,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   // in increasing order. Static schedule: units (query tile, split of the key tiles) in a fixed order; for a
   // pair, units (pair of query tiles, split) and this CTA takes the pair's tile of its rank.
   const bool dyn = !PAIR && p.tile_ctr != nullptr;
-  if (dyn && threadIdx.x == 0 && blockIdx.x == 0) *p.tile_ctr_next = 0;   // for the next launch (see TcParams)
   const int unit0 = PAIR ? (int)cluster_id_x() : (int)blockIdx.x;
   const int ustep = PAIR ? (int)cluster_count_x() : (int)gridDim.x;
   const int per_split = PAIR ? p.pairs : p.q_tiles;
@@ -445,6 +443,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           mbar_arrive(tid_full_bar(slot));               // release: the index is visible to its readers
           if (done) break;
           ok = load_tile(0, t);
+        }
+        // This CTA has made its last claim. The last CTA of the launch to get here zeroes both counters, so the
+        // next launch (which reads them only after this grid has completed) starts from zero: the schedule keeps
+        // no state on the host, and a lookup captured in a CUDA graph replays correctly.
+        __threadfence();
+        if (atomicAdd(p.tile_ctr + 1, 1) == (int)gridDim.x - 1) {
+          p.tile_ctr[0] = 0;
+          p.tile_ctr[1] = 0;
         }
       } else {
         for (int u = unit0; ok && u < p.units; u += ustep) {
@@ -791,10 +797,7 @@ cudaError_t launch_key_check(TcParams p, const Stage1Args& a, EncodeTiledFn enco
   if (s < 1) s = 1;
   p.splits = s;
   p.units = p.q_tiles * s;
-  if (p.q_tiles == 1 && a.tile_ctr) {
-    p.tile_ctr = a.tile_ctr;
-    p.tile_ctr_next = a.tile_ctr_next;
-  }
+  if (p.q_tiles == 1 && a.tile_ctr) p.tile_ctr = a.tile_ctr;
   *splits = s;
   const int grid = p.units < num_sms ? p.units : num_sms;
   return launch_cpad<CPAD, false, false>(&tq, &tk, p, grid, st);

@@ -314,3 +314,37 @@ def test_candidate_list_sizes(top_c, batch):
     rep = run_parity(w, L.LACACHE_STAGE1_TENSOR)
     assert rep.exact + rep.band == w.batch and rep.band <= 2
     assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
+
+
+@pytest.mark.parametrize("batch", [32, 200], ids=["dynamic-schedule", "cta-pairs"])
+def test_lookup_captured_in_a_cuda_graph_replays_like_eager_lookups(batch):
+    # the stage-1 schedule keeps no host-side state between launches, so one captured lookup can be replayed
+    w = wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch)
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+        fill(cache, w)
+        q0, q1 = wl.batch(w, 0, device="cuda"), wl.batch(w, 1, device="cuda")
+        eager = []
+        for q in (q0, q1):
+            eager.append({k: v.clone() for k, v in cache.lookup(q["emb"], q["prefix"], q["ids"]).items()})
+        torch.cuda.synchronize()
+        cache.sync()
+        inp = {k: q0[k].clone() for k in ("emb", "prefix", "ids")}
+        out = L.alloc_result(w.batch, w.top_c, "cuda")
+        side = torch.cuda.Stream()
+        side.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(side):                 # warm-up on the capture stream, as torch asks
+            L.lacache_lookup(cache.h, inp["emb"], inp["prefix"], inp["ids"], out, side)
+        torch.cuda.current_stream().wait_stream(side)
+        torch.cuda.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, capture_error_mode="relaxed"):
+            L.lacache_lookup(cache.h, inp["emb"], inp["prefix"], inp["ids"], out)
+        for step, want in ((0, eager[0]), (0, eager[0]), (1, eager[1]), (0, eager[0])):
+            src = q0 if step == 0 else q1
+            for k in inp:
+                inp[k].copy_(src[k])
+            graph.replay()
+            torch.cuda.synchronize()
+            cache.sync()
+            for k in out:
+                assert torch.equal(out[k].view(torch.uint8), want[k].view(torch.uint8)), (step, k)
