@@ -174,7 +174,8 @@ lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_
  * cfg->stage1 == LACACHE_STAGE1_LSH a lookup applies the exact key check only to the entries whose signature
  * differs from the query's in at most `radius` bits; stage 2 is unchanged. Existing entries are signed now and
  * later inserts and appends are signed as they arrive. Allocates (capacity + max_batch) * bits / 8 bytes.
- * Asynchronous on cuda_stream; calling it again replaces the index. */
+ * Asynchronous on cuda_stream; calling it again replaces the index. A lookup on a handle whose cfg->stage1 is
+ * LACACHE_STAGE1_LSH returns LACACHE_ERR_INVALID_ARG, and runs nothing, until this call has been made. */
 lacache_status lacache_enable_lsh(lacache_t* h, int32_t bits, int32_t radius, const void* hyperplanes_dev,
                                   void* cuda_stream);
 

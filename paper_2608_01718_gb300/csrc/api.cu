@@ -258,6 +258,7 @@ void free_all(lacache* h) {
 lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* q_prefix, const int32_t* q_ids,
                           const lacache_result& out, cudaStream_t st) {
   const lacache_config& c = h->cfg;
+  if (c.stage1 == LACACHE_STAGE1_LSH && !h->lsh_bits) return LACACHE_ERR_INVALID_ARG;   // no index yet
   int splits = 0;
   int kernel = 0;
   cudaEvent_t* ev = nullptr;

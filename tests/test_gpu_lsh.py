@@ -102,3 +102,17 @@ def test_full_radius_equals_the_exact_scan_and_appends_are_signed():
         rows = wl.bf16_bits(q["emb"][miss])
     want, amb = oracle.signatures(rows, wl.bf16_bits(R))
     assert not np.any((_unpack(sig.cpu().numpy().view(np.uint32), 256) != want) & ~amb)
+
+
+def test_lookup_before_the_index_is_enabled_is_refused():
+    w = wl.WORKLOADS["mid-1m"].scaled(n=5_000, batch=8)
+    q = wl.batch(w, 0, device="cuda")
+    with new_cache(w, L.LACACHE_STAGE1_LSH) as cache:
+        fill(cache, w)
+        with pytest.raises(L.LacacheError) as e:
+            cache.lookup(q["emb"], q["prefix"], q["ids"])
+        assert e.value.status == L.LACACHE_ERR_INVALID_ARG
+        L.lacache_enable_lsh(cache.h, 256, 256, wl.hyperplanes(256, w.d, device="cuda"))
+        out = cache.lookup(q["emb"], q["prefix"], q["ids"])
+        torch.cuda.synchronize()
+        assert out["status"].shape == (w.batch,)
