@@ -2,12 +2,14 @@
 // sim(x, x') >= tau_c applied only to the entries whose signature is within `radius` bits of the query's.
 //
 // One CTA per contiguous split of the entries (two per SM); one entry per thread per tile of 512. A thread loads
-// its entry's signature (16-byte loads) and counts the differing bits against each of up to 8 query signatures
-// held in shared memory. Admitted (query, entry) pairs are queued in shared memory; when the queue is half full, and at the end
-// of the split, all warps take queue items two at a time and compute the exact fp32 score over the gathered key row
-// (each lane's 8-element chunks in order, then a butterfly sum). The warp of each query then folds the scores
-// that clear tau_c into that query's top-c list. The partial lists have the format of the other stage-1 kernels,
-// so stage 2 is shared.
+// its entry's signature (16-byte loads, one tile ahead, into registers) and counts the differing bits against each
+// of up to 32 query signatures held in shared memory. Admitted (query, entry) pairs are queued in shared memory.
+// When the queue passes three quarters of its capacity, and at the end of the split, all warps take queue items two
+// at a time and compute the exact fp32 score over the gathered key row (each lane's 8-element chunks in order,
+// then a butterfly sum). The warp of each query then folds the scores that clear tau_c into that query's top-c
+// list. A tile can admit more pairs than the queue has room for (up to 512 x 32, e.g. with radius = bits): a pair
+// that finds the queue full stays in its thread's pending mask and is queued again after the next flush. The
+// partial lists have the format of the other stage-1 kernels, so stage 2 is shared.
 #include "internal.cuh"
 
 namespace lc {
@@ -16,8 +18,9 @@ namespace {
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
 constexpr int kTile = kThreads;     // entries per tile, one per thread
-constexpr int kQC = 8;              // queries per pass over the entries
-constexpr int kCap = 8192;          // queue capacity; a tile adds at most kTile * kQC = 4096 items
+constexpr int kQC = 32;             // queries per pass over the entries (one bit each in a thread's masks)
+constexpr int kCap = 8192;          // queue capacity
+constexpr int kFlushAt = kCap - kCap / 4;   // a tile that leaves more items than this is followed by a flush
 constexpr unsigned kFull = 0xffffffffu;
 
 struct Item {
@@ -56,7 +59,7 @@ struct Shared {
 // Exact scores of the queued items, then each query's warp folds its items into the query's list.
 __device__ void flush(Shared& sh, const Stage1Args& a, int q0, int qn) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int total = sh.count;
+  const int total = min(sh.count, kCap);   // pairs that found the queue full were not stored
   const int v = a.d / 8;
   for (int base = warp * 2; base < total; base += kWarps * 2) {
     float acc0 = 0.f, acc1 = 0.f;
@@ -116,8 +119,27 @@ __device__ void flush(Shared& sh, const Stage1Args& a, int q0, int qn) {
   __syncthreads();
 }
 
+// Signature words of entry j into e (zeros past the split's end).
 template <int W>
-__global__ void __launch_bounds__(kThreads) lsh_scan_kernel(Stage1Args a, LshArgs l, int splits) {
+__device__ __forceinline__ void load_sig(const uint32_t* sig, int64_t j, int64_t j_end, uint32_t (&e)[W]) {
+  if (j < j_end) {
+    const uint4* src = reinterpret_cast<const uint4*>(sig + j * W);
+#pragma unroll
+    for (int w = 0; w < W / 4; ++w) {
+      const uint4 u = __ldg(src + w);
+      e[4 * w] = u.x;
+      e[4 * w + 1] = u.y;
+      e[4 * w + 2] = u.z;
+      e[4 * w + 3] = u.w;
+    }
+  } else {
+#pragma unroll
+    for (int w = 0; w < W; ++w) e[w] = 0u;
+  }
+}
+
+template <int W>
+__global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, LshArgs l, int splits) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   Shared& sh = *reinterpret_cast<Shared*>(smem_raw);
   asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -134,31 +156,56 @@ __global__ void __launch_bounds__(kThreads) lsh_scan_kernel(Stage1Args a, LshArg
     if (threadIdx.x < kQC) sh.best[threadIdx.x] = score_order(-INFINITY);
     if (threadIdx.x == 0) sh.count = 0;
     __syncthreads();
+    // The next tile's signatures are loaded before the current tile is counted, so the load latency is hidden
+    // behind the popcounts.
+    uint32_t nxt[W];
+    load_sig<W>(l.sig, j_begin + threadIdx.x, j_end, nxt);
+    const unsigned qmask = qn >= 32 ? kFull : (1u << qn) - 1u;
     for (int64_t t0 = j_begin; t0 < j_end; t0 += kTile) {
       const int64_t j = t0 + threadIdx.x;
-      if (j < j_end) {
-        uint32_t e[W];
-        const uint4* src = reinterpret_cast<const uint4*>(l.sig + j * W);
+      uint32_t e[W];
+#pragma unroll
+      for (int w = 0; w < W; ++w) e[w] = nxt[w];
+      load_sig<W>(l.sig, j + kTile, j_end, nxt);
+      // every query's distance first, as a mask of the admitted queries (the queue stores below could alias the
+      // query signatures for the compiler)
+      unsigned pend = 0;
+#pragma unroll 8
+      for (int qq = 0; qq < kQC; ++qq) {
+        const uint4* qs = reinterpret_cast<const uint4*>(sh.qsig[qq]);
+        int h = 0;
 #pragma unroll
         for (int w = 0; w < W / 4; ++w) {
-          const uint4 u = __ldg(src + w);
-          e[4 * w] = u.x;
-          e[4 * w + 1] = u.y;
-          e[4 * w + 2] = u.z;
-          e[4 * w + 3] = u.w;
+          const uint4 u = qs[w];
+          h += __popc(e[4 * w] ^ u.x) + __popc(e[4 * w + 1] ^ u.y) + __popc(e[4 * w + 2] ^ u.z) +
+               __popc(e[4 * w + 3] ^ u.w);
         }
-        for (int qq = 0; qq < qn; ++qq) {
-          int hd = 0;
-#pragma unroll
-          for (int w = 0; w < W; ++w) hd += __popc(e[w] ^ sh.qsig[qq][w]);
-          if (hd <= l.radius) {
-            const int slot = atomicAdd(&sh.count, 1);
+        pend |= (h <= l.radius ? 1u : 0u) << qq;
+      }
+      pend = j < j_end ? pend & qmask : 0u;
+      // Queue the admitted pairs; flush while the queue is past kFlushAt or a pair found it full. Every round of
+      // this loop either queues all pending pairs or fills the queue, so it ends.
+      int top = -1;   // the highest queue slot this thread took in this round
+      for (;;) {
+        unsigned full = 0;
+        while (pend) {
+          const int qq = __ffs(pend) - 1;
+          pend &= pend - 1;
+          const int slot = atomicAdd(&sh.count, 1);
+          if (slot < kCap) {
             sh.items[slot] = Item{(int32_t)j, qq};
+            top = slot;
+          } else {
+            full |= 1u << qq;
           }
         }
+        pend = full;
+        // the barrier's OR gives every thread the same answer (a read of the count after a plain barrier
+        // could already see the next tile's items in some threads)
+        if (!__syncthreads_or(pend != 0 || top >= kFlushAt)) break;
+        flush(sh, a, q0, qn);
+        top = -1;
       }
-      __syncthreads();
-      if (sh.count > kCap - kTile * kQC) flush(sh, a, q0, qn);
     }
     flush(sh, a, q0, qn);
     for (int i = threadIdx.x; i < qn * C; i += kThreads) {
@@ -171,13 +218,24 @@ __global__ void __launch_bounds__(kThreads) lsh_scan_kernel(Stage1Args a, LshArg
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
+// The scan is a programmatic dependent launch of the query-signature GEMM: its CTAs may be scheduled while the
+// signatures are computed and wait in griddepcontrol.wait, which hides the launch gap.
 template <int W>
 cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStream_t st) {
   const size_t smem = sizeof(Shared);
   cudaError_t e = cudaFuncSetAttribute(lsh_scan_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  lsh_scan_kernel<W><<<splits, kThreads, smem, st>>>(a, l, splits);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(splits);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, lsh_scan_kernel<W>, a, l, splits);
 }
 
 }  // namespace
