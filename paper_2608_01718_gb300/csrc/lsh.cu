@@ -119,6 +119,42 @@ __device__ void flush(Shared& sh, const Stage1Args& a, int q0, int qn) {
   __syncthreads();
 }
 
+// Carry-save adder on 32 bit positions at once: a + b + c = lo + 2 hi in every position (two LOP3 operations).
+__device__ __forceinline__ void csa(uint32_t& hi, uint32_t& lo, uint32_t a, uint32_t b, uint32_t c) {
+  const uint32_t u = a ^ b;
+  lo = u ^ c;
+  hi = (a & b) | (u & c);
+}
+
+// Number of set bits in x[0..W). Population count runs at 16 per clock per SM, the logic operations at 64, so
+// carry-save adders first fold words into sum and carry words, each group of 8 words into 5 popcounts (3 adders):
+//   x0 + x1 + x2 = sa + 2 ca,  x3 + x4 + x5 = sb + 2 cb,  sa + sb + x6 = sc + 2 cc,
+//   |x0..x7| = |sc| + |x7| + 2 (|ca| + |cb| + |cc|);
+// a group of 4 words into 3 (one adder). The count is exact.
+template <int W>
+__device__ __forceinline__ int hamming(const uint32_t (&x)[W]) {
+  int h = 0;
+  if constexpr (W % 8 == 0) {
+#pragma unroll
+    for (int g = 0; g < W; g += 8) {
+      uint32_t ca, sa, cb, sb, cc, sc;
+      csa(ca, sa, x[g], x[g + 1], x[g + 2]);
+      csa(cb, sb, x[g + 3], x[g + 4], x[g + 5]);
+      csa(cc, sc, sa, sb, x[g + 6]);
+      h += __popc(sc) + __popc(x[g + 7]) + 2 * (__popc(ca) + __popc(cb) + __popc(cc));
+    }
+  } else {
+    static_assert(W % 4 == 0, "signature words come in groups of 4");
+#pragma unroll
+    for (int g = 0; g < W; g += 4) {
+      uint32_t c, s;
+      csa(c, s, x[g], x[g + 1], x[g + 2]);
+      h += __popc(s) + __popc(x[g + 3]) + 2 * __popc(c);
+    }
+  }
+  return h;
+}
+
 // Signature words of entry j into e (zeros past the split's end).
 template <int W>
 __device__ __forceinline__ void load_sig(const uint32_t* sig, int64_t j, int64_t j_end, uint32_t (&e)[W]) {
@@ -173,14 +209,16 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
 #pragma unroll 8
       for (int qq = 0; qq < kQC; ++qq) {
         const uint4* qs = reinterpret_cast<const uint4*>(sh.qsig[qq]);
-        int h = 0;
+        uint32_t x[W];
 #pragma unroll
         for (int w = 0; w < W / 4; ++w) {
           const uint4 u = qs[w];
-          h += __popc(e[4 * w] ^ u.x) + __popc(e[4 * w + 1] ^ u.y) + __popc(e[4 * w + 2] ^ u.z) +
-               __popc(e[4 * w + 3] ^ u.w);
+          x[4 * w] = e[4 * w] ^ u.x;
+          x[4 * w + 1] = e[4 * w + 1] ^ u.y;
+          x[4 * w + 2] = e[4 * w + 2] ^ u.z;
+          x[4 * w + 3] = e[4 * w + 3] ^ u.w;
         }
-        pend |= (h <= l.radius ? 1u : 0u) << qq;
+        pend |= (hamming<W>(x) <= l.radius ? 1u : 0u) << qq;
       }
       pend = j < j_end ? pend & qmask : 0u;
       // Queue the admitted pairs; flush while the queue is past kFlushAt or a pair found it full. Every round of
