@@ -159,6 +159,19 @@ lacache_status lacache_lookup(lacache_t* h, int32_t B, const void* q_emb_dev, co
 lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_host, const void* q_prefix_host,
                                    const int32_t* q_ids_host, const lacache_result* out_host, void* cuda_stream);
 
+/* lacache_lookup_host without the synchronization, for pipelined serving: a caller may keep several lookups in
+ * flight on one stream, each with its own output arrays. Every input array and every non-NULL field of *out_host
+ * must lie in pinned host memory that the handle's device can map (cudaHostAlloc or cudaMallocHost, or
+ * cudaHostRegister with mapping; with unified addressing all pinned memory is mapped), and each output field must
+ * be aligned to its element size; otherwise the call returns LACACHE_ERR_INVALID_ARG and runs nothing. One kernel
+ * gathers the inputs into the handle's device staging, the lookup's kernels follow, and they write the results
+ * straight into the output arrays. The call returns once they are enqueued on cuda_stream. The output arrays hold
+ * the results, and the input arrays may be reused, only after the stream has passed the call (an event recorded
+ * after it, or cudaStreamSynchronize). Calls on one handle must all use one stream: the staging is the handle's. */
+lacache_status lacache_lookup_host_async(lacache_t* h, int32_t B, const void* q_emb_host, const void* q_prefix_host,
+                                         const int32_t* q_ids_host, const lacache_result* out_host,
+                                         void* cuda_stream);
+
 /* The cache update of the serve loop: append, in query order, every query of a looked-up batch whose status is
  * not LACACHE_HIT (a key miss or a lookahead rejection is decoded from scratch and added; Algorithm 1). The
  * inputs are those of the lookup (device pointers) and its status_dev output. The rows are gathered on the

@@ -171,6 +171,17 @@ const void* mapped_device_pointer(const void* p) {
   return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
 }
 
+// Output field p of an asynchronous host lookup as a device-writable address in *d: NULL stays NULL; anything else
+// must be mapped pinned memory aligned to T.
+template <typename T>
+bool map_output(T* p, T** d) {
+  *d = nullptr;
+  if (!p) return true;
+  if (reinterpret_cast<uintptr_t>(p) % alignof(T)) return false;
+  *d = static_cast<T*>(const_cast<void*>(mapped_device_pointer(p)));
+  return *d != nullptr;
+}
+
 size_t stage_in_bytes(const lacache_config& c, int pd) {
   return (size_t)c.max_batch * ((size_t)2 * c.d + (size_t)2 * pd + (size_t)4 * c.k);
 }
@@ -564,6 +575,50 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
   for (const Copy& cp : copies)
     if (cp.dst && cp.src) memcpy(cp.dst, cp.src, cp.bytes);
   return LACACHE_OK;
+}
+
+lacache_status lacache_lookup_host_async(lacache_t* h, int32_t B, const void* q_emb_host, const void* q_prefix_host,
+                                         const int32_t* q_ids_host, const lacache_result* out_host,
+                                         void* cuda_stream) {
+  lc::NvtxRange nvtx("lacache_lookup_host_async");
+  if (!h || B < 1 || B > h->cfg.max_batch) return LACACHE_ERR_INVALID_ARG;
+  if (!q_emb_host || !q_prefix_host || !q_ids_host || !result_ok(out_host)) return LACACHE_ERR_INVALID_ARG;
+  DeviceGuard guard(h->cfg.device);
+  if (!guard.ok()) return LACACHE_ERR_CUDA;
+  const lacache_config& c = h->cfg;
+  unsigned char* q_emb = h->stage_in;
+  unsigned char* q_pre = q_emb + (size_t)c.max_batch * c.d * 2;
+  int32_t* q_ids = reinterpret_cast<int32_t*>(q_pre + (size_t)c.max_batch * h->pd * 2);
+  // every address is checked before anything is enqueued
+  const void* src[3] = {q_emb_host, q_prefix_host, q_ids_host};
+  unsigned char* dst[3] = {q_emb, q_pre, reinterpret_cast<unsigned char*>(q_ids)};
+  const size_t nbytes[3] = {(size_t)B * c.d * 2, (size_t)B * h->pd * 2, (size_t)B * c.k * 4};
+  GatherArgs g{};
+  size_t gathered = 0;
+  for (int i = 0; i < 3; ++i) {
+    const void* dev_src = mapped_device_pointer(src[i]);
+    if (!dev_src) return LACACHE_ERR_INVALID_ARG;
+    g.seg[i] = GatherSeg{static_cast<const unsigned char*>(dev_src), dst[i], nbytes[i]};
+    gathered += nbytes[i];
+  }
+  const lacache_result& o = *out_host;
+  lacache_result dev{};
+  const bool mapped = map_output(o.entry_id, &dev.entry_id) && map_output(o.status, &dev.status) &&
+                      map_output(o.key_score, &dev.key_score) && map_output(o.prefix_score, &dev.prefix_score) &&
+                      map_output(o.token_matches, &dev.token_matches) && map_output(o.n_cand, &dev.n_cand) &&
+                      map_output(o.cand_id, &dev.cand_id) && map_output(o.cand_score, &dev.cand_score) &&
+                      map_output(o.cand_prefix_score, &dev.cand_prefix_score) &&
+                      map_output(o.cand_matches, &dev.cand_matches) &&
+                      map_output(o.prefix_scores, &dev.prefix_scores) && map_output(o.cand_pass, &dev.cand_pass) &&
+                      map_output(o.cand_prefix_scores, &dev.cand_prefix_scores);
+  if (!mapped) return LACACHE_ERR_INVALID_ARG;
+  if (c.stage1 == LACACHE_STAGE1_LSH && !h->lsh_bits) return LACACHE_ERR_INVALID_ARG;
+  cudaStream_t st = (cudaStream_t)cuda_stream;
+  const size_t vec = (gathered + 15) / 16;
+  const int grid = (int)std::min<size_t>((vec + 255) / 256, (size_t)2 * h->num_sms);
+  gather_host_kernel<<<grid, 256, 0, st>>>(g);
+  if (cudaGetLastError() != cudaSuccess) return LACACHE_ERR_CUDA;
+  return run_lookup(h, B, q_emb, q_pre, q_ids, dev, st);
 }
 
 lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,

@@ -22,7 +22,8 @@ LACACHE_MISS_KEY, LACACHE_HIT, LACACHE_REJECT = 0, 1, 2
 LACACHE_MAX_MODELS = 8
 LACACHE_MAX_SHARDS = 16
 
-EXPORTS = ["lacache_create", "lacache_create_ensemble", "lacache_destroy", "lacache_insert", "lacache_lookup", "lacache_lookup_host",
+EXPORTS = ["lacache_create", "lacache_create_ensemble", "lacache_destroy", "lacache_insert", "lacache_lookup",
+           "lacache_lookup_host", "lacache_lookup_host_async",
            "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
            "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_enable_lsh", "lacache_read_signatures", "lacache_calibrate", "lacache_calibrate_workspace_bytes", "lacache_verify_draft",
            "lacache_lookup_noalloc", "lacache_merge_shards", "lacache_get_stats", "lacache_save", "lacache_load",
@@ -89,6 +90,7 @@ def load() -> ctypes.CDLL:
         "lacache_insert": ([vp, i64, vp, vp, vp, i32, p64, vp], i32),
         "lacache_lookup": ([vp, i32, vp, vp, vp, ctypes.POINTER(lacache_result), vp], i32),
         "lacache_lookup_host": ([vp, i32, vp, vp, vp, ctypes.POINTER(lacache_result), vp], i32),
+        "lacache_lookup_host_async": ([vp, i32, vp, vp, vp, ctypes.POINTER(lacache_result), vp], i32),
         "lacache_append_misses": ([vp, i32, vp, vp, vp, vp, p64, p64, vp], i32),
         "lacache_read_rows": ([vp, i64, i64, vp, vp, vp, vp], i32),
         "lacache_size": ([vp, p64], i32),
@@ -240,6 +242,14 @@ def lacache_lookup_host(h: int, q_emb, q_prefix, q_ids, out: dict, cuda_stream=N
     res = _result_struct(out)
     _check("lacache_lookup_host", load().lacache_lookup_host(h, int(q_emb.shape[0]), _ptr(q_emb), _ptr(q_prefix),
                                                              _ptr(q_ids), ctypes.byref(res), _stream(cuda_stream)))
+
+
+def lacache_lookup_host_async(h: int, q_emb, q_prefix, q_ids, out: dict, cuda_stream=None) -> None:
+    """Lookup of queries in pinned host tensors into pinned host results, enqueued on the stream without waiting:
+    the results are there once the stream has passed the call."""
+    res = _result_struct(out)
+    _check("lacache_lookup_host_async", load().lacache_lookup_host_async(
+        h, int(q_emb.shape[0]), _ptr(q_emb), _ptr(q_prefix), _ptr(q_ids), ctypes.byref(res), _stream(cuda_stream)))
 
 
 def lacache_append_misses(h: int, q_emb, q_prefix, q_ids, status, cuda_stream=None) -> tuple[int, int]:

@@ -226,6 +226,54 @@ def test_host_buffer_lookup_any_host_memory(kinds):
 
 
 @pytest.mark.parametrize("stage1", PATHS)
+def test_async_host_lookups_in_flight_match_device_lookups(stage1):
+    # three lookups enqueued back to back on one stream, each into its own mapped pinned outputs, read only after
+    # the stream has passed them; the inputs sit in mapped pinned memory, two of them off 16-byte boundaries
+    w = wl.WORKLOADS["serve-2m"].scaled(n=12_050, batch=300 if stage1 == L.LACACHE_STAGE1_TENSOR else 64,
+                                        clusters=120)
+    with new_cache(w, stage1) as cache:
+        fill(cache, w)
+        qs = [wl.batch(w, i, device="cuda") for i in range(3)]
+        want = [gpu_lookup(cache, q) for q in qs]
+        hq = [{k: _host_copy(q[k], "pinned", off) for k, off in (("emb", 0), ("prefix", 2), ("ids", 4))}
+              for q in qs]
+        outs = [L.alloc_result(w.batch, w.top_c, "cpu", pinned=True) for _ in qs]
+        stream = torch.cuda.current_stream()
+        for q, o in zip(hq, outs):
+            L.lacache_lookup_host_async(cache.h, q["emb"], q["prefix"], q["ids"], o, stream)
+        stream.synchronize()
+        cache.sync()
+        for o, g in zip(outs, want):
+            for k, v in o.items():
+                assert np.array_equal(v.numpy(), g[k], equal_nan=True), k
+
+
+def test_async_host_lookup_refuses_unmapped_or_misaligned_buffers():
+    w = wl.WORKLOADS["tiny-4k"]
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+        fill(cache, w)
+        q = wl.batch(w, 0, device="cuda")
+        pinned = {k: q[k].cpu().pin_memory() for k in ("emb", "prefix", "ids")}
+        pageable = {k: q[k].cpu() for k in ("emb", "prefix", "ids")}
+        out = L.alloc_result(w.batch, w.top_c, "cpu", pinned=True)
+        for v in out.values():
+            v.fill_(7)
+        cases = []
+        for key in ("emb", "prefix", "ids"):    # one pageable input
+            cases.append(({**pinned, key: pageable[key]}, out))
+        cases.append((pinned, {**out, "cand_score": torch.empty((w.batch, w.top_c))}))   # a pageable output
+        raw = torch.empty(w.batch * 4 + 4, dtype=torch.uint8).pin_memory()
+        cases.append((pinned, {**out, "key_score": raw.data_ptr() + 2}))                # a misaligned output
+        for qi, o in cases:
+            with pytest.raises(L.LacacheError) as e:
+                L.lacache_lookup_host_async(cache.h, qi["emb"], qi["prefix"], qi["ids"], o)
+            assert e.value.status == L.LACACHE_ERR_INVALID_ARG
+        torch.cuda.synchronize()
+        for v in out.values():      # nothing ran
+            assert torch.all(v == 7)
+
+
+@pytest.mark.parametrize("stage1", PATHS)
 def test_serve_loop_appends_misses_like_the_oracle(stage1):
     w = wl.WORKLOADS["serve-2m"].scaled(n=20_000, batch=64, clusters=200)
     steps = 12
