@@ -6,7 +6,9 @@
  *   queries 4-5  an entry's key with a fresh prefix and fresh ids -> REJECT (the lookahead check fails)
  *   queries 6-7  fresh random keys                                -> MISS_KEY
  * Random unit vectors in d = 64 have |cos| < 0.9 with overwhelming probability, so every copied key's only
- * candidate is its own entry. Exits 0 and prints "ok" when every decision is as listed. */
+ * candidate is its own entry. The same batch then goes twice through lacache_lookup_host_async, from and into
+ * mapped pinned buffers (cudaHostAlloc), both calls in flight on one stream before it is synchronized; both must
+ * give the same decisions. Exits 0 and prints "ok" when every decision is as listed. */
 #include <math.h>
 #include <stdint.h>
 #include <stdio.h>
@@ -134,6 +136,44 @@ int main(void) {
       bad = 1;
     }
   }
+
+  /* the pipelined form: inputs and outputs in mapped pinned memory, two lookups in flight */
+  struct Pinned {
+    uint16_t emb[B * D], pre[B * D];
+    int32_t ids[B * K];
+    int32_t entry_id[2][B], token_matches[2][B], n_cand[2][B];
+    float key_score[2][B], prefix_score[2][B];
+    uint8_t status[2][B];
+  }* pin = NULL;
+  if (cudaHostAlloc((void**)&pin, sizeof *pin, cudaHostAllocMapped) != cudaSuccess) return 1;
+  memcpy(pin->emb, q_emb, sizeof q_emb);
+  memcpy(pin->pre, q_pre, sizeof q_pre);
+  memcpy(pin->ids, q_ids, sizeof q_ids);
+  cudaStream_t stream;
+  if (cudaStreamCreate(&stream) != cudaSuccess) return 1;
+  for (int r = 0; r < 2; ++r) {
+    lacache_result o;
+    memset(&o, 0, sizeof o);
+    o.entry_id = pin->entry_id[r];
+    o.status = pin->status[r];
+    o.key_score = pin->key_score[r];
+    o.prefix_score = pin->prefix_score[r];
+    o.token_matches = pin->token_matches[r];
+    o.n_cand = pin->n_cand[r];
+    CHECK(lacache_lookup_host_async(h, B, pin->emb, pin->pre, pin->ids, &o, stream));
+  }
+  if (cudaStreamSynchronize(stream) != cudaSuccess) return 1;
+  CHECK(lacache_sync(h));
+  for (int r = 0; r < 2; ++r)
+    for (int b = 0; b < B; ++b)
+      if (pin->status[r][b] != status[b] || pin->entry_id[r][b] != entry_id[b] || pin->n_cand[r][b] != n_cand[b]) {
+        fprintf(stderr, "async call %d, query %d: status %d entry %d\n", r, b, pin->status[r][b],
+                pin->entry_id[r][b]);
+        bad = 1;
+      }
+  cudaStreamDestroy(stream);
+  cudaFreeHost(pin);
+
   CHECK(lacache_destroy(h));
   cudaFree(key_dev);
   cudaFree(pre_dev);
