@@ -182,6 +182,33 @@ bool map_output(T* p, T** d) {
   return *d != nullptr;
 }
 
+// The three inputs of a host-buffer lookup (key embeddings, prefix embeddings, token ids): where they are, where
+// they go in the handle's device staging, and their sizes.
+struct HostInputs {
+  const void* src[3];
+  unsigned char* dst[3];
+  size_t bytes[3];
+};
+HostInputs host_inputs(const lacache* h, int B, const void* emb, const void* pre, const int32_t* ids) {
+  const lacache_config& c = h->cfg;
+  HostInputs in{{emb, pre, ids}, {}, {(size_t)B * c.d * 2, (size_t)B * h->pd * 2, (size_t)B * c.k * 4}};
+  in.dst[0] = h->stage_in;
+  in.dst[1] = in.dst[0] + (size_t)c.max_batch * c.d * 2;
+  in.dst[2] = in.dst[1] + (size_t)c.max_batch * h->pd * 2;
+  return in;
+}
+
+// One gather kernel for the segments of g, `bytes` in all.
+cudaError_t launch_gather(const lacache* h, const GatherArgs& g, size_t bytes, cudaStream_t st) {
+  const size_t vec = (bytes + 15) / 16;
+  const int grid = (int)std::min<size_t>((vec + 255) / 256, (size_t)2 * h->num_sms);
+  gather_host_kernel<<<grid, 256, 0, st>>>(g);
+  return cudaGetLastError();
+}
+
+// A handle set to the SimHash stage can look up only once its index is enabled.
+bool lookup_ready(const lacache* h) { return h->cfg.stage1 != LACACHE_STAGE1_LSH || h->lsh_bits; }
+
 size_t stage_in_bytes(const lacache_config& c, int pd) {
   return (size_t)c.max_batch * ((size_t)2 * c.d + (size_t)2 * pd + (size_t)4 * c.k);
 }
@@ -269,7 +296,7 @@ void free_all(lacache* h) {
 lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* q_prefix, const int32_t* q_ids,
                           const lacache_result& out, cudaStream_t st) {
   const lacache_config& c = h->cfg;
-  if (c.stage1 == LACACHE_STAGE1_LSH && !h->lsh_bits) return LACACHE_ERR_INVALID_ARG;   // no index yet
+  if (!lookup_ready(h)) return LACACHE_ERR_INVALID_ARG;
   int splits = 0;
   int kernel = 0;
   cudaEvent_t* ev = nullptr;
@@ -520,38 +547,29 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
   if (!q_emb_host || !q_prefix_host || !q_ids_host || !result_ok(out_host)) return LACACHE_ERR_INVALID_ARG;
   DeviceGuard guard(h->cfg.device);
   if (!guard.ok()) return LACACHE_ERR_CUDA;
+  if (!lookup_ready(h)) return LACACHE_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
   const lacache_config& c = h->cfg;
-  unsigned char* q_emb = h->stage_in;
-  unsigned char* q_pre = q_emb + (size_t)c.max_batch * c.d * 2;
-  int32_t* q_ids = reinterpret_cast<int32_t*>(q_pre + (size_t)c.max_batch * h->pd * 2);
+  const HostInputs in = host_inputs(h, B, q_emb_host, q_prefix_host, q_ids_host);
   // Inputs: arrays in mapped pinned memory are gathered by one kernel; any other array is copied by DMA.
-  const void* src[3] = {q_emb_host, q_prefix_host, q_ids_host};
-  unsigned char* dst[3] = {q_emb, q_pre, reinterpret_cast<unsigned char*>(q_ids)};
-  const size_t nbytes[3] = {(size_t)B * c.d * 2, (size_t)B * h->pd * 2, (size_t)B * c.k * 4};
   GatherArgs g{};
   size_t gathered = 0;
   for (int i = 0; i < 3; ++i) {
-    const void* dev_src = mapped_device_pointer(src[i]);
+    const void* dev_src = mapped_device_pointer(in.src[i]);
     if (dev_src) {
-      g.seg[i] = GatherSeg{static_cast<const unsigned char*>(dev_src), dst[i], nbytes[i]};
-      gathered += nbytes[i];
-    } else if (cudaMemcpyAsync(dst[i], src[i], nbytes[i], cudaMemcpyHostToDevice, st) != cudaSuccess) {
+      g.seg[i] = GatherSeg{static_cast<const unsigned char*>(dev_src), in.dst[i], in.bytes[i]};
+      gathered += in.bytes[i];
+    } else if (cudaMemcpyAsync(in.dst[i], in.src[i], in.bytes[i], cudaMemcpyHostToDevice, st) != cudaSuccess) {
       return LACACHE_ERR_CUDA;
     }
   }
-  if (gathered) {
-    const size_t vec = (gathered + 15) / 16;
-    const int grid = (int)std::min<size_t>((vec + 255) / 256, (size_t)2 * h->num_sms);
-    gather_host_kernel<<<grid, 256, 0, st>>>(g);
-    if (cudaGetLastError() != cudaSuccess) return LACACHE_ERR_CUDA;
-  }
+  if (gathered && launch_gather(h, g, gathered, st) != cudaSuccess) return LACACHE_ERR_CUDA;
   size_t bytes = 0;
   // Results: written by the kernels straight into the mapped pinned staging when the device can map it.
   unsigned char* out_stage = h->stage_host_dev ? h->stage_host_dev : h->stage_out;
   lacache_result dev = staged_result(out_stage, B, c.top_c, h->ens.m, *out_host, &bytes);
   lacache_result host = staged_result(h->stage_host, B, c.top_c, h->ens.m, *out_host, &bytes);
-  lacache_status s = run_lookup(h, B, q_emb, q_pre, q_ids, dev, st);
+  lacache_status s = run_lookup(h, B, in.dst[0], in.dst[1], reinterpret_cast<const int32_t*>(in.dst[2]), dev, st);
   if (s != LACACHE_OK) return s;
   if (!h->stage_host_dev &&
       cudaMemcpyAsync(h->stage_host, h->stage_out, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess)
@@ -585,21 +603,16 @@ lacache_status lacache_lookup_host_async(lacache_t* h, int32_t B, const void* q_
   if (!q_emb_host || !q_prefix_host || !q_ids_host || !result_ok(out_host)) return LACACHE_ERR_INVALID_ARG;
   DeviceGuard guard(h->cfg.device);
   if (!guard.ok()) return LACACHE_ERR_CUDA;
-  const lacache_config& c = h->cfg;
-  unsigned char* q_emb = h->stage_in;
-  unsigned char* q_pre = q_emb + (size_t)c.max_batch * c.d * 2;
-  int32_t* q_ids = reinterpret_cast<int32_t*>(q_pre + (size_t)c.max_batch * h->pd * 2);
+  if (!lookup_ready(h)) return LACACHE_ERR_INVALID_ARG;
   // every address is checked before anything is enqueued
-  const void* src[3] = {q_emb_host, q_prefix_host, q_ids_host};
-  unsigned char* dst[3] = {q_emb, q_pre, reinterpret_cast<unsigned char*>(q_ids)};
-  const size_t nbytes[3] = {(size_t)B * c.d * 2, (size_t)B * h->pd * 2, (size_t)B * c.k * 4};
+  const HostInputs in = host_inputs(h, B, q_emb_host, q_prefix_host, q_ids_host);
   GatherArgs g{};
   size_t gathered = 0;
   for (int i = 0; i < 3; ++i) {
-    const void* dev_src = mapped_device_pointer(src[i]);
+    const void* dev_src = mapped_device_pointer(in.src[i]);
     if (!dev_src) return LACACHE_ERR_INVALID_ARG;
-    g.seg[i] = GatherSeg{static_cast<const unsigned char*>(dev_src), dst[i], nbytes[i]};
-    gathered += nbytes[i];
+    g.seg[i] = GatherSeg{static_cast<const unsigned char*>(dev_src), in.dst[i], in.bytes[i]};
+    gathered += in.bytes[i];
   }
   const lacache_result& o = *out_host;
   lacache_result dev{};
@@ -612,13 +625,9 @@ lacache_status lacache_lookup_host_async(lacache_t* h, int32_t B, const void* q_
                       map_output(o.prefix_scores, &dev.prefix_scores) && map_output(o.cand_pass, &dev.cand_pass) &&
                       map_output(o.cand_prefix_scores, &dev.cand_prefix_scores);
   if (!mapped) return LACACHE_ERR_INVALID_ARG;
-  if (c.stage1 == LACACHE_STAGE1_LSH && !h->lsh_bits) return LACACHE_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
-  const size_t vec = (gathered + 15) / 16;
-  const int grid = (int)std::min<size_t>((vec + 255) / 256, (size_t)2 * h->num_sms);
-  gather_host_kernel<<<grid, 256, 0, st>>>(g);
-  if (cudaGetLastError() != cudaSuccess) return LACACHE_ERR_CUDA;
-  return run_lookup(h, B, q_emb, q_pre, q_ids, dev, st);
+  if (launch_gather(h, g, gathered, st) != cudaSuccess) return LACACHE_ERR_CUDA;
+  return run_lookup(h, B, in.dst[0], in.dst[1], reinterpret_cast<const int32_t*>(in.dst[2]), dev, st);
 }
 
 lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
