@@ -46,6 +46,18 @@ def test_each_model_uses_its_own_threshold():
         assert oracle.lookup(st, q, p).status[0] == want, taus
 
 
+def test_thresholds_belong_to_their_models():
+    # model 0 scores 0.75 and model 1 scores 0.5, so swapping the two thresholds changes the outcome
+    a = np.array([0.75, 0.5, 0.25, 0.0])
+    b = np.array([0.5, 0.5, 0.5, 0.5])
+    st = store_of([E[0]], [np.concatenate([E[0], E[0]])], [[0]])
+    q = queries_of(E[0], np.concatenate([a, b]), [0])
+    for taus, want in [((0.7, 0.4), HIT), ((0.4, 0.7), REJECT), ((0.75, 0.5), HIT), ((0.5, 0.75), REJECT)]:
+        r = oracle.lookup(st, q, Params(0.5, 0.0, 1, prefix_dims=(4, 4), tau_a_models=taus))
+        assert r.status[0] == want, taus
+        assert list(r.prefix_scores[0]) == [0.75, 0.5] and list(r.cand_prefix_scores[0, 0]) == [0.75, 0.5]
+
+
 def test_single_model_ensemble_is_the_plain_check():
     rng = np.random.default_rng(5)
     n, d, B = 200, 16, 30

@@ -69,6 +69,15 @@ def test_round_to_bf16_ties_to_even():
     assert [int(v) for v in oracle.round_to_bf16(x)] == want
 
 
+def test_round_to_bf16_keeps_nans_nan():
+    # a NaN whose payload lies only in the dropped half would truncate to an infinity; it must stay a NaN of the
+    # same sign (quieted: the top fraction bit set)
+    x = np.array([0x7F800001, 0xFF800001, 0x7FC00000, 0x7FA00000], np.uint32).view(np.float32)
+    got = [int(v) for v in oracle.round_to_bf16(x)]
+    assert got == [0x7FC0, 0xFFC0, 0x7FC0, 0x7FE0]
+    assert all(np.isnan(oracle.widen(np.array(got, np.uint16))))
+
+
 def test_round_to_bf16_agrees_with_library():
     torch = pytest.importorskip("torch")
     rng = np.random.default_rng(3)
@@ -132,6 +141,16 @@ def test_collision_with_distinct_prefix_is_rejected():
     assert r.status[0] == REJECT and r.entry_id[0] == -1
     assert r.n_cand[0] == 1 and r.prefix_score[0] == 0.0 and r.token_matches[0] == 0
     assert r.key_score[0] == 1.0
+
+
+def test_reject_shows_the_first_candidate():
+    # two candidates, neither passing: the shown lookahead score and token matches are those of the first (the
+    # higher key score), not of the last
+    st = store_of([E[0], [0.875, 0, 0, 0]], [[0.25, 0, 0, 0], [0.5, 0, 0, 0]], [[1, 2], [1, 0]])
+    r = oracle.lookup(st, queries_of(E[0], E[0], [1, 2]), Params(0.5, 0.75, 4, check_mode=CHECK_BOTH))
+    assert r.status[0] == REJECT and list(r.cand_id[0, :2]) == [0, 1]
+    assert r.prefix_score[0] == 0.25 and r.token_matches[0] == 2
+    assert list(r.cand_prefix_score[0, :2]) == [0.25, 0.5] and list(r.cand_matches[0, :2]) == [2, 1]
 
 
 def test_prefix_check_reads_prefix_rows_not_key_rows():
@@ -225,6 +244,11 @@ def test_margin_terms():
     st = store_of(keys, [E[2], E[3], E[3]], [[0]] * 3)
     r = oracle.lookup(st, queries_of(q, E[3], [0]), Params(0.5, 0.5, 2))
     assert r.status[0] == HIT and r.entry_id[0] == 1 and r.margin[0] == 0.875 - 0.859375
+    # the served entry's key score sits 2^-6 above tau_c, its prefix score 0.5 above tau_a: falling out of A_q is
+    # the closest change.
+    st = store_of([E[0]], [E[1]], [[0]])
+    r = oracle.lookup(st, queries_of(q, E[1], [0]), Params(0.984375, 0.5, 1))
+    assert r.status[0] == HIT and r.margin[0] == 1.0 - 0.984375
 
 
 # --- brute force in exact arithmetic on tiny inputs ---------------------------------------------------------------

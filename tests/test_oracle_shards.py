@@ -106,6 +106,26 @@ def test_equal_scores_across_shards_order_by_global_id(dup_at):
     assert merged.entry_id[b] == min(j, dup_at)
 
 
+def test_merged_key_score_is_the_best_over_shards_when_a_shard_hit_falls_past_the_cut():
+    # query e0, top_c 2, entries scoring 1, 0.9375 (shard A, ids 0-1) and 0.984375, 0.96875 (shard B, ids 2-3).
+    # Only entry 1 passes the lookahead check. Shard A serves it (a HIT reporting key score 0.9375), but globally
+    # it is third, past the cut: the whole-store result is a REJECT whose key score is the best one, 1.
+    E4 = np.eye(4)
+    keys = [[1.0, 0, 0, 0], [0.9375, 0, 0, 0], [0.984375, 0, 0, 0], [0.96875, 0, 0, 0]]
+    st = oracle.Store.of(oracle.round_to_bf16(np.array(keys, np.float32)),
+                         oracle.round_to_bf16(np.array([E4[2], E4[1], E4[2], E4[2]], np.float32)),
+                         np.zeros((4, 1), np.int32))
+    oq = {"emb": oracle.round_to_bf16(E4[:1].astype(np.float32)),
+          "prefix": oracle.round_to_bf16(E4[1:2].astype(np.float32)), "ids": np.zeros((1, 1), np.int32)}
+    p = oracle.Params(0.5, 0.5, 2)
+    whole = oracle.lookup(st, oq, p)
+    parts = [oracle.lookup(_sub(st, 0, 2), oq, p), oracle.lookup(_sub(st, 2, 4), oq, p)]
+    assert parts[0].status[0] == oracle.HIT and parts[0].key_score[0] == 0.9375
+    assert whole.status[0] == oracle.REJECT and whole.key_score[0] == 1.0 and list(whole.cand_id[0]) == [0, 2]
+    merged = oracle.merge_shards(parts, [0, 2], p)
+    _assert_same(merged, whole)
+
+
 def test_merge_rejects_mismatched_bases():
     w = wl.WORKLOADS["tiny-4k"]
     st, oq, p = _store(w), _queries(w), _params(w)
