@@ -121,14 +121,15 @@ def algorithmic(w, batch):
     return stage1_bytes, stage2_bytes, flops
 
 
-def kernel_traffic(stage1: str, workload: str):
+def kernel_traffic(stage1: str, workload: str, variant: str = ""):
     """DRAM bytes per launch of the stage-1 kernel from the committed ncu capture, if the kernel source has not
-    changed since the capture (else None)."""
+    changed since the capture (else None). `variant` names a setting the traffic depends on (the SimHash
+    signature width)."""
     path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
-        rec = json.load(f).get(f"stage1_{stage1}/{workload}")
+        rec = json.load(f).get(f"stage1_{stage1}{variant}/{workload}")
     if not rec:
         return None
     src = os.path.join(ROOT, "paper_2608_01718_gb300", "csrc", STAGE1_SOURCES[stage1])
@@ -387,7 +388,7 @@ def run_ours(args, w):
     peaks, peak_src = load_peaks()
     s1_bytes, s2_bytes, flops = algorithmic(w, w.batch)
     t1_avg_s = t1_ms / max(1, timed) / 1e3
-    traffic = None if args.entries else kernel_traffic(kernel_name, w.name)
+    traffic = None if args.entries else kernel_traffic(kernel_name, w.name, f"-b{lsh['bits']}" if lsh else "")
     value = job["value"]
     # the stage-1 kernel is bound by HBM below the ridge (flops per byte of the measured peaks), else by the
     # tensor pipe; a kernel timed back to back for over a second is compared with the sustained bf16 peak

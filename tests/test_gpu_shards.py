@@ -104,3 +104,35 @@ def test_merge_rejects_bad_arguments():
         with pytest.raises(L.LacacheError) as e:
             L.lacache_merge_shards(shards, c, models, out)
         assert e.value.status == L.LACACHE_ERR_INVALID_ARG
+
+
+def test_merged_key_score_when_a_shard_hit_falls_past_the_cut():
+    # query e0, top_c 2; shard A holds entries scoring 1 and 0.9375, shard B 0.984375 and 0.96875. Only entry 1
+    # (0.9375) passes the lookahead check: shard A serves it, but globally it is third, past the cut. The merged
+    # result is the whole store's: a REJECT of candidates [0, 2] whose key score is the best one, 1.
+    d, B, c = 64, 1, 2
+    eye = torch.eye(d, dtype=torch.float32)
+    keys = torch.zeros((4, d))
+    keys[:, 0] = torch.tensor([1.0, 0.9375, 0.984375, 0.96875])
+    pres = torch.stack([eye[2], eye[1], eye[2], eye[2]])
+    ids = torch.zeros((4, 1), dtype=torch.int32)
+    q = {"emb": eye[:1].to(torch.bfloat16).cuda(), "prefix": eye[1:2].to(torch.bfloat16).cuda(),
+         "ids": torch.zeros((1, 1), dtype=torch.int32, device="cuda")}
+    gathered = torch.zeros((2, sharded.record_bytes(B, c, 1)), dtype=torch.uint8, device="cuda")
+    shards, own = [], []
+    for g, (a, b) in enumerate([(0, 2), (2, 4)]):
+        with L.LaCache(d, 1, 2, 0.5, 0.5, c, max_batch=4) as part:
+            part.insert(keys[a:b].to(torch.bfloat16).cuda(), pres[a:b].to(torch.bfloat16).cuda(), ids[a:b].cuda())
+            rec = sharded.views(gathered[g], B, c, 1)
+            out = {**L.alloc_result(B, c, "cuda", candidates=False), **rec}
+            part.lookup(q["emb"], q["prefix"], q["ids"], out=out)
+            torch.cuda.synchronize()
+            own.append((int(out["status"][0]), float(out["key_score"][0])))
+        shards.append((rec, a))
+    assert own[0] == (L.LACACHE_HIT, 0.9375) and own[1] == (L.LACACHE_REJECT, 0.984375)
+    merged = L.alloc_result(B, c, "cuda", candidates=True)
+    L.lacache_merge_shards(shards, c, 1, merged)
+    torch.cuda.synchronize()
+    assert int(merged["status"][0]) == L.LACACHE_REJECT and float(merged["key_score"][0]) == 1.0
+    assert merged["cand_id"][0].tolist() == [0, 2] and int(merged["entry_id"][0]) == -1
+    assert float(merged["prefix_score"][0]) == 0.0
