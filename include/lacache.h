@@ -58,9 +58,10 @@ typedef enum {
 
 typedef enum { LACACHE_BF16 = 0, LACACHE_F32 = 1 } lacache_dtype;
 
-/* Which stage-1 kernel lookups run. AUTO picks by batch size. */
+/* Which stage-1 kernel lookups run. */
 typedef enum {
-  LACACHE_STAGE1_AUTO = 0,
+  LACACHE_STAGE1_AUTO = 0,   /* the tensor-core scan at every batch size: even one query keeps the scan bound by
+                                HBM, where the CUDA-core scan is bound by FFMA issue from a few queries up */
   LACACHE_STAGE1_TENSOR = 1, /* tcgen05 tensor-core scan (TMA-fed, TMEM accumulators) */
   LACACHE_STAGE1_SIMT = 2,   /* CUDA-core FFMA scan */
   LACACHE_STAGE1_LSH = 3,    /* SimHash index, then the exact key check (requires lacache_enable_lsh) */
