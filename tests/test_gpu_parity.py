@@ -79,6 +79,16 @@ def test_ragged_batch_dimension_and_k(stage1):
 
 
 @pytest.mark.parametrize("stage1", PATHS)
+@pytest.mark.parametrize("d,k,batch", [(8, 1, 1), (8192, 256, 40)], ids=["smallest", "largest"])
+def test_dimension_and_window_extremes(stage1, d, k, batch):
+    # the smallest dimension, window and batch a handle accepts, and the largest dimension and window: one k-step of
+    # 8 elements against 128 k-steps, and 1 token id against 256 per candidate row
+    w = wl.WORKLOADS["mid-1m"].scaled(n=3_000, d=d, k=k, batch=batch, clusters=30, vocab=5)
+    rep = run_parity(w, stage1, steps=(0, 1))
+    assert rep.exact + rep.band == 2 * w.batch
+
+
+@pytest.mark.parametrize("stage1", PATHS)
 def test_odd_number_of_query_tiles(stage1):
     # B = 300: three query tiles; the tensor kernel pairs query tiles on two-CTA clusters, so the third tile's
     # partner has no queries. n = 12,050: the last key tile holds 18 keys, so its upper half (the second CTA's
