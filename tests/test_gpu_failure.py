@@ -27,7 +27,10 @@ def library():
 
 @pytest.mark.parametrize("batch", [32, 256], ids=["single-cta", "cta-pairs"])
 def test_stage1_wait_timeout_is_reported_and_the_context_stays_usable(batch):
-    w = wl.WORKLOADS["mid-1m"].scaled(n=40_000, batch=batch)
+    # A single query tile runs on the dynamic schedule, where CTAs claim key tiles as they start: with about one
+    # tile per CTA a late-starting CTA 0 could claim none and have no load to withhold. 400,000 entries are
+    # 1,563 tiles, so CTA 0 always claims some.
+    w = wl.WORKLOADS["mid-1m"].scaled(n=400_000 if batch <= 128 else 40_000, batch=batch)
     with L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch,
                    stage1=L.LACACHE_STAGE1_TENSOR) as cache:
         for ch in wl.iter_store(w, "cuda"):
