@@ -259,7 +259,9 @@ lacache_status lacache_stage_times(lacache_t* h, double* stage1_ms, double* stag
  * issuer's bounded wait (about one second) runs out. The kernel then records LACACHE_ERR_DEVICE_TIMEOUT, its other
  * roles stop, its issued copies and MMAs drain, TMEM is freed and it exits. The context stays usable: the next
  * lacache_sync reports the timeout and later lookups run normally. The affected lookup's outputs are undefined.
- * On CTA pairs (B > 128) the first CTA is the leader of the first pair; its abort stops its peer too. 0 cancels. */
+ * On CTA pairs (B > 128) the first CTA is the leader of the first pair; its abort stops its peer too. A single
+ * query tile (B <= 128) runs on a dynamic schedule: the stall happens only if the first CTA claims a key tile, which
+ * is certain when the store holds many more 256-key tiles than the GPU has SMs. 0 cancels. */
 lacache_status lacache_inject_stall(lacache_t* h, int32_t lookups);
 
 /* Lookup that allocates nothing, for callers that cannot allocate device memory. Examples: a serving runtime or
