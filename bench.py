@@ -32,7 +32,8 @@ sys.path.insert(0, ROOT)
 METRIC = "lookups/sec at 1 GB300 (N entries, batch B, k) + % of HBM or bf16 roofline"
 UNIT = "queries/s"
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "tensor-pair": "stage1_tensor.cu", "simt": "stage1_simt.cu", "lsh": "lsh.cu"}
+STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "tensor-pair": "stage1_tensor.cu", "simt": "stage1_simt.cu",
+                  "lsh": "lsh.cu"}
 
 
 def parse_args():

@@ -199,7 +199,8 @@ lacache_status lacache_read_signatures(const lacache_t* h, int64_t first, int64_
                                        void* cuda_stream);
 
 /* Copy entries [first, first + n) of the store into caller device buffers (key_dev [n x d], prefix_dev
- * [n x prefix row] bf16, ids_dev [n x k]); any of the three may be NULL. For checkpoints and checks. Asynchronous on cuda_stream. */
+ * [n x prefix row] bf16, ids_dev [n x k]); any of the three may be NULL. For checkpoints and checks. Asynchronous on
+ * cuda_stream. */
 lacache_status lacache_read_rows(const lacache_t* h, int64_t first, int64_t n, void* key_dev, void* prefix_dev,
                                  int32_t* ids_dev, void* cuda_stream);
 

@@ -181,7 +181,8 @@ extern "C" lacache_status lacache_calibrate(int64_t n, int32_t d, const void* x_
   if (rank < 1) rank = 1;
   if (rank > n) rank = n;
   int dev = 0, sms = 0;
-  if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return LACACHE_ERR_CUDA;
   return lc::launch_calibrate(x_dev, y_dev, n, d, rank - 1, cap, sims_dev, result_dev, workspace_dev, sms,
                               (cudaStream_t)cuda_stream) == cudaSuccess

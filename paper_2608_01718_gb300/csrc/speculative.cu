@@ -41,7 +41,8 @@ extern "C" lacache_status lacache_verify_draft(int32_t B, int32_t k, const float
   if (B < 1 || k < 1 || k > lc::kMaxK || !p_target_dev || !p_draft_dev || !accepted_dev)
     return LACACHE_ERR_INVALID_ARG;
   const int blocks = (B + lc::kVerifyWarps - 1) / lc::kVerifyWarps;
-  lc::verify_draft_kernel<<<blocks, lc::kVerifyWarps * 32, 0, (cudaStream_t)cuda_stream>>>(B, k, p_target_dev, p_draft_dev,
-                                                                                    status_dev, accepted_dev);
+  const cudaStream_t st = (cudaStream_t)cuda_stream;
+  lc::verify_draft_kernel<<<blocks, lc::kVerifyWarps * 32, 0, st>>>(B, k, p_target_dev, p_draft_dev, status_dev,
+                                                                   accepted_dev);
   return cudaGetLastError() == cudaSuccess ? LACACHE_OK : LACACHE_ERR_CUDA;
 }

@@ -114,7 +114,8 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
       keep(loc, x[u]);
     }
   }
-  for (int s = threadIdx.x + 2 * kThreads; s < a.splits; s += kThreads) best = fmaxf(best, a.part_best[(int64_t)s * a.B + q]);
+  for (int s = threadIdx.x + 2 * kThreads; s < a.splits; s += kThreads)
+    best = fmaxf(best, a.part_best[(int64_t)s * a.B + q]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(kFull, best, o));
   if (lane == 0) warp_best[warp] = best;

@@ -23,11 +23,11 @@ LACACHE_MAX_MODELS = 8
 LACACHE_MAX_SHARDS = 16
 
 EXPORTS = ["lacache_create", "lacache_create_ensemble", "lacache_destroy", "lacache_insert", "lacache_lookup",
-           "lacache_lookup_host", "lacache_lookup_host_async",
-           "lacache_append_misses", "lacache_read_rows", "lacache_size", "lacache_sync", "lacache_last_launch",
-           "lacache_stage_timing", "lacache_stage_times", "lacache_inject_stall", "lacache_enable_lsh", "lacache_read_signatures", "lacache_calibrate", "lacache_calibrate_workspace_bytes", "lacache_verify_draft",
-           "lacache_lookup_noalloc", "lacache_merge_shards", "lacache_get_stats", "lacache_save", "lacache_load",
-           "lacache_get_config",
+           "lacache_lookup_host", "lacache_lookup_host_async", "lacache_append_misses", "lacache_read_rows",
+           "lacache_size", "lacache_sync", "lacache_last_launch", "lacache_stage_timing", "lacache_stage_times",
+           "lacache_inject_stall", "lacache_enable_lsh", "lacache_read_signatures", "lacache_calibrate",
+           "lacache_calibrate_workspace_bytes", "lacache_verify_draft", "lacache_lookup_noalloc",
+           "lacache_merge_shards", "lacache_get_stats", "lacache_save", "lacache_load", "lacache_get_config",
            "lacache_status_string"]
 
 

@@ -132,7 +132,8 @@ def compare(gpu: dict, res: oracle.Result, p: oracle.Params, rows=None, pair_sco
         msg = f"query {g} (oracle row {b})"
         assert st == res.status[b], f"{msg}: status {st} vs oracle {res.status[b]}"
         assert gpu["entry_id"][g] == res.entry_id[b], f"{msg}: entry {gpu['entry_id'][g]} vs {res.entry_id[b]}"
-        assert _close(gpu["key_score"][g], res.key_score[b]), f"{msg}: key score {gpu['key_score'][g]} vs {res.key_score[b]}"
+        assert _close(gpu["key_score"][g], res.key_score[b]), \
+            f"{msg}: key score {gpu['key_score'][g]} vs {res.key_score[b]}"
         assert _close(gpu["prefix_score"][g], res.prefix_score[b]), f"{msg}: prefix score"
         assert gpu["token_matches"][g] == res.token_matches[b], f"{msg}: token matches"
         if "prefix_scores" in gpu:

@@ -174,7 +174,8 @@ def _of_views(rec):
         prefix_score=nan, token_matches=np.full(B, -1, np.int32), n_cand=rec["n_cand"].numpy(),
         n_above=rec["n_cand"].numpy().astype(np.int64), cand_id=rec["cand_id"].numpy(),
         cand_score=rec["cand_score"].numpy(), cand_prefix_score=rec["cand_prefix_score"].numpy(),
-        cand_matches=rec["cand_matches"].numpy(), prefix_scores=np.full((B, rec["cand_prefix_scores"].shape[2]), np.nan),
+        cand_matches=rec["cand_matches"].numpy(),
+        prefix_scores=np.full((B, rec["cand_prefix_scores"].shape[2]), np.nan),
         cand_pass=rec["cand_pass"].numpy().astype(bool), cand_prefix_scores=rec["cand_prefix_scores"].numpy(),
         margin=nan, list_margin=nan, literal_margin=nan, next_id=np.full(B, -1, np.int32), next_score=nan)
 
