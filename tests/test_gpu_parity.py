@@ -311,6 +311,36 @@ def test_serve_loop_appends_misses_like_the_oracle(stage1):
         assert np.array_equal(ids.cpu().numpy(), loop.store.ids[w.n:loop.n])
 
 
+@pytest.mark.parametrize("batch", [32, 200], ids=["dynamic-schedule", "cta-pairs"])
+def test_two_handles_look_up_concurrently_on_two_streams(batch):
+    # Each handle owns its store, scratch and schedule counters: lookups of two handles interleaved on two streams,
+    # several in flight at once, give each handle's own sequential results.
+    wa = wl.WORKLOADS["mid-1m"].scaled(n=60_000, batch=batch)
+    wb = wl.WORKLOADS["serve-2m"].scaled(n=45_000, batch=batch, clusters=300)
+    with new_cache(wa, L.LACACHE_STAGE1_TENSOR) as ca, new_cache(wb, L.LACACHE_STAGE1_TENSOR) as cb:
+        fill(ca, wa)
+        fill(cb, wb)
+        qa = [wl.batch(wa, i, device="cuda") for i in range(3)]
+        qb = [wl.batch(wb, i, device="cuda") for i in range(3)]
+        want_a = [gpu_lookup(ca, q) for q in qa]
+        want_b = [gpu_lookup(cb, q) for q in qb]
+        sa, sb = torch.cuda.Stream(), torch.cuda.Stream()
+        outs_a = [L.alloc_result(batch, wa.top_c, "cuda") for _ in qa]
+        outs_b = [L.alloc_result(batch, wb.top_c, "cuda") for _ in qb]
+        torch.cuda.synchronize()
+        for _ in range(2):
+            for i in range(3):
+                ca.lookup(qa[i]["emb"], qa[i]["prefix"], qa[i]["ids"], out=outs_a[i], cuda_stream=sa)
+                cb.lookup(qb[i]["emb"], qb[i]["prefix"], qb[i]["ids"], out=outs_b[i], cuda_stream=sb)
+        torch.cuda.synchronize()
+        ca.sync()
+        cb.sync()
+        for outs, want in ((outs_a, want_a), (outs_b, want_b)):
+            for o, g in zip(outs, want):
+                for k, v in o.items():
+                    assert np.array_equal(v.cpu().numpy(), g[k], equal_nan=True), k
+
+
 def test_insert_is_all_or_nothing_on_capacity():
     with L.LaCache(64, 2, 10, 0.9, 0.8, 2, max_batch=4) as c:
         rows = _dev(np.eye(64)[:8])
