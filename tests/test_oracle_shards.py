@@ -217,3 +217,50 @@ def test_two_gloo_ranks_merge_to_the_whole_store_lookup():
             assert pr.exitcode == 0
         res = dict(results)
     assert res[0] == res[1] and res[0][0] == [0, 2048] and res[0][1] > 0
+
+
+# ---- failure detection on the host: a rank that dies between lookups ---------------------------------------------
+
+def _rank_that_may_die(rank, world, port, results):
+    import datetime
+    import time
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world, timeout=datetime.timedelta(seconds=10))
+    w = wl.WORKLOADS["tiny-4k"]
+    st, oq, p = _store(w), _queries(w), _params(w)
+    a, b = w.n * rank // world, w.n * (rank + 1) // world
+    mine = _sub(st, a, b)
+    lk = sharded.ShardedLookup(
+        w.batch, w.top_c, 1, a, "cpu",
+        local_lookup=lambda queries, rec: _to_views(oracle.lookup(mine, queries, p), rec),
+        merge=lambda shards, o: o.update(res=oracle.merge_shards([_of_views(v) for v, _ in shards],
+                                                                 [base for _, base in shards], p)),
+        float_dtype=torch.float64)
+    out = {}
+    lk(oq, out)                     # one lookup completes on both ranks
+    if rank == 1:
+        os._exit(3)                 # then this rank dies, with nothing of the next exchange started
+    t0 = time.monotonic()
+    try:
+        lk(oq, out)
+        results[rank] = ("completed", 0.0)
+    except Exception as e:          # the exchange reports the lost peer instead of waiting forever
+        results[rank] = (type(e).__name__, time.monotonic() - t0)
+
+
+def test_a_dead_rank_fails_the_next_exchange_instead_of_hanging():
+    world = 2
+    ctx = mp.get_context("spawn")
+    with ctx.Manager() as mgr:
+        results = mgr.dict()
+        port = _free_port()
+        procs = [ctx.Process(target=_rank_that_may_die, args=(r, world, port, results)) for r in range(world)]
+        for pr in procs:
+            pr.start()
+        for pr in procs:
+            pr.join(120)
+        codes = [pr.exitcode for pr in procs]
+        res = dict(results)
+    assert codes[1] == 3
+    assert 0 in res and res[0][0] != "completed", res
+    assert res[0][1] < 60.0, res    # bounded by the process group's timeout, not an indefinite wait
