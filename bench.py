@@ -33,7 +33,7 @@ METRIC = "lookups/sec at 1 GB300 (N entries, batch B, k) + % of HBM or bf16 roof
 UNIT = "queries/s"
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "tensor-pair": "stage1_tensor.cu", "simt": "stage1_simt.cu",
-                  "lsh": "lsh.cu"}
+                  "lsh": "lsh.cu", "lsh-tensor": "lsh_tc.cu"}
 
 
 def parse_args():
@@ -295,8 +295,8 @@ def run_ours(args, w):
     torch.cuda.synchronize()
     cache.sync()
     kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_TENSOR_PAIR: "tensor-pair",
-                   L.LACACHE_STAGE1_SIMT: "simt",
-                   L.LACACHE_STAGE1_LSH: "lsh"}[cache.last_launch()[1]]
+                   L.LACACHE_STAGE1_SIMT: "simt", L.LACACHE_STAGE1_LSH: "lsh",
+                   L.LACACHE_STAGE1_LSH_TENSOR: "lsh-tensor"}[cache.last_launch()[1]]
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
@@ -394,7 +394,13 @@ def run_ours(args, w):
     # the stage-1 kernel is bound by HBM below the ridge (flops per byte of the measured peaks), else by the
     # tensor pipe; a kernel timed back to back for over a second is compared with the sustained bf16 peak
     ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
-    if lsh:
+    if lsh and kernel_name == "lsh-tensor":
+        # The tensor-core SimHash scan streams the expanded index, N x bits bytes per lookup (one byte per signature
+        # bit), and is bound by HBM; the admitted key rows it gathers are not counted.
+        index_bytes = w.n * lsh["bits"]
+        roof = {"bound": "hbm", "achieved": index_bytes / t1_avg_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "peak_source": f"{peak_src} (copy bandwidth)", "algorithmic_index_bytes_per_launch": index_bytes}
+    elif lsh:
         # The SimHash scan is bound by integer work on its B x N x (bits / 32) signature-word comparisons per
         # lookup. Population count runs at 16 per clock per SM (the CUDA arithmetic-throughput table), the logic
         # and integer operations at 64. The scan's carry-save adders fold 8 words into 5 popcounts (4 into 3), whose
@@ -425,7 +431,8 @@ def run_ours(args, w):
         "stage1_kernel": kernel_name,
         "lsh_index": lsh,
         "roofline": roof | {"traffic": traffic, "kernel": f"stage1_{kernel_name}",
-                            "algorithmic_bytes_per_launch": s1_bytes, "algorithmic_flops_per_launch": flops,
+                            "algorithmic_bytes_per_launch": roof.get("algorithmic_index_bytes_per_launch", s1_bytes),
+                            "algorithmic_flops_per_launch": flops,
                             "avg_launch_ms": t1_avg_s * 1e3},
         "tensor": {"achieved_tflops": flops / (elapsed_ms / args.steps / 1e3) / 1e12,
                    "peak_tflops": peaks["bf16_tflops"],

@@ -21,8 +21,7 @@ LIB = os.path.join(BUILD, "liblacache.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["api.cu", "stage1_simt.cu", "stage1_tensor.cu", "stage2.cu", "noalloc.cu", "calibrate.cu", "lsh.cu",
-           "speculative.cu",
-           "shards.cu"]
+           "lsh_tc.cu", "speculative.cu", "shards.cu"]
 
 
 def nvcc() -> str:
@@ -44,7 +43,8 @@ def build(verbose: bool = False, force: bool = False) -> str:
     """Compile every CUDA source and link liblacache.so; returns its path."""
     os.makedirs(BUILD, exist_ok=True)
     srcs = [os.path.join(CSRC, s) for s in SOURCES]
-    deps = srcs + [os.path.join(CSRC, "internal.cuh"), os.path.join(INCLUDE, "lacache.h"), __file__]
+    deps = srcs + [os.path.join(CSRC, h) for h in ("internal.cuh", "tcgen05.cuh")]
+    deps += [os.path.join(INCLUDE, "lacache.h"), __file__]
     if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= max(os.path.getmtime(p) for p in deps):
         return LIB
     tool = nvcc()

@@ -44,6 +44,7 @@ struct lacache {
   uint32_t* sig;             // [capacity x lsh_bits/32] entry signatures
   uint32_t* qsig;            // [max_batch x lsh_bits/32] query signatures of the current lookup
   __nv_bfloat16* hyper;      // [lsh_bits x d] hyperplanes
+  uint8_t* sig_index;        // the signatures expanded for the tensor-core scan (lsh_index_bytes)
   cudaEvent_t* events;       // [3 x event_cap] stage-timing events, or NULL
   int event_cap;
   int event_used;
@@ -261,17 +262,22 @@ void free_lsh(lacache* h) {
   cudaFree(h->sig);
   cudaFree(h->qsig);
   cudaFree(h->hyper);
+  cudaFree(h->sig_index);
   h->sig = h->qsig = nullptr;
   h->hyper = nullptr;
+  h->sig_index = nullptr;
   h->lsh_bits = 0;
 }
 
-// Signatures of store rows [first, first + n), when the index is enabled.
+// Signatures of store rows [first, first + n), packed and expanded, when the index is enabled.
 cudaError_t sign_rows(lacache* h, int64_t first, int64_t n, cudaStream_t st) {
   if (!h->lsh_bits || n <= 0) return cudaSuccess;
   const int words = h->lsh_bits / 32;
-  return lc::launch_signatures(h->key + first * h->cfg.d, n, h->cfg.d, h->hyper, h->lsh_bits, h->sig + first * words,
-                               h->dev_status, h->encode, h->num_sms, st);
+  cudaError_t e = lc::launch_signatures(h->key + first * h->cfg.d, n, h->cfg.d, h->hyper, h->lsh_bits,
+                                        h->sig + first * words, h->dev_status, h->encode, h->num_sms, st);
+  if (e == cudaSuccess && h->sig_index)
+    e = lc::launch_expand_signatures(h->sig, first, n, h->lsh_bits, h->sig_index, h->num_sms, st);
+  return e;
 }
 
 void free_all(lacache* h) {
@@ -332,8 +338,13 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
       e = lc::launch_signatures(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, h->dev_status, h->encode, h->num_sms,
                                 st);
       if (e == cudaSuccess) {
-        lc::LshArgs l{h->sig, h->qsig, h->lsh_bits / 32, h->lsh_radius};
-        e = lc::launch_stage1_lsh(a, l, h->num_sms, h->max_splits, st, &splits);
+        lc::LshArgs l{h->sig, h->qsig, h->lsh_bits / 32, h->lsh_radius, h->sig_index};
+        if (B >= lc::kLshTensorMinBatch && h->sig_index) {
+          e = lc::launch_stage1_lsh_tc(a, l, h->num_sms, h->max_splits, st, &splits);
+          kernel = LACACHE_STAGE1_LSH_TENSOR;
+        } else {
+          e = lc::launch_stage1_lsh(a, l, h->num_sms, h->max_splits, st, &splits);
+        }
       }
     } else {
       e = lc::launch_stage1_simt(a, h->num_sms, h->max_splits, st, &splits);
@@ -674,13 +685,18 @@ lacache_status lacache_enable_lsh(lacache_t* h, int32_t bits, int32_t radius, co
   free_lsh(h);
   const int words = bits / 32;
   const lacache_config& c = h->cfg;
+  // the expanded copy only where batches can be large enough to use it
+  const size_t index_bytes = c.max_batch >= lc::kLshTensorMinBatch ? lc::lsh_index_bytes(c.capacity, bits) : 0;
   if (cudaMalloc(&h->sig, (size_t)c.capacity * words * 4) != cudaSuccess ||
       cudaMalloc(&h->qsig, (size_t)c.max_batch * words * 4) != cudaSuccess ||
-      cudaMalloc(&h->hyper, (size_t)bits * c.d * 2) != cudaSuccess) {
+      cudaMalloc(&h->hyper, (size_t)bits * c.d * 2) != cudaSuccess ||
+      (index_bytes && cudaMalloc(&h->sig_index, index_bytes) != cudaSuccess)) {
     cudaGetLastError();
     free_lsh(h);
     return LACACHE_ERR_OOM;
   }
+  // rows past the valid entries of the last block are read by the scan (and never used): keep them defined
+  if (index_bytes && cudaMemsetAsync(h->sig_index, 0, index_bytes, st) != cudaSuccess) return LACACHE_ERR_CUDA;
   h->lsh_bits = bits;
   h->lsh_radius = radius;
   if (cudaMemcpyAsync(h->hyper, hyperplanes_dev, (size_t)bits * c.d * 2, cudaMemcpyDeviceToDevice, st) !=

@@ -130,9 +130,20 @@ struct LshArgs {
   const uint32_t* qsig;    // [B x words] query signatures
   int words;
   int radius;
+  const uint8_t* index;    // the same signatures as e4m3 +-1 bytes in swizzled 128-entry blocks (lsh_tc.cu)
 };
+// Popcount scan (small batches) and the tensor-core scan over the expanded index (batches of at least
+// kLshTensorMinBatch queries).
 cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits, cudaStream_t st,
                               int* splits);
+cudaError_t launch_stage1_lsh_tc(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits,
+                                 cudaStream_t st, int* splits);
+constexpr int kLshTensorMinBatch = 48;
+// Bytes of the expanded index for `capacity` entries (whole 128-entry blocks of `bits` bytes each), and its update
+// from the packed signatures of entries [first, first + n).
+size_t lsh_index_bytes(int64_t capacity, int bits);
+cudaError_t launch_expand_signatures(const uint32_t* sig, int64_t first, int64_t n, int bits, uint8_t* index,
+                                     int num_sms, cudaStream_t st);
 
 // Largest split count any stage-1 launcher uses for a given SM count (sizes the scratch): the SimHash scan runs two
 // CTAs per SM, the other kernels at most one split per SM.

@@ -17,6 +17,7 @@ LACACHE_CHECK_EMB, LACACHE_CHECK_TOKENS, LACACHE_CHECK_BOTH = 0, 1, 2
 LACACHE_BF16, LACACHE_F32 = 0, 1
 LACACHE_STAGE1_AUTO, LACACHE_STAGE1_TENSOR, LACACHE_STAGE1_SIMT, LACACHE_STAGE1_LSH = 0, 1, 2, 3
 LACACHE_STAGE1_TENSOR_PAIR = 4   # reported by lacache_last_launch only
+LACACHE_STAGE1_LSH_TENSOR = 5    # reported by lacache_last_launch only
 LACACHE_MISS_KEY, LACACHE_HIT, LACACHE_REJECT = 0, 1, 2
 
 LACACHE_MAX_MODELS = 8

@@ -51,9 +51,14 @@ def test_signatures_match_the_oracle(bits):
     assert amb.mean() < 1e-3
 
 
+def _expected_lsh_kernel(batch):
+    return L.LACACHE_STAGE1_LSH_TENSOR if batch >= 48 else L.LACACHE_STAGE1_LSH
+
+
+@pytest.mark.parametrize("batch", [5, 40, 64], ids=["popcount-5", "popcount-40", "tensor"])
 @pytest.mark.parametrize("bits", [128, 256, 512])
-def test_lsh_lookup_matches_the_oracle(bits):
-    w = wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=40)
+def test_lsh_lookup_matches_the_oracle(bits, batch):
+    w = wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch)
     radius = wl.lsh_radius(w.tau_c, bits)
     R = wl.hyperplanes(bits, w.d, device="cuda")
     st = oracle_store(w)
@@ -62,22 +67,27 @@ def test_lsh_lookup_matches_the_oracle(bits):
         L.lacache_enable_lsh(cache.h, bits, radius, R)
         q = wl.batch(w, 0, device="cuda")
         g = gpu_lookup(cache, q)
+        assert cache.last_launch()[1] == _expected_lsh_kernel(batch)
     oq = oracle_queries(q)
     p = params(w)
     res, amb = oracle.lookup_lsh(st, oq, p, wl.bf16_bits(R), radius)
     keep = np.nonzero(~amb)[0]
     sub = oracle.Result(**{f: getattr(res, f)[keep] for f in res.__dataclass_fields__})
     rep = compare(g, sub, p, rows=keep)
-    log_report(f"lsh bits={bits} radius={radius} ({w.batch - len(keep)} queries with ambiguous bits)", rep)
+    log_report(f"lsh bits={bits} B={batch} radius={radius} ({w.batch - len(keep)} queries with ambiguous bits)", rep)
     assert rep.exact + rep.band == len(keep) and len(keep) >= w.batch - 2
-    assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
+    if batch >= 16:
+        assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
     # at this radius the index keeps every near-duplicate's target: the decisions equal the exact lookup's
     exact = oracle.lookup(st, oq, p)
     assert np.array_equal(res.status, exact.status) and np.array_equal(res.entry_id, exact.entry_id)
 
 
-def test_full_radius_equals_the_exact_scan_and_appends_are_signed():
-    w = wl.WORKLOADS["serve-2m"].scaled(n=30_000, batch=64, clusters=300)
+@pytest.mark.parametrize("batch", [16, 64], ids=["popcount", "tensor"])
+def test_full_radius_equals_the_exact_scan_and_appends_are_signed(batch):
+    # radius = bits admits every pair: the queue overflows on every tile, and appended entries must be signed (in
+    # both the packed and the expanded form) before the next lookup
+    w = wl.WORKLOADS["serve-2m"].scaled(n=30_000, batch=batch, clusters=300)
     R = wl.hyperplanes(256, w.d, device="cuda")
     with new_cache(w, L.LACACHE_STAGE1_TENSOR, capacity=w.n + 4 * w.batch) as exact_cache, \
             new_cache(w, L.LACACHE_STAGE1_LSH, capacity=w.n + 4 * w.batch) as lsh_cache:
@@ -88,6 +98,7 @@ def test_full_radius_equals_the_exact_scan_and_appends_are_signed():
             q = wl.batch(w, step, device="cuda")
             a = exact_cache.lookup(q["emb"], q["prefix"], q["ids"])
             b = lsh_cache.lookup(q["emb"], q["prefix"], q["ids"])
+            assert lsh_cache.last_launch()[1] == _expected_lsh_kernel(batch)
             assert torch.equal(a["status"], b["status"]) and torch.equal(a["entry_id"], b["entry_id"])
             assert torch.equal(a["cand_id"], b["cand_id"])
             assert torch.allclose(a["cand_score"], b["cand_score"], atol=2e-3, equal_nan=True)
