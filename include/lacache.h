@@ -147,8 +147,11 @@ lacache_status lacache_insert(lacache_t* h, int64_t n, const void* key_dev, cons
  * queries, q_prefix_dev [B x prefix row] bf16 embeddings of their speculatively decoded k-token prefixes f_k(x),
  * q_ids_dev [B x k] int32 those token ids. Stage 1 keeps per query the top_c entries with key score >= tau_c by
  * (score desc, id asc); stage 2 checks them in that order and serves the first that passes. Writes every
- * non-NULL field of *out (device pointers). Asynchronous on cuda_stream; no host synchronization. The call may be
- * captured into a CUDA graph (stream capture). Replays then read the captured input and output pointers, and scan
+ * non-NULL field of *out (device pointers). Asynchronous on cuda_stream; no host synchronization. Back-to-back
+ * lookups on one stream overlap: a lookup's stage 1 scans while the previous lookup's stage 2 finishes, so the
+ * query inputs of a lookup must not alias the output arrays of the lookup issued just before it on the stream
+ * (any other work issued in between orders them as usual). The call may be captured into a CUDA graph (stream
+ * capture). Replays then read the captured input and output pointers, and scan
  * the entries present at capture time: capture again after inserts or appends. */
 lacache_status lacache_lookup(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,
                               const int32_t* q_ids_dev, const lacache_result* out, void* cuda_stream);

@@ -137,7 +137,7 @@ __global__ void append_rows_kernel(const uint4* __restrict__ q_emb, const uint4*
 // lookup_host's inputs, read by the device straight from mapped pinned host memory (NVLink-C2C on Grace) into the
 // device staging: one launch for the three arrays instead of one DMA copy each. Segments with zero bytes are
 // skipped; 16-byte vectors where both ends are aligned, bytes otherwise. Lets the stage-1 grid (a programmatic
-// dependent) start its set-up at once; that grid reads nothing before this one has completed.
+// dependent) start its set-up at once; that grid is launched to wait for this one before reading anything.
 struct GatherSeg {
   const unsigned char* src;
   unsigned char* dst;
@@ -299,8 +299,9 @@ void free_all(lacache* h) {
   if (h->stage_host) cudaFreeHost(h->stage_host);
 }
 
+// gathered: the queries were just written by gather_host_kernel, so the first kernel waits for it before reading.
 lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* q_prefix, const int32_t* q_ids,
-                          const lacache_result& out, cudaStream_t st) {
+                          const lacache_result& out, cudaStream_t st, bool gathered = false) {
   const lacache_config& c = h->cfg;
   if (!lookup_ready(h)) return LACACHE_ERR_INVALID_ARG;
   int splits = 0;
@@ -320,6 +321,7 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
     a.part_cand = h->part_cand;
     a.part_best = h->part_best;
     a.dev_status = h->dev_status;
+    a.inputs_from_previous = gathered ? 1 : 0;
     kernel = c.stage1 == LACACHE_STAGE1_AUTO ? LACACHE_STAGE1_TENSOR : c.stage1;
     if (h->inject_stall > 0 && kernel == LACACHE_STAGE1_TENSOR) {
       a.inject_stall = 1;
@@ -336,7 +338,7 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
       if (paired) kernel = LACACHE_STAGE1_TENSOR_PAIR;
     } else if (kernel == LACACHE_STAGE1_LSH) {
       e = lc::launch_signatures(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, h->dev_status, h->encode, h->num_sms,
-                                st);
+                                st, gathered);
       if (e == cudaSuccess) {
         lc::LshArgs l{h->sig, h->qsig, h->lsh_bits / 32, h->lsh_radius, h->sig_index};
         if (B >= lc::kLshTensorMinBatch && h->sig_index) {
@@ -580,7 +582,8 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
   unsigned char* out_stage = h->stage_host_dev ? h->stage_host_dev : h->stage_out;
   lacache_result dev = staged_result(out_stage, B, c.top_c, h->ens.m, *out_host, &bytes);
   lacache_result host = staged_result(h->stage_host, B, c.top_c, h->ens.m, *out_host, &bytes);
-  lacache_status s = run_lookup(h, B, in.dst[0], in.dst[1], reinterpret_cast<const int32_t*>(in.dst[2]), dev, st);
+  lacache_status s =
+      run_lookup(h, B, in.dst[0], in.dst[1], reinterpret_cast<const int32_t*>(in.dst[2]), dev, st, gathered != 0);
   if (s != LACACHE_OK) return s;
   if (!h->stage_host_dev &&
       cudaMemcpyAsync(h->stage_host, h->stage_out, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess)
@@ -638,7 +641,7 @@ lacache_status lacache_lookup_host_async(lacache_t* h, int32_t B, const void* q_
   if (!mapped) return LACACHE_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
   if (launch_gather(h, g, gathered, st) != cudaSuccess) return LACACHE_ERR_CUDA;
-  return run_lookup(h, B, in.dst[0], in.dst[1], reinterpret_cast<const int32_t*>(in.dst[2]), dev, st);
+  return run_lookup(h, B, in.dst[0], in.dst[1], reinterpret_cast<const int32_t*>(in.dst[2]), dev, st, true);
 }
 
 lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_dev, const void* q_prefix_dev,

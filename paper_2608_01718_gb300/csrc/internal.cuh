@@ -80,6 +80,8 @@ struct Stage1Args {
   int* tile_ctr;              // tensor kernel, one query tile: dynamic tile schedule on these two counters
                               // [next tile, CTAs done], zero at launch and zero again when the grid ends
                               // (nullptr: static schedule)
+  int inputs_from_previous;   // tensor kernel: the queries are written by the grid launched just before (the
+                              // host-input gather), so wait for it before reading anything
 };
 
 struct Stage2Args {
@@ -119,9 +121,10 @@ cudaError_t launch_stage2(const Stage2Args& a, cudaStream_t st);
 
 // SimHash signatures of n rows ([n x d] bf16) against `bits` hyperplanes ([bits x d] bf16), bits a multiple of 32:
 // sig[j * bits/32 + w] bit i is set iff <hyperplane 32w + i, row j> >= 0 (tensor-core GEMM, sign epilogue).
+// rows_from_previous: the rows are written by the grid launched just before (wait for it before reading).
 cudaError_t launch_signatures(const __nv_bfloat16* rows, int64_t n, int d, const __nv_bfloat16* hyperplanes,
                               int bits, uint32_t* sig, unsigned int* dev_status, EncodeTiledFn encode, int num_sms,
-                              cudaStream_t st);
+                              cudaStream_t st, bool rows_from_previous = false);
 
 // The SimHash-indexed key check: entries whose signature is within `radius` of the query's get the exact key
 // check (threshold + top-c partial lists, as the other stage-1 kernels).

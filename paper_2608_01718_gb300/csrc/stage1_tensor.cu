@@ -81,6 +81,7 @@ struct TcParams {
   int a_rows;     // rows of the query box: B rounded up to 8 when B <= 128, else 128
   int inject_stall;  // test support: CTA 0 withholds its second load, so its MMA issuer's bounded wait runs out
   int* tile_ctr;      // dynamic schedule: [next tile, CTAs done], zero at launch and left zero (nullptr: static)
+  int wait_first;     // wait for the preceding grids before reading anything (they write the queries)
   uint32_t* sig;     // signature mode: [n x sig_words] output words
   int sig_words;
   uint64_t* part_cand;
@@ -258,10 +259,14 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  // Launched as a programmatic dependent of the previous lookup's stage 2: the set-up above overlaps it, and no
-  // global memory is read or written before the preceding grids have completed. Then let this lookup's stage 2
-  // be scheduled; it waits for this grid's completion before reading anything.
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // Launched as a programmatic dependent of the previous lookup's stage 2. That grid reads the partial lists
+  // this one writes, and writes nothing this one reads, so the scan runs alongside it: each epilogue thread waits
+  // for the preceding grids (griddepcontrol.wait) only before its first global write. Inputs written by earlier
+  // work on the stream are complete, because those kernels let their dependents start only when they finish. The
+  // one exception, the host-input gather, writes the queries and starts its dependent early: then every thread
+  // waits here, before reading anything. This lookup's stage 2 may be scheduled now; it waits for this grid's
+  // completion before reading anything.
+  if (p.wait_first) asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   auto fail = [&]() {
@@ -437,6 +442,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     TopC<CPAD> top;
     float best = -INFINITY;
     // One finished accumulator: the 256 scores of key tile t for this thread's query row.
+    bool waited = p.wait_first != 0;   // this thread has waited for the preceding grids
+    auto dep_wait = [&]() {
+      if (!waited) {
+        asm volatile("griddepcontrol.wait;" ::: "memory");
+        waited = true;
+      }
+    };
     auto epi_tile = [&](int64_t t, bool active, int word) -> bool {
       const int b = tile_i & 1u;
       const uint32_t par = (tile_i >> 1) & 1u;
@@ -463,6 +475,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t w = __ballot_sync(full, v[e] >= 0.f);
             if (lane == e) mine = w;
           }
+          dep_wait();
           if (word < p.sig_words && jc + lane < p.n) p.sig[(jc + lane) * p.sig_words + word] = mine;
         } else if (active) {
           const int64_t jc = j0 + ch * 32;
@@ -504,6 +517,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       return true;
     };
     auto write_partial = [&](int sp, int q) {
+      dep_wait();
       uint64_t* dst = p.part_cand + ((int64_t)sp * p.B + q) * p.top_c;
 #pragma unroll
       for (int i = 0; i < CPAD; ++i)
@@ -696,9 +710,10 @@ cudaError_t launch_key_check(TcParams p, const Stage1Args& a, EncodeTiledFn enco
 
 cudaError_t launch_signatures(const __nv_bfloat16* rows, int64_t n, int d, const __nv_bfloat16* hyperplanes,
                               int bits, uint32_t* sig, unsigned int* dev_status, EncodeTiledFn encode, int num_sms,
-                              cudaStream_t st) {
+                              cudaStream_t st, bool rows_from_previous) {
   if (n <= 0) return cudaSuccess;
   TcParams p{};
+  p.wait_first = rows_from_previous ? 1 : 0;
   p.n = n;
   p.d = d;
   p.B = bits;
@@ -740,6 +755,7 @@ cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int 
   p.part_best = a.part_best;
   p.dev_status = a.dev_status;
   p.inject_stall = a.inject_stall;
+  p.wait_first = a.inputs_from_previous;
   if (a.top_c <= 4) return launch_key_check<4>(p, a, encode, num_sms, max_splits, st, splits, paired);
   if (a.top_c <= 8) return launch_key_check<8>(p, a, encode, num_sms, max_splits, st, splits, paired);
   if (a.top_c <= 16) return launch_key_check<16>(p, a, encode, num_sms, max_splits, st, splits, paired);
