@@ -268,7 +268,12 @@ def run_ours(args, w):
     build.build()
     stage1 = {"auto": L.LACACHE_STAGE1_AUTO, "tensor": L.LACACHE_STAGE1_TENSOR, "simt": L.LACACHE_STAGE1_SIMT,
               "lsh": L.LACACHE_STAGE1_LSH}
-    cache = L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch, device=local_rank,
+    # A workload with a step count is a serve loop (Algorithm 1 batch by batch): every timed step looks up a fresh
+    # batch and then appends its misses, so the store grows while it is timed; the capacity holds that growth.
+    serve = w.steps > 1
+    warm = max(3, args.warmup)
+    capacity = w.n + (warm + args.steps) * w.batch if serve else w.n
+    cache = L.LaCache(w.d, w.k, capacity, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch, device=local_rank,
                       stage1=stage1[args.stage1], prefix_dims=w.prefix_dims, tau_a_models=w.tau_a_models)
     dtype = L.LACACHE_F32 if w.key_dtype == "f32" else L.LACACHE_BF16
     for ch in wl.iter_store(w, "cuda"):
@@ -290,10 +295,21 @@ def run_ours(args, w):
         q = batches[i % nb]
         L.lacache_lookup(cache.h, q["emb"], q["prefix"], q["ids"], outs[i % nb], stream)
 
-    for i in range(max(3, args.warmup)):
-        step(i)
+    if serve:
+        # distinct batches for the warm-up and timed steps, generated before timing starts
+        serve_batches = [wl.batch(w, step=i, device="cuda") for i in range(warm + args.steps)]
+
+        def serve_step(i):
+            q = serve_batches[i]
+            out = outs[i % nb]
+            L.lacache_lookup(cache.h, q["emb"], q["prefix"], q["ids"], out, stream)
+            cache.append_misses(q["emb"], q["prefix"], q["ids"], out["status"], stream)   # synchronizes
+
+    for i in range(warm):
+        (serve_step if serve else step)(i)
     torch.cuda.synchronize()
     cache.sync()
+    n_timed_begin = cache.size
     kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_TENSOR_PAIR: "tensor-pair",
                    L.LACACHE_STAGE1_SIMT: "simt", L.LACACHE_STAGE1_LSH: "lsh",
                    L.LACACHE_STAGE1_LSH_TENSOR: "lsh-tensor"}[cache.last_launch()[1]]
@@ -305,7 +321,7 @@ def run_ours(args, w):
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     ev0.record(stream)
     for i in range(args.steps):
-        step(i)
+        serve_step(warm + i) if serve else step(i)
     ev1.record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -313,6 +329,7 @@ def run_ours(args, w):
     clock = clocks.stop()
     cache.sync()
     elapsed_ms = ev0.elapsed_time(ev1)
+    n_timed_end = cache.size
     # Second pass over the same steps with the library's stage events (recorded on the lookup's stream around
     # each kernel) for the per-kernel times of the roofline. The events sit between the two kernels, so this pass
     # is kept out of the throughput measurement above.
@@ -387,7 +404,9 @@ def run_ours(args, w):
     d2h = w.batch * (4 + 1 + 4 + 4 + 4 + 4)
 
     peaks, peak_src = load_peaks()
-    s1_bytes, s2_bytes, flops = algorithmic(w, w.batch)
+    # a serve loop scans a growing store: the stage-timing pass ran on the store as the timed steps left it
+    w_alg = w.scaled(n=n_timed_end) if serve else w
+    s1_bytes, s2_bytes, flops = algorithmic(w_alg, w.batch)
     t1_avg_s = t1_ms / max(1, timed) / 1e3
     traffic = None if args.entries else kernel_traffic(kernel_name, w.name, f"-b{lsh['bits']}" if lsh else "")
     value = job["value"]
@@ -427,7 +446,11 @@ def run_ours(args, w):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": workload_config(w) | {"parallelism": f"replicas{world}" if world > 1 else "single"},
+        "config": workload_config(w) | {"parallelism": f"replicas{world}" if world > 1 else "single"} |
+                  ({"serve_loop": {"steps_timed": args.steps, "entries_at_start": n_timed_begin,
+                                   "entries_at_end": n_timed_end,
+                                   "step": "lookup, then append of the batch's misses (lacache_append_misses)"}}
+                   if serve else {}),
         "stage1_kernel": kernel_name,
         "lsh_index": lsh,
         "roofline": roof | {"traffic": traffic, "kernel": f"stage1_{kernel_name}",
@@ -444,7 +467,7 @@ def run_ours(args, w):
                 "api": f"lacache_lookup_host_async (mapped pinned host buffers, {depth} lookups in flight)"},
         "e2e_sync": {"value": sync_job["e2e_value"], "unit": UNIT, "steps": args.e2e_steps,
                      "api": "lacache_lookup_host (pinned host buffers, one synchronous call per step)"},
-        "gpu_launches": (3 if lsh else 2) * args.steps,
+        "gpu_launches": ((3 if lsh else 2) + (2 if serve else 0)) * args.steps,
         "clocks": clock,
         "decisions": decision_rates(w, batches[0], outs[0]),
     }
