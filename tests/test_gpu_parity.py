@@ -341,6 +341,30 @@ def test_two_handles_look_up_concurrently_on_two_streams(batch):
                     assert np.array_equal(v.cpu().numpy(), g[k], equal_nan=True), k
 
 
+def test_back_to_back_lookups_of_mixed_sizes_match_lookups_run_alone():
+    # A lookup's stage 1 scans while the previous lookup's stage 2 finishes, and both use the handle's partial-list
+    # scratch and schedule counters. Lookups of changing batch size (single CTAs on the dynamic schedule and CTA
+    # pairs, growing and shrinking the scratch they cover), enqueued back to back with no synchronization, must
+    # each give the result of the same lookup run alone.
+    w = wl.WORKLOADS["mid-1m"].scaled(n=60_000, batch=200)
+    sizes = [32, 7, 200, 64, 1, 130, 32, 200, 5]
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+        fill(cache, w)
+        full = [wl.batch(w, i, device="cuda") for i in range(len(sizes))]
+        qs = [{k: full[i][k][:b].contiguous() for k in ("emb", "prefix", "ids")} for i, b in enumerate(sizes)]
+        alone = [gpu_lookup(cache, q) for q in qs]
+        outs = [L.alloc_result(b, w.top_c, "cuda") for b in sizes]
+        torch.cuda.synchronize()
+        for rep in range(2):
+            for q, o in zip(qs, outs):
+                cache.lookup(q["emb"], q["prefix"], q["ids"], out=o)
+            torch.cuda.synchronize()
+            cache.sync()
+            for o, g in zip(outs, alone):
+                for k, v in o.items():
+                    assert np.array_equal(v.cpu().numpy(), g[k], equal_nan=True), (rep, k)
+
+
 def test_insert_is_all_or_nothing_on_capacity():
     with L.LaCache(64, 2, 10, 0.9, 0.8, 2, max_batch=4) as c:
         rows = _dev(np.eye(64)[:8])
