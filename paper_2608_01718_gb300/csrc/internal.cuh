@@ -141,7 +141,7 @@ cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms
                               int* splits);
 cudaError_t launch_stage1_lsh_tc(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits,
                                  cudaStream_t st, int* splits);
-constexpr int kLshTensorMinBatch = 48;
+constexpr int kLshTensorMinBatch = 40;
 // Bytes of the expanded index for `capacity` entries (whole 128-entry blocks of `bits` bytes each), and its update
 // from the packed signatures of entries [first, first + n).
 size_t lsh_index_bytes(int64_t capacity, int bits);

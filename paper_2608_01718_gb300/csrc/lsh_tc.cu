@@ -12,10 +12,12 @@
 // whenever entries are signed, so one bulk copy moves a block from HBM into an operand stage.
 //
 // One CTA per contiguous range of blocks, warp-specialised:
-//   warp 5 (loader): cp.async.bulk of one block per stage into a kS-deep ring;
-//   warp 4 (MMA): allocates TMEM; per block issues tcgen05.mma.kind::f8f6f4 (M = 128 entries, N = the pass's
+//   warp 17 (loader): cp.async.bulk of one block per stage into a kS-deep ring;
+//   warp 16 (MMA): allocates TMEM; per block issues tcgen05.mma.kind::f8f6f4 (M = 128 entries, N = the pass's
 //     queries rounded up to 16, K = 32) over the resident query operand, into one of kNbuf accumulators;
-//   warps 0-3 (epilogue, TMEM lane quadrants 0-3): expand the pass's query signatures into the query operand; per
+//   warps 0-15 (epilogue; warp w reads TMEM lane quadrant w % 4 and the 32-query column chunks c with
+//     c % 4 = w / 4, so up to four warps share each entry's dot products): expand the pass's query signatures into
+//     the query operand; per
 //     block read each entry's dot products, turn them into a mask of the admitted queries, release the
 //     accumulator, and queue the admitted (query, entry) pairs in shared memory. When the queue passes three
 //     quarters of its capacity, and at the end of the range, they compute the exact fp32 key score of every queued
@@ -31,10 +33,11 @@
 namespace lc {
 namespace {
 
-constexpr int kEpiWarps = 4;                             // warps 0-3: TMEM lane quadrants 0-3
-constexpr int kMmaWarp = 4;
-constexpr int kLoadWarp = 5;
-constexpr int kThreads = 6 * 32;
+constexpr int kEpiGroups = 4;                            // epilogue warps per TMEM lane quadrant
+constexpr int kEpiWarps = 4 * kEpiGroups;                // warps 0-15: lane quadrant w % 4, group w / 4
+constexpr int kMmaWarp = kEpiWarps;                      // warp 16
+constexpr int kLoadWarp = kEpiWarps + 1;                 // warp 17
+constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr int kCap = 1024;                               // queue capacity
 constexpr int kFlushAt = kCap - kCap / 4;                // a block that leaves more items than this is flushed
 constexpr int kBlockRows = 128;                          // entries per block and MMA (TMEM lanes)
@@ -98,7 +101,7 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// The epilogue warps' own barrier (named barrier 1, 128 threads), and its OR form.
+// The epilogue warps' own barrier (named barrier 1, all epilogue threads), and its OR form.
 __device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory"); }
 __device__ __forceinline__ bool epi_any(bool p) {
   uint32_t r;
@@ -157,8 +160,8 @@ __device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a_desc, uint6
       : "memory");
 }
 
-// Exact scores of the queued items (the four epilogue warps), then the warp of each query folds its items into
-// the query's list. ew = epilogue warp 0..3.
+// Exact scores of the queued items (all epilogue warps), then the warp of each query folds its items into
+// the query's list. ew = epilogue warp.
 __device__ void flush(Tail& t, uint64_t* lists, const Stage1Args& a, int q0, int qn, int ew, int lane) {
   const int total = min(t.count, kCap);   // pairs that found the queue full were not stored
   const int v = a.d / 8;
@@ -366,8 +369,9 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
       it += (uint32_t)nb;
     } else {
       // ---------------- epilogue ----------------
-      const int ew = warp;                                 // = TMEM lane quadrant
-      const uint32_t lane_addr = (uint32_t)(ew * 32) << 16;
+      const int ew = warp;                                 // epilogue warp
+      const int quad = ew % 4, group = ew / 4;             // TMEM lane quadrant; column chunks c % 4 == group
+      const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
       bool stop = false;
       for (int64_t ti = 0; ti < nb && !stop; ++ti) {
         const int b = tb % G::kNbuf;
@@ -382,7 +386,7 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
           tc_fence_after();
 #pragma unroll
           for (int c = 0; c < G::kQC / 32; ++c) {
-            if (32 * c < npad) {   // the same for the whole warp
+            if (c % kEpiGroups == group && 32 * c < npad) {   // the same for the whole warp
               float v[32];
               tmem_ld32(tmem + lane_addr + (uint32_t)(b * G::kQC) + 32u * c, v);
               uint32_t mask = 0;
@@ -396,10 +400,10 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
           __syncwarp();
           if (lane == 0) mbar_arrive(tempty_bar(b));
         }
-        const int64_t j = (g_begin + ti) * kBlockRows + ew * 32 + lane;
+        const int64_t j = (g_begin + ti) * kBlockRows + quad * 32 + lane;
         const bool valid = got && j < j_end;
         // queue the admitted pairs; flush while the queue is past kFlushAt or a pair found it full (every round
-        // either queues all pending pairs or fills the queue, so this ends). All four warps leave together.
+        // either queues all pending pairs or fills the queue, so this ends). All epilogue warps leave together.
         int top = -1;
         for (;;) {
           bool left = false;

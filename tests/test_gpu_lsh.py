@@ -52,10 +52,10 @@ def test_signatures_match_the_oracle(bits):
 
 
 def _expected_lsh_kernel(batch):
-    return L.LACACHE_STAGE1_LSH_TENSOR if batch >= 48 else L.LACACHE_STAGE1_LSH
+    return L.LACACHE_STAGE1_LSH_TENSOR if batch >= 40 else L.LACACHE_STAGE1_LSH
 
 
-@pytest.mark.parametrize("batch", [5, 40, 64], ids=["popcount-5", "popcount-40", "tensor"])
+@pytest.mark.parametrize("batch", [5, 32, 40, 64], ids=["popcount-5", "popcount-32", "tensor-40", "tensor-64"])
 @pytest.mark.parametrize("bits", [128, 256, 512])
 def test_lsh_lookup_matches_the_oracle(bits, batch):
     w = wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch)
