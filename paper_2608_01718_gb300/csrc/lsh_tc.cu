@@ -17,13 +17,13 @@
 //     queries rounded up to 16, K = 32) over the resident query operand, into one of kNbuf accumulators;
 //   warps 0-15 (epilogue; warp w reads TMEM lane quadrant w % 4 and the 32-query column chunks c with
 //     c % 4 = w / 4, so up to four warps share each entry's dot products): expand the pass's query signatures into
-//     the query operand; per
-//     block read each entry's dot products, turn them into a mask of the admitted queries, release the
-//     accumulator, and queue the admitted (query, entry) pairs in shared memory. When the queue passes three
-//     quarters of its capacity, and at the end of the range, they compute the exact fp32 key score of every queued
-//     pair over the gathered key row (each lane's 8-element chunks in order, then a butterfly sum) and fold the
-//     scores that clear tau_c into the query's top-c list. A pair that finds the queue full stays in its thread's
-//     pending mask and is queued again after the next flush.
+//     the query operand; per block read each entry's dot products, and only where their maximum reaches the
+//     threshold turn them into a mask of the admitted queries; release the accumulator; after every kRound blocks
+//     queue the admitted (query, entry) pairs in shared memory. When the queue passes three quarters of its
+//     capacity, and at the end of the range, they compute the exact fp32 key score of every queued pair over the
+//     gathered key row (four pairs per warp at a time; each lane's 8-element chunks in order, then a butterfly sum),
+//     and one thread per query folds that query's scores that clear tau_c into its top-c list. A pair that finds
+//     the queue full stays in its thread's pending mask and is queued again after the next flush.
 // Queries are taken kQC at a time (one pass over the range each). Every mbarrier wait is bounded: on a timeout the
 // CTA records LACACHE_ERR_DEVICE_TIMEOUT in the status word, the roles stop at the next pass boundary, in-flight
 // copies and MMAs are drained, TMEM is freed and the CTA exits.
@@ -39,7 +39,8 @@ constexpr int kMmaWarp = kEpiWarps;                      // warp 16
 constexpr int kLoadWarp = kEpiWarps + 1;                 // warp 17
 constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr int kCap = 1024;                               // queue capacity
-constexpr int kFlushAt = kCap - kCap / 4;                // a block that leaves more items than this is flushed
+constexpr int kFlushAt = kCap - kCap / 4;                // a round that leaves more items than this is flushed
+constexpr int kRound = 4;                                // blocks the epilogue takes between its barriers
 constexpr int kBlockRows = 128;                          // entries per block and MMA (TMEM lanes)
 constexpr int kAtomBytes = 128;                          // K bytes per swizzle atom (128 e4m3 values)
 constexpr unsigned kFull = 0xffffffffu;
@@ -57,6 +58,8 @@ struct TcGeo {
   static constexpr int kNbuf = 512 / kQC;                      // 4 or 8
   static_assert(kNbuf * kQC == 512, "TMEM columns");
 };
+constexpr int kPer = (128 / 32 + kEpiGroups - 1) / kEpiGroups;   // column chunks per epilogue warp (at most)
+static_assert(kEpiWarps * 32 >= 128, "one epilogue thread per query of a pass folds that query's items");
 
 struct Item {
   int32_t j;      // entry id
@@ -160,49 +163,64 @@ __device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a_desc, uint6
       : "memory");
 }
 
-// Exact scores of the queued items (all epilogue warps), then the warp of each query folds its items into
-// the query's list. ew = epilogue warp.
-__device__ void flush(Tail& t, uint64_t* lists, const Stage1Args& a, int q0, int qn, int ew, int lane) {
+// Exact scores of the queued items (all epilogue warps), then one thread per query folds that query's items into
+// its list. ew = epilogue warp. Inlined, with the kernel's arguments passed as values: the queue and the lists
+// stay shared-memory accesses and nothing goes through local memory, which the exact check's key rows evict from
+// L1.
+__device__ __forceinline__ void flush(Tail& t, uint64_t* lists, const __nv_bfloat16* __restrict__ keys,
+                                      const __nv_bfloat16* __restrict__ q, int d, float tau_c, int C, int q0, int qn,
+                                      int ew, int lane) {
   const int total = min(t.count, kCap);   // pairs that found the queue full were not stored
-  const int v = a.d / 8;
-  for (int base = ew * 2; base < total; base += kEpiWarps * 2) {
-    float acc0 = 0.f, acc1 = 0.f;
-    const Item i0 = t.items[base];
-    const bool two = base + 1 < total;
-    const Item i1 = two ? t.items[base + 1] : i0;
-    const uint4* k0 = reinterpret_cast<const uint4*>(a.keys + (int64_t)i0.j * a.d);
-    const uint4* k1 = reinterpret_cast<const uint4*>(a.keys + (int64_t)i1.j * a.d);
-    const uint4* x0 = reinterpret_cast<const uint4*>(a.q + (int64_t)(q0 + i0.q) * a.d);
-    const uint4* x1 = reinterpret_cast<const uint4*>(a.q + (int64_t)(q0 + i1.q) * a.d);
-    for (int c = lane; c < v; c += 32) {
-      acc0 = dot8(__ldg(x0 + c), __ldg(k0 + c), acc0);
-      acc1 = dot8(__ldg(x1 + c), __ldg(k1 + c), acc1);
+  const int v = d / 8;
+  constexpr int kItems = 4;   // queue items per warp at a time: their key-row loads are in flight together
+  for (int base = ew * kItems; base < total; base += kEpiWarps * kItems) {
+    float acc[kItems];
+    const uint4* kp[kItems];
+    const uint4* xp[kItems];
+#pragma unroll
+    for (int u = 0; u < kItems; ++u) {
+      const Item it = t.items[base + u < total ? base + u : base];
+      kp[u] = reinterpret_cast<const uint4*>(keys + (int64_t)it.j * d);
+      xp[u] = reinterpret_cast<const uint4*>(q + (int64_t)(q0 + it.q) * d);
+      acc[u] = 0.f;
     }
-    acc0 = warp_sum(acc0);
-    acc1 = warp_sum(acc1);
+#pragma unroll 1
+    for (int c = lane; c < v; c += 32) {
+      uint4 kv[kItems], xv[kItems];
+#pragma unroll
+      for (int u = 0; u < kItems; ++u) {
+        kv[u] = __ldg(kp[u] + c);
+        xv[u] = __ldg(xp[u] + c);
+      }
+#pragma unroll
+      for (int u = 0; u < kItems; ++u) acc[u] = dot8(xv[u], kv[u], acc[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < kItems; ++u) acc[u] = warp_sum(acc[u]);
     if (lane == 0) {
-      t.score[base] = acc0;
-      if (two) t.score[base + 1] = acc1;
+#pragma unroll
+      for (int u = 0; u < kItems; ++u)
+        if (base + u < total) t.score[base + u] = acc[u];
     }
   }
   epi_sync();
-  const int C = a.top_c;
-  for (int qq = ew; qq < qn; qq += kEpiWarps) {
+  // one thread per query of the pass takes that query's items, in queue order, into its list
+  const int qq = ew * 32 + lane;
+  if (qq < qn) {
     float best = -INFINITY;
     uint64_t* L = lists + (size_t)qq * C;
-    for (int base = 0; base < total; base += 32) {
-      const int idx = base + lane;
-      const bool mine = idx < total && t.items[idx].q == qq;
-      const float sc = mine ? t.score[idx] : -INFINITY;
-      best = fmaxf(best, sc);
-      unsigned pass = __ballot_sync(kFull, mine && sc >= a.tau_c);
-      while (pass) {   // lane 0 inserts the passing items of this group one by one
-        const int src = __ffs(pass) - 1;
-        pass &= pass - 1;
-        const float s = __shfl_sync(kFull, sc, src);
-        const int j = __shfl_sync(kFull, mine ? t.items[idx].j : 0, src);
-        if (lane == 0) {
-          const uint64_t x = pack_cand(s, (uint32_t)j);
+    for (int i0 = 0; i0 < total; i0 += 8) {
+      uint32_t m = 0;   // this query's items among the next 8 (the loads are independent and overlap)
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (i0 + u < total && t.items[i0 + u].q == qq) m |= 1u << u;
+      while (m) {
+        const int i = i0 + __ffs(m) - 1;
+        m &= m - 1;
+        const float sc = t.score[i];
+        best = fmaxf(best, sc);
+        if (sc >= tau_c) {
+          const uint64_t x = pack_cand(sc, (uint32_t)t.items[i].j);
           if (x > L[C - 1]) {
             int p = C - 1;
             while (p > 0 && L[p - 1] < x) {
@@ -214,9 +232,7 @@ __device__ void flush(Tail& t, uint64_t* lists, const Stage1Args& a, int q0, int
         }
       }
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(kFull, best, o));
-    if (lane == 0 && best > -INFINITY) atomicMax(&t.best[qq], score_order(best));
+    if (best > -INFINITY) t.best[qq] = max(t.best[qq], score_order(best));
   }
   epi_sync();
   if (ew == 0 && lane == 0) t.count = 0;
@@ -373,57 +389,76 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
       const int quad = ew % 4, group = ew / 4;             // TMEM lane quadrant; column chunks c % 4 == group
       const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
       bool stop = false;
-      for (int64_t ti = 0; ti < nb && !stop; ++ti) {
-        const int b = tb % G::kNbuf;
-        const uint32_t tph = (tb / G::kNbuf) & 1u;
-        ++tb;
-        const bool got = mbar_wait(tfull_bar(b), tph, abort_flag);
-        // the admitted queries of this thread's entry, as bit masks over the pass's queries
-        uint32_t pend[G::kQC / 32];
+      for (int64_t t0 = 0; t0 < nb && !stop; t0 += kRound) {
+        // the admitted queries of this thread's entry in each block of the round, as bit masks over the warp's
+        // column chunks (chunk group + kEpiGroups u)
+        uint32_t pend[kRound][kPer];
+        bool got = true;
 #pragma unroll
-        for (int c = 0; c < G::kQC / 32; ++c) pend[c] = 0;
-        if (__all_sync(kFull, got)) {   // the warp-collective loads below need the whole warp
+        for (int r = 0; r < kRound; ++r) {
+#pragma unroll
+          for (int u = 0; u < kPer; ++u) pend[r][u] = 0;
+          if (t0 + r >= nb || !got) continue;              // the same for every epilogue warp
+          const int b = tb % G::kNbuf;
+          const uint32_t tph = (tb / G::kNbuf) & 1u;
+          ++tb;
+          got = __all_sync(kFull, mbar_wait(tfull_bar(b), tph, abort_flag));
+          if (!got) continue;   // the warp-collective loads below need the whole warp
           tc_fence_after();
 #pragma unroll
-          for (int c = 0; c < G::kQC / 32; ++c) {
-            if (c % kEpiGroups == group && 32 * c < npad) {   // the same for the whole warp
+          for (int u = 0; u < kPer; ++u) {
+            const int c = group + kEpiGroups * u;
+            if (c < G::kQC / 32 && 32 * c < npad) {   // the same for the whole warp
               float v[32];
               tmem_ld32(tmem + lane_addr + (uint32_t)(b * G::kQC) + 32u * c, v);
-              uint32_t mask = 0;
+              // admitted pairs are rare: a max over the 32 scores decides whether the mask is built at all
+              float m[16];
 #pragma unroll
-              for (int i = 0; i < 32; ++i) mask |= (v[i] >= thr ? 1u : 0u) << i;
-              const int left = qn - 32 * c;
-              pend[c] = left >= 32 ? mask : (left > 0 ? mask & ((1u << left) - 1u) : 0u);
+              for (int i = 0; i < 16; ++i) m[i] = fmaxf(v[i], v[i + 16]);
+#pragma unroll
+              for (int w = 8; w > 0; w >>= 1)
+#pragma unroll
+                for (int i = 0; i < w; ++i) m[i] = fmaxf(m[i], m[i + w]);
+              if (m[0] >= thr) {
+                uint32_t mask = 0;
+#pragma unroll
+                for (int i = 0; i < 32; ++i) mask |= (v[i] >= thr ? 1u : 0u) << i;
+                const int left = qn - 32 * c;
+                pend[r][u] = left >= 32 ? mask : (left > 0 ? mask & ((1u << left) - 1u) : 0u);
+              }
             }
           }
           tc_fence_before();
           __syncwarp();
           if (lane == 0) mbar_arrive(tempty_bar(b));
         }
-        const int64_t j = (g_begin + ti) * kBlockRows + quad * 32 + lane;
-        const bool valid = got && j < j_end;
         // queue the admitted pairs; flush while the queue is past kFlushAt or a pair found it full (every round
         // either queues all pending pairs or fills the queue, so this ends). All epilogue warps leave together.
         int top = -1;
         for (;;) {
           bool left = false;
 #pragma unroll
-          for (int c = 0; c < G::kQC / 32; ++c) {
-            uint32_t p = valid ? pend[c] : 0u;
-            uint32_t full = 0;
-            while (p) {
-              const int bit = __ffs(p) - 1;
-              p &= p - 1;
-              const int slot = atomicAdd(&t.count, 1);
-              if (slot < kCap) {
-                t.items[slot] = Item{(int32_t)j, 32 * c + bit};
-                top = slot;
-              } else {
-                full |= 1u << bit;
+          for (int r = 0; r < kRound; ++r) {
+            const int64_t j = (g_begin + t0 + r) * kBlockRows + quad * 32 + lane;
+            const bool valid = got && j < j_end;
+#pragma unroll
+            for (int u = 0; u < kPer; ++u) {
+              uint32_t p = valid ? pend[r][u] : 0u;
+              uint32_t full = 0;
+              while (p) {
+                const int bit = __ffs(p) - 1;
+                p &= p - 1;
+                const int slot = atomicAdd(&t.count, 1);
+                if (slot < kCap) {
+                  t.items[slot] = Item{(int32_t)j, 32 * (group + kEpiGroups * u) + bit};
+                  top = slot;
+                } else {
+                  full |= 1u << bit;
+                }
               }
+              pend[r][u] = full;
+              left |= full != 0;
             }
-            pend[c] = full;
-            left |= full != 0;
           }
           if (!epi_any(!got || *abort_flag || left || top >= kFlushAt)) break;
           if (epi_any(!got || *abort_flag)) {
@@ -431,7 +466,7 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
             stop = true;
             break;
           }
-          flush(t, lists, a, q0, qn, ew, lane);
+          flush(t, lists, a.keys, a.q, a.d, a.tau_c, C, q0, qn, ew, lane);
           top = -1;
         }
       }
@@ -441,7 +476,7 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
     // ---- pass end: every role is here; a timeout anywhere stops them all together ----
     if (__syncthreads_or(*abort_flag != 0)) break;
     if (warp < kEpiWarps) {
-      flush(t, lists, a, q0, qn, warp, lane);
+      flush(t, lists, a.keys, a.q, a.d, a.tau_c, C, q0, qn, warp, lane);
       const int et = threadIdx.x;
       for (int i = et; i < qn * C; i += kEpiWarps * 32) {
         const int qq = i / C;
