@@ -55,7 +55,10 @@ def _expected_lsh_kernel(batch):
     return L.LACACHE_STAGE1_LSH_TENSOR if batch >= 40 else L.LACACHE_STAGE1_LSH
 
 
-@pytest.mark.parametrize("batch", [5, 32, 40, 64], ids=["popcount-5", "popcount-32", "tensor-40", "tensor-64"])
+# popcount-36: two passes of 32 queries (the handle's max_batch is below the tensor scan's minimum, so it keeps no
+# expanded index); tensor-200: two passes of 128 queries at 128 and 256 bits, four of 64 at 512, ragged last pass
+@pytest.mark.parametrize("batch", [5, 32, 36, 40, 64, 200],
+                         ids=["popcount-5", "popcount-32", "popcount-36", "tensor-40", "tensor-64", "tensor-200"])
 @pytest.mark.parametrize("bits", [128, 256, 512])
 def test_lsh_lookup_matches_the_oracle(bits, batch):
     w = wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch)
@@ -75,7 +78,8 @@ def test_lsh_lookup_matches_the_oracle(bits, batch):
     sub = oracle.Result(**{f: getattr(res, f)[keep] for f in res.__dataclass_fields__})
     rep = compare(g, sub, p, rows=keep)
     log_report(f"lsh bits={bits} B={batch} radius={radius} ({w.batch - len(keep)} queries with ambiguous bits)", rep)
-    assert rep.exact + rep.band == len(keep) and len(keep) >= w.batch - 2
+    # queries with a signature bit within the fp32/fp64 ambiguity of zero are set aside: at most 1 in 50
+    assert rep.exact + rep.band == len(keep) and len(keep) >= w.batch - max(2, w.batch // 50)
     if batch >= 16:
         assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
     # at this radius the index keeps every near-duplicate's target: the decisions equal the exact lookup's
