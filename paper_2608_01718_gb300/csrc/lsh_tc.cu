@@ -15,15 +15,20 @@
 //   warp 17 (loader): cp.async.bulk of one block per stage into a kS-deep ring;
 //   warp 16 (MMA): allocates TMEM; per block issues tcgen05.mma.kind::f8f6f4 (M = 128 entries, N = the pass's
 //     queries rounded up to 16, K = 32) over the resident query operand, into one of kNbuf accumulators;
-//   warps 0-15 (epilogue; warp w reads TMEM lane quadrant w % 4 and the 32-query column chunks c with
-//     c % 4 = w / 4, so up to four warps share each entry's dot products): expand the pass's query signatures into
-//     the query operand; per block read each entry's dot products, and only where their maximum reaches the
+//   warps 0-7 (mask warps; warp w reads TMEM lane quadrant w % 4 and the 32-query column chunks c with
+//     c % 2 = w / 4): per block read each entry's dot products, and only where their maximum reaches the
 //     threshold turn them into a mask of the admitted queries; release the accumulator; after every kRound blocks
-//     queue the admitted (query, entry) pairs in shared memory. When the queue passes three quarters of its
-//     capacity, and at the end of the range, they compute the exact fp32 key score of every queued pair over the
-//     gathered key row (four pairs per warp at a time; each lane's 8-element chunks in order, then a butterfly sum),
-//     and one thread per query folds that query's scores that clear tau_c into its top-c list. A pair that finds
-//     the queue full stays in its thread's pending mask and is queued again after the next flush.
+//     queue the admitted (query, entry) pairs in shared memory, each slot stamped with the queue's epoch;
+//   warps 8-15 (checker warps): claim queued pairs kItems at a time as they arrive, compute their exact fp32 key
+//     scores over the gathered key rows (each lane's 8-element chunks in order, then a butterfly sum) while the
+//     scan goes on, and fold each score into its query's best score and, if it clears tau_c, into the query's
+//     top-c list (under a per-query lock).
+// When the queue passes three quarters of its capacity, and at the end of the range, the mask warps close it: the
+// checkers finish what was queued below the close, then the queue is emptied and reopened in a new epoch. A pair
+// that finds the queue full stays in its thread's pending mask and is queued after the reopening. All sixteen
+// epilogue warps expand the pass's query signatures into the query operand and write the lists out. The checker
+// warps leave their loop only at a reopening, which the mask warps always run at the end of a pass, also after a
+// timeout, so every named barrier sees all its warps.
 // Queries are taken kQC at a time (one pass over the range each). Every mbarrier wait is bounded: on a timeout the
 // CTA records LACACHE_ERR_DEVICE_TIMEOUT in the status word, the roles stop at the next pass boundary, in-flight
 // copies and MMAs are drained, TMEM is freed and the CTA exits.
@@ -33,14 +38,17 @@
 namespace lc {
 namespace {
 
-constexpr int kEpiGroups = 4;                            // epilogue warps per TMEM lane quadrant
-constexpr int kEpiWarps = 4 * kEpiGroups;                // warps 0-15: lane quadrant w % 4, group w / 4
+constexpr int kMaskGroups = 2;                           // mask warps per TMEM lane quadrant
+constexpr int kMaskWarps = 4 * kMaskGroups;              // warps 0-7: lane quadrant w % 4, group w / 4
+constexpr int kCheckWarps = 8;                           // warps 8-15: exact checks of the queued pairs
+constexpr int kEpiWarps = kMaskWarps + kCheckWarps;      // warps 0-15
 constexpr int kMmaWarp = kEpiWarps;                      // warp 16
 constexpr int kLoadWarp = kEpiWarps + 1;                 // warp 17
 constexpr int kThreads = (kEpiWarps + 2) * 32;
 constexpr int kCap = 1024;                               // queue capacity
-constexpr int kFlushAt = kCap - kCap / 4;                // a round that leaves more items than this is flushed
-constexpr int kRound = 4;                                // blocks the epilogue takes between its barriers
+constexpr int kFlushAt = kCap - kCap / 4;                // a round that leaves more items than this closes the queue
+constexpr int kRound = 4;                                // blocks the mask warps take between their barriers
+constexpr int kItems = 4;                                // queue items a checker warp claims at a time
 constexpr int kBlockRows = 128;                          // entries per block and MMA (TMEM lanes)
 constexpr int kAtomBytes = 128;                          // K bytes per swizzle atom (128 e4m3 values)
 constexpr unsigned kFull = 0xffffffffu;
@@ -58,21 +66,26 @@ struct TcGeo {
   static constexpr int kNbuf = 512 / kQC;                      // 4 or 8
   static_assert(kNbuf * kQC == 512, "TMEM columns");
 };
-constexpr int kPer = (128 / 32 + kEpiGroups - 1) / kEpiGroups;   // column chunks per epilogue warp (at most)
-static_assert(kEpiWarps * 32 >= 128, "one epilogue thread per query of a pass folds that query's items");
+constexpr int kPer = (128 / 32 + kMaskGroups - 1) / kMaskGroups;   // column chunks per mask warp (at most)
+static_assert(kEpiWarps * 32 >= 128, "the epilogue threads cover a pass's queries when they set up the lists");
 
 struct Item {
   int32_t j;      // entry id
   int32_t q;      // query within the pass
 };
 
-// Shared memory after the operands: the queue, the per-query best scores, flags and barriers; the per-query
-// lists follow it.
+// Shared memory after the operands: the queue, the per-query best scores and locks, flags and barriers; the
+// per-query lists follow it.
 struct Tail {
   Item items[kCap];
-  float score[kCap];
+  uint32_t ready[kCap];        // the epoch (reopenings so far) whose item the slot holds, written after the item
   unsigned int best[128];      // score_order of the best admitted score, per query of the pass
+  int lock[128];               // per query of the pass: its list is being updated
   int count;                   // queued items (may run past kCap: those pairs stay pending)
+  int claim;                   // queue positions claimed by the checker warps
+  int closed_at;               // while closing: min(count, kCap) when the queue was closed
+  uint32_t closing;            // the mask warps closed the queue
+  uint32_t pass_end;           // ... for the last time in the pass
   uint32_t abort_flag;
   uint32_t tmem_slot;
   uint32_t pad;
@@ -104,9 +117,8 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
-// The epilogue warps' own barrier (named barrier 1, all epilogue threads), and its OR form.
-__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 1, %0;" ::"n"(kEpiWarps * 32) : "memory"); }
-__device__ __forceinline__ bool epi_any(bool p) {
+// The mask warps' OR barrier (named barrier 1), and the barrier of all epilogue warps (named barrier 2).
+__device__ __forceinline__ bool mask_any(bool p) {
   uint32_t r;
   asm volatile(
       "{\n\t.reg .pred pi, po;\n\t"
@@ -114,10 +126,14 @@ __device__ __forceinline__ bool epi_any(bool p) {
       "bar.red.or.pred po, 1, %2, pi;\n\t"
       "selp.u32 %0, 1, 0, po;\n\t}"
       : "=r"(r)
-      : "r"((uint32_t)p), "n"(kEpiWarps * 32)
+      : "r"((uint32_t)p), "n"(kMaskWarps * 32)
       : "memory");
   return r != 0;
 }
+__device__ __forceinline__ void epi_sync() { asm volatile("bar.sync 2, %0;" ::"n"(kEpiWarps * 32) : "memory"); }
+
+__device__ __forceinline__ uint32_t ld_volatile(const uint32_t* p) { return *reinterpret_cast<const volatile uint32_t*>(p); }
+__device__ __forceinline__ void st_volatile(uint32_t* p, uint32_t v) { *reinterpret_cast<volatile uint32_t*>(p) = v; }
 
 // Four signature bits (bit i = K index i) as four e4m3 bytes: +1 (0x38) for a set bit, -1 (0xB8) for a clear one.
 // The complement's bit i lands on bit 8i + 7, the sign of byte i: 0x10204080 = 2^7 + 2^14 + 2^21 + 2^28, whose
@@ -163,79 +179,102 @@ __device__ __forceinline__ void mma_e4m3(uint32_t d_tmem, uint64_t a_desc, uint6
       : "memory");
 }
 
-// Exact scores of the queued items (all epilogue warps), then one thread per query folds that query's items into
-// its list. ew = epilogue warp. Inlined, with the kernel's arguments passed as values: the queue and the lists
-// stay shared-memory accesses and nothing goes through local memory, which the exact check's key rows evict from
-// L1.
-__device__ __forceinline__ void flush(Tail& t, uint64_t* lists, const __nv_bfloat16* __restrict__ keys,
-                                      const __nv_bfloat16* __restrict__ q, int d, float tau_c, int C, int q0, int qn,
-                                      int ew, int lane) {
-  const int total = min(t.count, kCap);   // pairs that found the queue full were not stored
+// A checker lane's wait for queue position `slot` of epoch ep: true once the item is there; false once the mask
+// warps closed the queue at or below the slot (that position holds nothing to check in this epoch), or after about
+// a second (the timeout is recorded; the mask warps then see the abort flag and close the queue).
+__device__ __forceinline__ bool wait_slot(Tail& t, int slot, uint32_t ep, unsigned int* dev_status) {
+  const long long t0 = clock64();
+  for (;;) {
+    if (slot < kCap && ld_volatile(&t.ready[slot]) == ep) {
+      __threadfence_block();   // the item was written before its ready stamp
+      return true;
+    }
+    if (ld_volatile(&t.closing)) {
+      __threadfence_block();   // closed_at was written before closing
+      if (slot >= (int)ld_volatile(reinterpret_cast<uint32_t*>(&t.closed_at))) return false;
+      // below closed_at: the item was queued before the close and its stamp is on the way
+    }
+    if (clock64() - t0 > kWaitCycles) {
+      st_volatile(&t.abort_flag, 1u);
+      atomicOr(dev_status, kDevTimeout);
+      return false;
+    }
+    __nanosleep(32);
+  }
+}
+
+// A checker warp's exact key scores of the queue items at base + u for the set bits u of `ready`: kItems key rows
+// in flight together, each lane's 8-element chunks in order, then a butterfly sum (every lane ends with every
+// score).
+__device__ __forceinline__ void check_items(const Tail& t, unsigned ready, int base, float (&acc)[kItems],
+                                            const __nv_bfloat16* __restrict__ keys,
+                                            const __nv_bfloat16* __restrict__ q, int d, int q0, int lane) {
   const int v = d / 8;
-  constexpr int kItems = 4;   // queue items per warp at a time: their key-row loads are in flight together
-  for (int base = ew * kItems; base < total; base += kEpiWarps * kItems) {
-    float acc[kItems];
-    const uint4* kp[kItems];
-    const uint4* xp[kItems];
+  const int first = base + __ffs(ready) - 1;
+  const uint4* kp[kItems];
+  const uint4* xp[kItems];
+#pragma unroll
+  for (int u = 0; u < kItems; ++u) {
+    const Item it = t.items[(ready >> u) & 1u ? base + u : first];
+    kp[u] = reinterpret_cast<const uint4*>(keys + (int64_t)it.j * d);
+    xp[u] = reinterpret_cast<const uint4*>(q + (int64_t)(q0 + it.q) * d);
+    acc[u] = 0.f;
+  }
+#pragma unroll 1
+  for (int c = lane; c < v; c += 32) {
+    uint4 kv[kItems], xv[kItems];
 #pragma unroll
     for (int u = 0; u < kItems; ++u) {
-      const Item it = t.items[base + u < total ? base + u : base];
-      kp[u] = reinterpret_cast<const uint4*>(keys + (int64_t)it.j * d);
-      xp[u] = reinterpret_cast<const uint4*>(q + (int64_t)(q0 + it.q) * d);
-      acc[u] = 0.f;
-    }
-#pragma unroll 1
-    for (int c = lane; c < v; c += 32) {
-      uint4 kv[kItems], xv[kItems];
-#pragma unroll
-      for (int u = 0; u < kItems; ++u) {
-        kv[u] = __ldg(kp[u] + c);
-        xv[u] = __ldg(xp[u] + c);
-      }
-#pragma unroll
-      for (int u = 0; u < kItems; ++u) acc[u] = dot8(xv[u], kv[u], acc[u]);
+      kv[u] = __ldg(kp[u] + c);
+      xv[u] = __ldg(xp[u] + c);
     }
 #pragma unroll
-    for (int u = 0; u < kItems; ++u) acc[u] = warp_sum(acc[u]);
-    if (lane == 0) {
-#pragma unroll
-      for (int u = 0; u < kItems; ++u)
-        if (base + u < total) t.score[base + u] = acc[u];
-    }
+    for (int u = 0; u < kItems; ++u) acc[u] = dot8(xv[u], kv[u], acc[u]);
   }
-  epi_sync();
-  // one thread per query of the pass takes that query's items, in queue order, into its list
-  const int qq = ew * 32 + lane;
-  if (qq < qn) {
-    float best = -INFINITY;
-    uint64_t* L = lists + (size_t)qq * C;
-    for (int i0 = 0; i0 < total; i0 += 8) {
-      uint32_t m = 0;   // this query's items among the next 8 (the loads are independent and overlap)
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
-        if (i0 + u < total && t.items[i0 + u].q == qq) m |= 1u << u;
-      while (m) {
-        const int i = i0 + __ffs(m) - 1;
-        m &= m - 1;
-        const float sc = t.score[i];
-        best = fmaxf(best, sc);
-        if (sc >= tau_c) {
-          const uint64_t x = pack_cand(sc, (uint32_t)t.items[i].j);
-          if (x > L[C - 1]) {
-            int p = C - 1;
-            while (p > 0 && L[p - 1] < x) {
-              L[p] = L[p - 1];
-              --p;
-            }
-            L[p] = x;
-          }
-        }
-      }
+  for (int u = 0; u < kItems; ++u) acc[u] = warp_sum(acc[u]);
+}
+
+// Fold one exact score into query qq's best score and, if it clears tau_c, into its top-c list (under the
+// query's lock: several checker warps fold concurrently). False after a lock timeout (recorded).
+__device__ __forceinline__ bool fold_one(Tail& t, uint64_t* lists, int C, float tau_c, int qq, int32_t j, float sc,
+                                         unsigned int* dev_status) {
+  atomicMax(&t.best[qq], score_order(sc));
+  if (!(sc >= tau_c)) return true;
+  const uint64_t x = pack_cand(sc, (uint32_t)j);
+  const long long t0 = clock64();
+  while (atomicCAS(&t.lock[qq], 0, 1) != 0) {
+    if (clock64() - t0 > kWaitCycles || ld_volatile(&t.abort_flag)) {
+      st_volatile(&t.abort_flag, 1u);
+      atomicOr(dev_status, kDevTimeout);
+      return false;
     }
-    if (best > -INFINITY) t.best[qq] = max(t.best[qq], score_order(best));
+    __nanosleep(32);
   }
+  __threadfence_block();
+  volatile uint64_t* L = lists + (size_t)qq * C;
+  if (x > L[C - 1]) {
+    int p = C - 1;
+    while (p > 0 && L[p - 1] < x) {
+      L[p] = L[p - 1];
+      --p;
+    }
+    L[p] = x;
+  }
+  __threadfence_block();
+  atomicExch(&t.lock[qq], 0);
+  return true;
+}
+
+// Run by all epilogue warps after the mask warps closed the queue: once every checker has arrived, every queued
+// pair has been checked and folded into its query's list; then the queue is emptied and reopened.
+__device__ __forceinline__ void reopen(Tail& t, int ew, int lane) {
   epi_sync();
-  if (ew == 0 && lane == 0) t.count = 0;
+  if (ew == 0 && lane == 0) {
+    t.count = 0;
+    t.claim = 0;
+    t.closing = 0;
+  }
   epi_sync();
 }
 
@@ -267,12 +306,13 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
     }
     for (int b = 0; b < G::kNbuf; ++b) {
       mbar_init(tfull_bar(b), 1);
-      mbar_init(tempty_bar(b), kEpiWarps);
+      mbar_init(tempty_bar(b), kMaskWarps);
     }
     mbar_init(drain_bar, 1);
     t.abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  for (int i = threadIdx.x; i < kCap; i += kThreads) t.ready[i] = ~0u;   // no epoch
   if (warp == kMmaWarp) {
     tmem_alloc<false>(smem_u32(&t.tmem_slot), 512);
     tmem_relinquish<false>();
@@ -299,6 +339,7 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
   uint32_t it = 0;        // blocks so far, over all passes (every role counts the same blocks)
   uint32_t tb = 0;        // accumulator uses so far
   uint32_t issued = 0;    // loader: copies issued, blocks 0 .. issued - 1
+  uint32_t ep = 0;        // epilogue: reopenings so far (the epoch of the queue's ready stamps)
 
   for (int q0 = 0; q0 < a.B; q0 += G::kQC) {
     const int qn = min(G::kQC, a.B - q0);
@@ -322,8 +363,16 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
       }
       asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
       for (int i = et; i < G::kQC * C; i += kEpiWarps * 32) lists[i] = 0;
-      for (int i = et; i < G::kQC; i += kEpiWarps * 32) t.best[i] = score_order(-INFINITY);
-      if (et == 0) t.count = 0;
+      for (int i = et; i < G::kQC; i += kEpiWarps * 32) {
+        t.best[i] = score_order(-INFINITY);
+        t.lock[i] = 0;
+      }
+      if (et == 0) {
+        t.count = 0;
+        t.claim = 0;
+        t.closing = 0;
+        t.pass_end = 0;
+      }
     }
     __syncthreads();
 
@@ -383,22 +432,33 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
       __syncwarp();
       tb = __shfl_sync(kFull, tb, 0);
       it += (uint32_t)nb;
-    } else {
-      // ---------------- epilogue ----------------
-      const int ew = warp;                                 // epilogue warp
-      const int quad = ew % 4, group = ew / 4;             // TMEM lane quadrant; column chunks c % 4 == group
+    } else if (warp < kMaskWarps) {
+      // ---------------- mask warps ----------------
+      const int mw = warp;                                 // mask warp
+      const int quad = mw % 4, group = mw / 4;             // TMEM lane quadrant; column chunks c % kMaskGroups == group
       const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+      // close the queue (every mask warp has queued its pairs); reopen it once the checkers are done with it
+      auto close_and_reopen = [&](bool last) {
+        if (mw == 0 && lane == 0) {
+          t.closed_at = min(t.count, kCap);
+          if (last) t.pass_end = 1;
+          __threadfence_block();
+          st_volatile(&t.closing, 1u);
+        }
+        reopen(t, mw, lane);
+        ++ep;
+      };
       bool stop = false;
       for (int64_t t0 = 0; t0 < nb && !stop; t0 += kRound) {
         // the admitted queries of this thread's entry in each block of the round, as bit masks over the warp's
-        // column chunks (chunk group + kEpiGroups u)
+        // column chunks (chunk group + kMaskGroups u)
         uint32_t pend[kRound][kPer];
         bool got = true;
 #pragma unroll
         for (int r = 0; r < kRound; ++r) {
 #pragma unroll
           for (int u = 0; u < kPer; ++u) pend[r][u] = 0;
-          if (t0 + r >= nb || !got) continue;              // the same for every epilogue warp
+          if (t0 + r >= nb || !got) continue;              // the same for every mask warp
           const int b = tb % G::kNbuf;
           const uint32_t tph = (tb / G::kNbuf) & 1u;
           ++tb;
@@ -407,7 +467,7 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
           tc_fence_after();
 #pragma unroll
           for (int u = 0; u < kPer; ++u) {
-            const int c = group + kEpiGroups * u;
+            const int c = group + kMaskGroups * u;
             if (c < G::kQC / 32 && 32 * c < npad) {   // the same for the whole warp
               float v[32];
               tmem_ld32(tmem + lane_addr + (uint32_t)(b * G::kQC) + 32u * c, v);
@@ -432,8 +492,9 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
           __syncwarp();
           if (lane == 0) mbar_arrive(tempty_bar(b));
         }
-        // queue the admitted pairs; flush while the queue is past kFlushAt or a pair found it full (every round
-        // either queues all pending pairs or fills the queue, so this ends). All epilogue warps leave together.
+        // queue the admitted pairs, each with its epoch stamp, for the checker warps; close while the queue is
+        // past kFlushAt or a pair found it full (every round either queues all pending pairs or fills the queue,
+        // so this ends). All mask warps leave together.
         int top = -1;
         for (;;) {
           bool left = false;
@@ -450,7 +511,9 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
                 p &= p - 1;
                 const int slot = atomicAdd(&t.count, 1);
                 if (slot < kCap) {
-                  t.items[slot] = Item{(int32_t)j, 32 * (group + kEpiGroups * u) + bit};
+                  t.items[slot] = Item{(int32_t)j, 32 * (group + kMaskGroups * u) + bit};
+                  __threadfence_block();
+                  st_volatile(&t.ready[slot], ep);
                   top = slot;
                 } else {
                   full |= 1u << bit;
@@ -460,15 +523,46 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
               left |= full != 0;
             }
           }
-          if (!epi_any(!got || *abort_flag || left || top >= kFlushAt)) break;
-          if (epi_any(!got || *abort_flag)) {
+          if (!mask_any(!got || *abort_flag || left || top >= kFlushAt)) break;
+          if (mask_any(!got || *abort_flag)) {
             if (!got) fail();
             stop = true;
             break;
           }
-          flush(t, lists, a.keys, a.q, a.d, a.tau_c, C, q0, qn, ew, lane);
+          close_and_reopen(false);
           top = -1;
         }
+      }
+      // the pass's last close, also after a timeout: the checker warps leave only at a reopening
+      close_and_reopen(true);
+      it += (uint32_t)nb;
+    } else {
+      // ---------------- checker warps ----------------
+      // claim kItems queue positions at a time, check and fold their pairs while the scan goes on; at a close,
+      // finish what was queued below it, then take part in the reopening
+      for (;;) {
+        for (;;) {
+          int base = 0;
+          if (lane == 0) base = atomicAdd(&t.claim, kItems);
+          base = __shfl_sync(kFull, base, 0);
+          const bool mine = lane < kItems && wait_slot(t, base + lane, ep, a.dev_status);
+          const unsigned ready = __ballot_sync(kFull, mine);
+          if (ready) {
+            float acc[kItems];
+            check_items(t, ready, base, acc, a.keys, a.q, a.d, q0, lane);
+            if (lane == 0) {
+#pragma unroll
+              for (int u = 0; u < kItems; ++u)
+                if ((ready >> u) & 1u)
+                  fold_one(t, lists, C, a.tau_c, t.items[base + u].q, t.items[base + u].j, acc[u], a.dev_status);
+            }
+            __syncwarp();
+          }
+          if (ready != (1u << kItems) - 1u) break;   // a position past the close (or a timeout)
+        }
+        reopen(t, warp, lane);
+        ++ep;
+        if (ld_volatile(&t.pass_end)) break;
       }
       it += (uint32_t)nb;
     }
@@ -476,7 +570,6 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
     // ---- pass end: every role is here; a timeout anywhere stops them all together ----
     if (__syncthreads_or(*abort_flag != 0)) break;
     if (warp < kEpiWarps) {
-      flush(t, lists, a.keys, a.q, a.d, a.tau_c, C, q0, qn, warp, lane);
       const int et = threadIdx.x;
       for (int i = et; i < qn * C; i += kEpiWarps * 32) {
         const int qq = i / C;
