@@ -61,7 +61,18 @@ def _expected_lsh_kernel(batch):
                          ids=["popcount-5", "popcount-32", "popcount-36", "tensor-40", "tensor-64", "tensor-200"])
 @pytest.mark.parametrize("bits", [128, 256, 512])
 def test_lsh_lookup_matches_the_oracle(bits, batch):
-    w = wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch)
+    _check_lsh_lookup(wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch), bits)
+
+
+@pytest.mark.parametrize("top_c", [1, 32])
+@pytest.mark.parametrize("batch", [16, 64], ids=["popcount", "tensor"])
+def test_lsh_top_c_extremes_match_the_oracle(batch, top_c):
+    # one candidate per query (every list insertion replaces the head) and the longest lists the kernels hold
+    _check_lsh_lookup(wl.WORKLOADS["mid-1m"].scaled(n=40_000, batch=batch, top_c=top_c), 256)
+
+
+def _check_lsh_lookup(w, bits):
+    batch = w.batch
     radius = wl.lsh_radius(w.tau_c, bits)
     R = wl.hyperplanes(bits, w.d, device="cuda")
     st = oracle_store(w)
@@ -77,7 +88,8 @@ def test_lsh_lookup_matches_the_oracle(bits, batch):
     keep = np.nonzero(~amb)[0]
     sub = oracle.Result(**{f: getattr(res, f)[keep] for f in res.__dataclass_fields__})
     rep = compare(g, sub, p, rows=keep)
-    log_report(f"lsh bits={bits} B={batch} radius={radius} ({w.batch - len(keep)} queries with ambiguous bits)", rep)
+    amb_n = w.batch - len(keep)
+    log_report(f"lsh bits={bits} B={batch} c={w.top_c} radius={radius} ({amb_n} queries with ambiguous bits)", rep)
     # queries with a signature bit within the fp32/fp64 ambiguity of zero are set aside: at most 1 in 50
     assert rep.exact + rep.band == len(keep) and len(keep) >= w.batch - max(2, w.batch // 50)
     if batch >= 16:
