@@ -121,3 +121,15 @@ def test_load_rejects_what_is_not_a_saved_cache_before_touching_a_device(lib, tm
     assert lib.lacache_load(str(short).encode(), 0, 0, ctypes.byref(h)) == lacache.LACACHE_ERR_IO
     assert lib.lacache_load(str(short).encode(), 0, -1, ctypes.byref(h)) == lacache.LACACHE_ERR_INVALID_ARG
     assert lib.lacache_save(None, b"x") == lacache.LACACHE_ERR_INVALID_ARG
+
+
+def test_a_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path):
+    # the product path has no CPU route: without liblacache.so every binding call fails loudly
+    monkeypatch.setattr(lacache, "LIB_PATH", str(tmp_path / "liblacache.so"))
+    monkeypatch.setattr(lacache, "_lib", None)
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        lacache.load()
+    with pytest.raises(RuntimeError, match="is missing"):
+        lacache.lacache_create(lacache.make_config(64, 8, 1024, 0.9, 0.8, 8, max_batch=16))
+    with pytest.raises(RuntimeError, match="is missing"):
+        lacache.status_string(lacache.LACACHE_OK)
