@@ -22,9 +22,10 @@ Readings where the paper leaves the batched form open:
   h(f_k(x')) = h(f_k(x)) under an identity hash on ids. BOTH: both.
 
 Beside the decision the oracle emits two margins per query. The decision margin is the smallest distance by which
-some score would have to move to change the status or the served entry. The list margin is the same for the
-candidate list and its order. A fp32 implementation may legitimately differ from this fp64 one only where the
-corresponding margin is small.
+some score would have to move to change the status or the served entry: while every key and prefix score moves by
+less than half of it, the decision stays as it is. The list margin is the same for the candidate list and its
+order. A fp32 implementation may legitimately differ from this fp64 one only where the corresponding margin is
+small.
 """
 from __future__ import annotations
 
@@ -112,8 +113,8 @@ class KeyCheck:
 
     s_qj = <q, K_j> for every valid entry j, in fp64 from the exact bf16 values. A_q = {j : s_qj >= tau_c} is
     the union of the blocks' contributions, so the blocks can come from anywhere: a resident array, or chunks
-    regenerated one at a time for a cache larger than host memory. Alongside A_q it keeps max_j s_qj and
-    min_j |s_qj - tau_c|, which the margin needs.
+    regenerated one at a time for a cache larger than host memory. Alongside A_q it keeps max_j s_qj,
+    min_j |s_qj - tau_c| and the best score below tau_c, which the margin needs.
     """
 
     def __init__(self, q_bits, tau_c: float):
@@ -124,6 +125,7 @@ class KeyCheck:
         self._j = [[] for _ in range(B)]
         self.best = np.full(B, -np.inf)
         self.closest = np.full(B, np.inf)
+        self.below = np.full(B, -np.inf)
         self.rows = 0
 
     def add_rows(self, key_bits, j0: int) -> None:
@@ -145,6 +147,7 @@ class KeyCheck:
                 self._j[b].append(sel.astype(np.int64) + j0)
         self.best = np.maximum(self.best, np.where(ok, s, -np.inf).max(axis=1))
         self.closest = np.minimum(self.closest, np.where(ok, np.abs(s - self.tau_c), np.inf).min(axis=1))
+        self.below = np.maximum(self.below, np.where(ok & (s < self.tau_c), s, -np.inf).max(axis=1))
         self.rows += s.shape[1]
 
     def above(self, b: int):
@@ -248,34 +251,52 @@ def decide(kc: KeyCheck, q_prefix_bits, q_ids, params: Params,
             res.prefix_score[b] = r[shown]
             res.prefix_scores[b] = rm[shown]
             res.token_matches[b] = m[shown]
-        next_ok = False
         if n_above > c:
-            # the best entry just outside C_q: only needed to know whether the cut can change the decision
-            jn = j_sorted[c:c + 1]
-            rn, mn = lookahead(q_prefix_bits[b], q_ids[b], prefix_rows(jn), id_rows(jn), segs)
-            next_ok = bool(passes(rn, mn, params, k, segs)[0])
-            res.next_id[b], res.next_score[b] = jn[0], s_sorted[c]
+            res.next_id[b], res.next_score[b] = j_sorted[c], s_sorted[c]   # the best entry just outside C_q
 
-        # decision margin: the smallest score change that alters status or entry_id
+        # decision margin: the smallest score change that alters status or entry_id. A gap between two scores
+        # closes when each moves by half of it, so the decision holds while every score moves by less than
+        # half the margin.
+        taus = [t for _, _, t in segs] if segs else [tau_a]
+
+        def flip(r_row, m_val):
+            # the smallest prefix-score change that flips a pass bit (none where the token ids decide it)
+            if uses_r and (not uses_m or m_val >= tmin):
+                return min(abs(r_row[h] - taus[h]) for h in range(len(taus)))
+            return np.inf
+
         gaps = []
         if nc:
-            taus = [t for _, _, t in segs] if segs else [tau_a]
             for i in range((served if served is not None else nc - 1) + 1):   # candidates examined
-                if uses_r and (not uses_m or m[i] >= tmin):
-                    gaps.append(min(abs(rm[i, h] - taus[h]) for h in range(len(taus))))
+                gaps.append(flip(rm[i], m[i]))
         if served is not None:
             gaps.append(cs[served] - tau_c)                         # j* falls out of A_q
-            if served == c - 1 and n_above > c:
-                gaps.append(cs[served] - s_sorted[c])               # j* pushed past the cut
+            if n_above > c:
+                # j* pushed past the cut: every entry ranked below it down to the one at the cut rises above it.
+                # This also covers any single entry from past the cut overtaking j*.
+                gaps.append(cs[served] - s_sorted[c])
             for i in range(nc):
                 if i != served and ok[i]:
                     gaps.append(abs(cs[served] - cs[i]))            # another passing candidate overtakes j*
+                elif i > served:                                    # a later failing one overtakes j* and passes
+                    gaps.append(max(cs[served] - cs[i], flip(rm[i], m[i])))
         elif n_above < c:
             gaps.append(kc.closest[b])                              # any entry entering or leaving A_q
         else:
             gaps.append(cs[0] - tau_c)                              # every candidate leaving A_q
-            if n_above > c and next_ok:
-                gaps.append(cs[-1] - s_sorted[c])                   # a passing entry entering C_q
+            gaps.append(cs[-1] - kc.below[b])                       # an entry from below tau_c entering C_q
+            # entries past the cut rising above the last candidate: a passing one is served, a failing one only
+            # if its pass bit flips too. Those farther below than the smallest gap so far cannot matter.
+            bound = min(gaps)
+            past = [i for i in range(c, n_above) if cs[-1] - s_sorted[i] < bound]
+            if past:
+                je = j_sorted[past]
+                re, me = lookahead(q_prefix_bits[b], q_ids[b], prefix_rows(je), id_rows(je), segs)
+                oke = passes(re, me, params, k, segs)
+                rme = re if segs else re[:, None]
+                for t, i in enumerate(past):
+                    key = cs[-1] - s_sorted[i]
+                    gaps.append(key if oke[t] else max(key, flip(rme[t], me[t])))
         res.margin[b] = min(gaps) if gaps else np.inf
 
         # candidate-list margin: the smallest score change that alters C_q or its order

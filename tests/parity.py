@@ -206,8 +206,10 @@ class StreamedOracle:
     """The oracle for caches too large for host memory: the store streams through it chunk by chunk.
 
     Each generated chunk is inserted into the GPU cache and its key bytes go through the oracle's block-wise key
-    check (A_q is a union over blocks). The prefix rows and ids of the entries stage 2 needs are then regenerated
-    from the generator, never read back from the device.
+    check (A_q is a union over blocks). The prefix rows and ids of the entries stage 2 and the decision margin
+    may need (every entry of each A_q: the margin of a rejection looks past the candidate cut) are then
+    regenerated from the generator, never read back from the device. With no cache the store is generated on
+    `device` only for the oracle.
     """
 
     def __init__(self, w: wl.Workload, q: dict, sample, p: oracle.Params):
@@ -215,24 +217,26 @@ class StreamedOracle:
         self.sample = np.asarray(sample)
         self.oq = oracle_queries(q, torch.as_tensor(self.sample))
         self.kc = oracle.KeyCheck(self.oq["emb"], p.tau_c)
+        self.device = "cuda"
 
     def fill(self, cache: L.LaCache | None, device="cuda") -> None:
+        self.device = device
         dtype = L.LACACHE_F32 if self.w.key_dtype == "f32" else L.LACACHE_BF16
         for ch in wl.iter_store(self.w, device):
             if cache is not None:
                 cache.insert(ch["key"], ch["prefix"], ch["ids"], dtype)
             self.kc.add_rows(_bits(ch["key"], self.w.key_dtype == "f32"), ch["j0"])
             del ch
-        torch.cuda.synchronize()
+        if device != "cpu":
+            torch.cuda.synchronize()
 
     def result(self) -> oracle.Result:
-        c = self.p.top_c
         need = set()
         for b in range(len(self.sample)):
             _, j = self.kc.above(b)
-            need.update(int(x) for x in j[:c + 1])
+            need.update(int(x) for x in j)
         ids = np.array(sorted(need), dtype=np.int64)
-        rows = wl.store_rows(self.w, torch.as_tensor(ids), "cuda")
+        rows = wl.store_rows(self.w, torch.as_tensor(ids), self.device)
         f32 = self.w.key_dtype == "f32"
         pre = _bits(rows["prefix"], f32)
         tok = rows["ids"].cpu().numpy()
@@ -242,7 +246,7 @@ class StreamedOracle:
                              lambda js: tok[[where[int(j)] for j in js]])
 
     def pair_scores(self, b, j):
-        row = wl.store_rows(self.w, torch.as_tensor([j]), "cuda")
+        row = wl.store_rows(self.w, torch.as_tensor([j]), self.device)
         f32 = self.w.key_dtype == "f32"
         kc = oracle.KeyCheck(self.oq["emb"][b:b + 1], -np.inf)
         kc.add_rows(_bits(row["key"], f32), j)

@@ -46,6 +46,19 @@ MUTATIONS = [
      "res.prefix_score[b] = r[0]", PINS),
     ("margin-drops-threshold-gap", "lookup.py", "gaps.append(cs[served] - tau_c)",
      "gaps.append(np.inf)", PINS),
+    ("margin-push-out-only-from-the-last-slot", "lookup.py",
+     "            if n_above > c:\n                # j* pushed past the cut",
+     "            if n_above > c and served == c - 1:\n                # j* pushed past the cut", PINS),
+    ("margin-ignores-later-failing-candidates", "lookup.py",
+     "gaps.append(max(cs[served] - cs[i], flip(rm[i], m[i])))", "pass", PINS),
+    ("margin-ignores-entries-below-threshold", "lookup.py", "gaps.append(cs[-1] - kc.below[b])",
+     "gaps.append(np.inf)", PINS),
+    ("margin-ignores-entries-past-the-cut", "lookup.py",
+     "gaps.append(key if oke[t] else max(key, flip(rme[t], me[t])))", "pass", PINS),
+    ("margin-past-the-cut-all-passing", "lookup.py",
+     "gaps.append(key if oke[t] else max(key, flip(rme[t], me[t])))", "gaps.append(key)", PINS),
+    ("below-threshold-best-of-all-scores", "lookup.py", "np.where(ok & (s < self.tau_c), s, -np.inf)",
+     "np.where(ok, s, -np.inf)", PINS),
     ("ensemble-any-model-passes", "lookup.py", "emb_ok = np.all(r >= np.array(", "emb_ok = np.any(r >= np.array(",
      ENS),
     ("ensemble-thresholds-reversed", "lookup.py", "np.array([t for _, _, t in segments])[None, :]",

@@ -251,6 +251,88 @@ def test_margin_terms():
     assert r.status[0] == HIT and r.margin[0] == 1.0 - 0.984375
 
 
+def test_margin_counts_changes_from_outside_the_examined_candidates():
+    q = np.array([1.0, 0, 0, 0])
+    # a passing entry just past the cut could rise above the served entry and be served instead
+    keys = [E[0], [0.99609375, 0, 0, 0], [0.9921875, 0, 0, 0]]
+    st = store_of(keys, [E[1], E[2], E[1]], [[0]] * 3)
+    r = oracle.lookup(st, queries_of(q, E[1], [0]), Params(0.5, 0.5, 2))
+    assert r.status[0] == HIT and r.entry_id[0] == 0 and r.margin[0] == 1.0 - 0.9921875
+    # a failing candidate after the served one, 2^-8 below it in key score and 2^-8 short of tau_a
+    st = store_of(keys[:2], [E[1], [0, 0.49609375, 0, 0]], [[0]] * 2)
+    r = oracle.lookup(st, queries_of(q, E[1], [0]), Params(0.5, 0.5, 2))
+    assert r.status[0] == HIT and r.entry_id[0] == 0 and r.margin[0] == 0.5 - 0.49609375
+    # a full candidate list rejected, and a passing entry 2^-8 below tau_c that could overtake the last candidate
+    keys = [E[0], [0.50390625, 0, 0, 0], [0.49609375, 0, 0, 0]]
+    st = store_of(keys, [E[2], E[2], E[1]], [[0]] * 3)
+    r = oracle.lookup(st, queries_of(q, E[1], [0]), Params(0.5, 0.5, 2))
+    assert r.status[0] == REJECT and r.margin[0] == 0.50390625 - 0.49609375
+    # rejected, the entry at the cut fails, and the one after it passes
+    keys = [E[0], [0.99609375, 0, 0, 0], [0.9921875, 0, 0, 0]]
+    st = store_of(keys, [E[2], E[2], E[1]], [[0]] * 3)
+    r = oracle.lookup(st, queries_of(q, E[1], [0]), Params(0.5, 0.5, 1))
+    assert r.status[0] == REJECT and r.margin[0] == 1.0 - 0.9921875
+
+
+def _decision_from_scores(s, r, m, tau_c, taus, c, mode, tmin):
+    """Algorithm 1's decision for one query from its key scores s[j], prefix scores r[j][h] and token matches m[j]."""
+    above = sorted((j for j in range(len(s)) if s[j] >= tau_c), key=lambda j: (-s[j], j))
+    for j in above[:c]:
+        emb = all(r[j][h] >= taus[h] for h in range(len(taus)))
+        tok = m[j] >= tmin
+        if (emb if mode == CHECK_EMB else tok if mode == CHECK_TOKENS else emb and tok):
+            return HIT, j
+    return (REJECT if above else MISS_KEY), -1
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_decision_survives_every_score_change_below_half_the_margin(seed):
+    """The margin's defining property: moving every key and prefix score by less than half the decision margin
+    (so that no gap between two scores closes) leaves the status and the served entry unchanged. Scores sit on a
+    2^-8 grid around the thresholds, so ties, near ties and entries on both sides of the cut are common."""
+    rng = np.random.default_rng(1000 + seed)
+    step, tau_c = 2.0 ** -8, 0.75
+    models = 2 if seed % 4 == 3 else 1
+    taus = [0.625, 0.5625][:models]
+    mode = [CHECK_EMB, CHECK_EMB, CHECK_TOKENS, CHECK_BOTH][seed % 4] if models == 1 else CHECK_EMB
+    for _ in range(25):
+        n, c, kt = int(rng.integers(1, 11)), int(rng.integers(1, 5)), 3
+        s = tau_c + step * rng.integers(-12, 13, size=n)
+        s[rng.random(n) < 0.15] = 0.5
+        rv = np.array(taus)[None, :] + step * rng.integers(-12, 13, size=(n, models))
+        keys = np.zeros((n, 4))
+        keys[:, 0] = s
+        pre = np.zeros((n, 2 * models))
+        pre[:, 0::2] = rv
+        ids = rng.integers(0, 2, size=(n, kt))
+        qi = rng.integers(0, 2, size=kt)
+        tmin = int(rng.integers(1, kt + 1))
+        qp = np.tile([1.0, 0.0], models)
+        p = Params(tau_c, taus[0], c, check_mode=mode, token_match_min=tmin,
+                   prefix_dims=(2,) * models if models > 1 else None,
+                   tau_a_models=tuple(taus) if models > 1 else None)
+        res = oracle.lookup(store_of(keys, pre, ids), queries_of(E[0], qp, qi), p)
+        m = (ids == qi[None, :]).sum(axis=1)
+        got = (int(res.status[0]), int(res.entry_id[0]))
+        assert _decision_from_scores(s, rv, m, tau_c, taus, c, mode, tmin) == got
+        mu = float(res.margin[0])
+        if mu == 0.0:
+            continue
+        delta = 0.49 * min(mu, 1.0)
+        moves = [(rng.uniform(-delta, delta, n), rng.uniform(-delta, delta, (n, models))) for _ in range(60)]
+        moves += [(delta * rng.choice([-1.0, 1.0], n), delta * rng.choice([-1.0, 1.0], (n, models)))
+                  for _ in range(60)]
+        for e in range(n):                 # one entry moves one way, every other entry the other way
+            for ss in (-1.0, 1.0):
+                for sr in (-1.0, 1.0):
+                    ds, dr = np.full(n, -ss * delta), np.full((n, models), -sr * delta)
+                    ds[e], dr[e] = ss * delta, sr * delta
+                    moves.append((ds, dr))
+        for ds, dr in moves:
+            assert _decision_from_scores(s + ds, rv + dr, m, tau_c, taus, c, mode, tmin) == got, \
+                f"margin {mu}: scores {s}, prefix scores {rv.tolist()}, c {c}, moved by {ds}, {dr.tolist()}"
+
+
 # --- brute force in exact arithmetic on tiny inputs ---------------------------------------------------------------
 
 def _brute(keys_b, pre_b, ids, q_b, p_b, t, tau_c, tau_a, c):
