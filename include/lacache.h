@@ -283,8 +283,11 @@ lacache_status lacache_inject_stall(lacache_t* h, int32_t lookups);
  * (16-byte aligned), ids_dev [n x k] int32. Queries and outputs are as for lacache_lookup. From *cfg it uses
  * d, k, tau_c, tau_a, top_c, token_match_min, check_mode, device and stage1; capacity and max_batch are ignored.
  * The stage-1 scratch lives in an 8 MiB file-scope device array of the library, which every GPU that loads the
- * library holds until the process exits. A batch needs B * (8 * top_c + 4) bytes of it; larger batches return
- * LACACHE_ERR_UNSUPPORTED and nothing runs. The first call on a device does a one-time set-up (it looks up the
+ * library holds until the process exits. 512 bytes of it hold a status word and alignment padding, so a batch
+ * fits only if B * (8 * top_c + 4) <= 8 MiB - 512 bytes (for top_c = 32, B <= 32261); larger batches return
+ * LACACHE_ERR_UNSUPPORTED and nothing runs. stage1 = LACACHE_STAGE1_AUTO runs the tensor-core scan, or the CUDA-core
+ * scan if the driver offers no TMA descriptor encoder; an explicit LACACHE_STAGE1_TENSOR then gives
+ * LACACHE_ERR_CUDA. The first call on a device does a one-time set-up (it looks up the
  * array's device address), so make that first call before any stream capture. All calls on a device share the
  * array: calls that overlap on the GPU (other streams, other host threads) race and give undefined results, so
  * issue them on one stream. A device-side timeout is not reported by this entry point (its outputs are then

@@ -35,6 +35,7 @@ constexpr unsigned int kDevTimeout = 1u;
 // Candidate keys. A stage-1 candidate (score s, entry id j) is packed into one uint64 whose unsigned order is the
 // candidate order of the lookup: higher score first, then lower entry id. The high word is the score's bits mapped
 // to an unsigned order; the low word is ~j. The value 0 is never produced by a finite score and marks "empty".
+// -0.0 and +0.0 are equal scores, so both map to the order of +0.0: equal scores then fall to the id rule.
 // ---------------------------------------------------------------------------------------------------------------
 __host__ __device__ __forceinline__ uint32_t score_order(float s) {
   uint32_t u;
@@ -43,6 +44,7 @@ __host__ __device__ __forceinline__ uint32_t score_order(float s) {
 #else
   memcpy(&u, &s, 4);
 #endif
+  if (u == 0x80000000u) u = 0u;
   return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
 

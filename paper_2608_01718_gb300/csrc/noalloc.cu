@@ -30,14 +30,15 @@ struct DeviceSetup {
   bool ready;
   unsigned char* scratch;   // device address of g_noalloc_scratch on this device
   int num_sms;
+  lc::EncodeTiledFn encode; // TMA descriptor encoder (nullptr if the driver does not provide it)
 };
 
 std::mutex g_setup_mutex;
 DeviceSetup g_setup[kMaxDevices];
-lc::EncodeTiledFn g_encode = nullptr;
 
 // One-time set-up for `dev`, which must be the current device: the device address of the scratch array, the SM
-// count, and the TMA descriptor encoder. Nothing here allocates.
+// count, and the TMA descriptor encoder. Every field is written and read under the lock, and the caller gets its
+// own copy. Nothing here allocates.
 lacache_status setup_device(int dev, DeviceSetup* out) {
   std::lock_guard<std::mutex> lock(g_setup_mutex);
   DeviceSetup& s = g_setup[dev];
@@ -46,14 +47,14 @@ lacache_status setup_device(int dev, DeviceSetup* out) {
     if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess) return LACACHE_ERR_CUDA;
     int sms = 0;
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return LACACHE_ERR_CUDA;
-    if (!g_encode) {
-      void* fn = nullptr;
-      cudaDriverEntryPointQueryResult q;
-      if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
-              cudaSuccess &&
-          q == cudaDriverEntryPointSuccess)
-        g_encode = reinterpret_cast<lc::EncodeTiledFn>(fn);
-    }
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      s.encode = reinterpret_cast<lc::EncodeTiledFn>(fn);
+    else
+      cudaGetLastError();
     s.scratch = static_cast<unsigned char*>(ptr);
     s.num_sms = sms;
     s.ready = true;
@@ -126,10 +127,13 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
       a.part_cand = part_cand;
       a.part_best = part_best;
       a.dev_status = status;
-      const int kernel = c.stage1 == LACACHE_STAGE1_AUTO ? LACACHE_STAGE1_TENSOR : c.stage1;
+      // AUTO takes the tensor-core scan, or the CUDA-core scan where the driver gives no TMA descriptor encoder;
+      // an explicit TENSOR request without the encoder is an error
+      int kernel = c.stage1 == LACACHE_STAGE1_AUTO ? LACACHE_STAGE1_TENSOR : c.stage1;
+      if (c.stage1 == LACACHE_STAGE1_AUTO && !s.encode) kernel = LACACHE_STAGE1_SIMT;
       cudaError_t e;
       if (kernel == LACACHE_STAGE1_TENSOR) {
-        e = g_encode ? lc::launch_stage1_tensor(a, g_encode, s.num_sms, max_splits, st, &splits)
+        e = s.encode ? lc::launch_stage1_tensor(a, s.encode, s.num_sms, max_splits, st, &splits)
                      : cudaErrorInvalidValue;
       } else {
         e = lc::launch_stage1_simt(a, s.num_sms, max_splits, st, &splits);

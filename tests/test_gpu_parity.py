@@ -178,6 +178,30 @@ def test_hand_built_duplicates_thresholds_and_order(stage1):
 
 
 @pytest.mark.parametrize("stage1", PATHS)
+@pytest.mark.parametrize("tau_c", [0.0, -0.25])
+def test_signed_zero_scores_tie_by_id(stage1, tau_c):
+    """Scores of +0.0 and -0.0 are equal: at a key threshold <= 0 every entry below is a candidate, and the tie
+    goes to the lower id whatever the zero's sign. Even entries are all +0.0, odd ones all -0.0, so every product
+    of a query with an odd entry is a negative zero."""
+    d, n = 64, 12
+    keys = np.zeros((n, d))
+    keys[1::2] = -0.0
+    pres = np.tile(np.eye(d)[1], (n, 1))
+    ids = np.zeros((n, 2), np.int32)
+    e = np.eye(d)
+    qs = np.stack([e[0], -e[0], e[3]])
+    with L.LaCache(d, 2, 16, tau_c, -1.0, 4, max_batch=8, stage1=stage1) as c:
+        c.insert(_dev(keys), _dev(pres), torch.tensor(ids, device="cuda"))
+        out = c.lookup(_dev(qs), _dev(qs), torch.zeros((3, 2), dtype=torch.int32, device="cuda"))
+        torch.cuda.synchronize()
+        g = {k: v.cpu().numpy() for k, v in out.items()}
+    for b in range(3):
+        assert list(g["cand_id"][b]) == [0, 1, 2, 3], (b, g["cand_id"][b])
+        assert np.all(g["cand_score"][b] == 0.0) and g["n_cand"][b] == 4
+        assert g["status"][b] == L.LACACHE_HIT and g["entry_id"][b] == 0
+
+
+@pytest.mark.parametrize("stage1", PATHS)
 def test_empty_cache_is_all_key_misses(stage1):
     with L.LaCache(64, 4, 128, 0.9, 0.8, 4, max_batch=8, stage1=stage1) as c:
         q = _dev(np.eye(64)[:3])
