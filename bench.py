@@ -1,15 +1,20 @@
 #!/usr/bin/env python3
 """Throughput of the LaCache two-stage lookahead lookup on GB300.
 
-    python bench.py [--gpus N --steps K --warmup W] [--workload mid-1m] [--stage1 auto|tensor|simt]
+    python bench.py [--gpus N --steps K --warmup W] [--workload large-16m] [--stage1 auto|tensor|simt]
     python bench.py --impl reference ...        # the fp64 oracle on the host cores, a bounded sample per step
 
 A step is one lookup: stage 1 (key check with fused threshold + top-c) and stage 2 (merge, lookahead check,
-decision) for one batch of B synthetic queries against a resident cache of N entries. The inputs are resident in
-HBM before timing starts. The key store is 1.6 GB for the default workload, larger than L2, so no L2 flush is
-needed between steps. The device time is taken with CUDA events on the launching stream, between barriers, as
-the max over ranks. With N > 1 GPUs (torchrun), every rank serves its own replica of the cache with its own
-query stream: the units are independent lookups, with no collective on the data path (weak scaling).
+decision) for one batch of B synthetic queries against a resident cache of N entries. The default workload is the
+largest single-GPU one: 16,777,216 entries of d = 1024 (34.4 GB of keys, 69.8 GB of store) and batches of 128
+queries. The inputs are resident in HBM before timing starts. Every step reads the whole key store, far larger
+than L2, so no L2 flush is needed between steps. The device time is taken with CUDA events on the launching
+stream, between barriers, as the max over ranks.
+
+With N > 1 GPUs, one process runs per GPU. Under torchrun (WORLD_SIZE set) this script is one of the ranks;
+otherwise `--gpus N` builds the library once and starts N ranks through torch.distributed.run itself. Every rank
+serves its own replica of the cache with its own query stream: the units are independent lookups, with no
+collective on the data path (weak scaling). `--mode shard` splits the store by entry range instead.
 
 Rank 0 prints one JSON line.
 """
@@ -42,7 +47,7 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="mid-1m")
+    ap.add_argument("--workload", default="large-16m")
     ap.add_argument("--stage1", choices=["auto", "tensor", "simt", "lsh"], default="auto")
     ap.add_argument("--lsh-bits", type=int, default=256, help="SimHash signature bits for --stage1 lsh")
     ap.add_argument("--batches", type=int, default=8, help="distinct query batches cycled through")
@@ -60,6 +65,37 @@ def parse_args():
 def rank_info():
     return (int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)),
             int(os.environ.get("WORLD_SIZE", 1)))
+
+
+def launch_ranks(n: int, argv: list[str]) -> int:
+    """Run this script on n ranks of this node, one process per GPU, through torch.distributed.run. The ranks
+    inherit stdout, so rank 0's JSON line is this process's output."""
+    import socket
+    with socket.socket() as sock:
+        sock.bind(("127.0.0.1", 0))
+        port = sock.getsockname()[1]
+    cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={n}",
+           "--master-addr", "127.0.0.1", "--master-port", str(port), os.path.abspath(__file__), *argv]
+    return subprocess.call(cmd)
+
+
+def read_peak_gbs() -> float:
+    """A read-only streaming rate of this GPU's HBM: the best of five CUDA-event-timed torch.sum reductions over a
+    4 GiB fp32 buffer. The peaks file's HBM figure is a copy, which reads and writes; a scan only reads."""
+    import torch
+    x = torch.ones(1 << 30, dtype=torch.float32, device="cuda")
+    best = float("inf")
+    for i in range(6):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        x.sum()
+        e1.record()
+        torch.cuda.synchronize()
+        if i:
+            best = min(best, e0.elapsed_time(e1))
+    del x
+    torch.cuda.empty_cache()
+    return (1 << 32) / (best / 1e3) / 1e9
 
 
 def load_peaks():
@@ -442,6 +478,11 @@ def run_ours(args, w):
         roof = {"bound": "tensor", "achieved": flops / t1_avg_s / 1e12, "peak": peak, "unit": "TFLOP/s",
                 "peak_source": f"{peak_src} ({'sustained' if sustained else 'burst'} bf16 dense)"}
     roof["frac"] = roof["achieved"] / roof["peak"]
+    if roof["bound"] == "hbm":
+        # secondary: the same bytes against a read-only streaming rate measured here (a scan only reads)
+        rp = read_peak_gbs()
+        roof |= {"read_peak_gbs": rp, "frac_of_read_peak": roof["achieved"] / rp,
+                 "read_peak_source": "measured live: best of 5 torch.sum over a 4 GiB fp32 buffer, CUDA events"}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
@@ -706,6 +747,12 @@ def run_calibration(args):
 
 def main():
     args = parse_args()
+    if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
+        # one process per GPU: build once here, so the ranks find the library up to date, then start them
+        if args.impl == "ours":
+            from paper_2608_01718_gb300 import build
+            build.build()
+        return launch_ranks(args.gpus, sys.argv[1:])
     from paper_2608_01718_gb300 import workloads as wl
     if args.workload in CALIBRATION:
         return run_calibration(args)

@@ -6,6 +6,7 @@ Output: paper_2608_01718_gb300/_build/liblacache.so (git-ignored). No cmake; nvc
 """
 from __future__ import annotations
 
+import fcntl
 import os
 import shutil
 import subprocess
@@ -40,8 +41,19 @@ def flags(verbose: bool = False) -> list[str]:
 
 
 def build(verbose: bool = False, force: bool = False) -> str:
-    """Compile every CUDA source and link liblacache.so; returns its path."""
+    """Compile every CUDA source and link liblacache.so; returns its path. Concurrent callers (the ranks of a
+    multi-GPU run, parallel test workers) take a file lock, so one of them compiles and the others then find the
+    library up to date."""
     os.makedirs(BUILD, exist_ok=True)
+    with open(os.path.join(BUILD, ".lock"), "w") as lock:
+        fcntl.flock(lock, fcntl.LOCK_EX)
+        try:
+            return _build_locked(verbose, force)
+        finally:
+            fcntl.flock(lock, fcntl.LOCK_UN)
+
+
+def _build_locked(verbose: bool, force: bool) -> str:
     srcs = [os.path.join(CSRC, s) for s in SOURCES]
     deps = srcs + [os.path.join(CSRC, h) for h in ("internal.cuh", "tcgen05.cuh")]
     deps += [os.path.join(INCLUDE, "lacache.h"), __file__]

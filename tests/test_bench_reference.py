@@ -36,3 +36,16 @@ def test_reference_arm_prints_one_complete_line():
 
 def test_reference_arm_runs_on_rank_zero_only():
     assert _run(RANK="1", LOCAL_RANK="1", WORLD_SIZE="2") == []
+
+
+def test_gpus_flag_starts_one_rank_per_gpu():
+    """Without torchrun, --gpus N starts the N ranks itself (torch.distributed.run on this node): every rank sees
+    WORLD_SIZE = N, and only rank 0 prints, with n_gpus = N."""
+    env = {k: v for k, v in os.environ.items()
+           if k not in ("RANK", "LOCAL_RANK", "WORLD_SIZE", "MASTER_ADDR", "MASTER_PORT")}
+    run = subprocess.run(CMD + ["--gpus", "2"], cwd=ROOT, env=env, capture_output=True, text=True, timeout=600)
+    assert run.returncode == 0, run.stderr[-2000:]
+    lines = [line for line in run.stdout.splitlines() if line.startswith("{")]
+    assert len(lines) == 1
+    line = json.loads(lines[0])
+    assert line["n_gpus"] == 2 and line["impl"] == "reference" and line["value"] > 0

@@ -1,9 +1,11 @@
 """Parity at the full sizes of the large workloads, in the launch configuration the benchmark uses.
 
-large-16m (70 GB store) and batch-4m (8192 queries) check a stratified sample of queries against the streamed
-oracle. serve-2m runs all 1000 steps: the oracle replays the first steps from its own state, and every step is
-checked for the properties that hold at any size (the append log, bit-exact appended rows, and both checks passing
-for every HIT).
+large-16m (70 GB store) checks its whole batch of 128 queries against the streamed oracle, and batch-4m a
+stratified sample of 513 of its 8192 queries. serve-2m runs all 1000 steps. The oracle replays steps 0-2 from its
+own state. Five seeded later steps are verified against the store rebuilt from the GPU's append log: every logged
+row is first checked, bit for bit, against the non-HIT query row the GPU reported. Every step is also checked for
+the properties that hold at any size: the append log, bit-exact appended rows, and both checks passing for every
+HIT on a sampled step.
 """
 import numpy as np
 import pytest
@@ -57,13 +59,15 @@ def _check_streamed(w, per_class):
 
 
 def test_large_cache_near_hbm_capacity():
-    """16,777,216 entries x 1024 dims (34 GB of keys), B = 128, Zipf(1.1) targets."""
-    _check_streamed(wl.WORKLOADS["large-16m"], per_class=12)
+    """16,777,216 entries x 1024 dims (34 GB of keys), B = 128, Zipf(1.1) targets: every query of the batch."""
+    rep = _check_streamed(wl.WORKLOADS["large-16m"], per_class=128)
+    assert rep.queries == 128
 
 
 def test_large_batch_tensor_core_regime():
-    """4,194,304 entries x 768, B = 8192 (64 query tiles), top_c = 16."""
-    _check_streamed(wl.WORKLOADS["batch-4m"], per_class=60)
+    """4,194,304 entries x 768, B = 8192 (64 query tiles), top_c = 16: 171 queries of each class."""
+    rep = _check_streamed(wl.WORKLOADS["batch-4m"], per_class=171)
+    assert rep.queries >= 512
 
 
 def test_serve_loop_thousand_steps():
@@ -71,14 +75,17 @@ def test_serve_loop_thousand_steps():
     w = wl.WORKLOADS["serve-2m"]
     capacity = w.n + w.steps * w.batch
     p = params(w)
-    replay = 2
+    replay = 3
+    later = set(np.random.default_rng(w.seed).choice(np.arange(replay, w.steps), size=5, replace=False).tolist())
     st = oracle_store(w)
-    loop = oracle.ServeLoop(w.n + replay * w.batch, w.d, w.k, p)
+    # the oracle's own store: its appends on the replayed steps, then the rows of the GPU's append log
+    loop = oracle.ServeLoop(capacity, w.d, w.k, p)
     loop.insert(st.key, st.prefix, st.ids)
     del st
     origin = {}          # appended entry id -> (step, query index) of the query it holds
     hits_checked = 0
     replayed = Report()
+    rebuilt = Report()
     with new_cache(w, L.LACACHE_STAGE1_TENSOR, capacity=capacity) as cache:
         fill(cache, w)
         for step in range(w.steps):
@@ -99,17 +106,30 @@ def test_serve_loop_thousand_steps():
             assert torch.equal(pre.view(torch.int16), q["prefix"][sel].view(torch.int16))
             assert torch.equal(ids, q["ids"][sel])
             origin.update({first + i: (step, int(qi)) for i, qi in enumerate(miss)})
+            oq = oracle_queries(q)
             if step < replay:
                 g = {k: v.cpu().numpy() for k, v in out.items()}
-                res, ofirst, om = loop.step(oracle_queries(q))
+                res, ofirst, om = loop.step(oq)
                 rep = compare(g, res, p)
                 replayed.add(rep)
                 assert rep.band == 0 and (ofirst, om) == (first, m)
+            else:
+                assert loop.n == n_before
+                if step in later:
+                    # this step's decisions, verified against the store as the append log left it
+                    g = {k: v.cpu().numpy() for k, v in out.items()}
+                    rep = compare(g, oracle.lookup(loop.store, oq, p), p)
+                    rebuilt.add(rep)
+                    assert rep.band <= max(1, w.batch // 50)
+                # the logged rows (checked above against the reported non-HIT queries) join the oracle's store
+                loop.insert(oq["emb"][miss], oq["prefix"][miss], oq["ids"][miss])
             if step % 97 == 0:
                 hits_checked += _check_hits(w, p, q, out, origin)
         assert cache.size > w.n + 100 * w.steps
         assert hits_checked > 100
     log_report(f"{w.name} oracle-replayed steps 0-{replay - 1}", replayed)
+    log_report(f"{w.name} steps {sorted(later)} against the store rebuilt from the append log", rebuilt)
+    assert rebuilt.queries == 5 * w.batch and rebuilt.hits > 0 and rebuilt.rejects > 0 and rebuilt.misses > 0
     print(f"PARITY {w.name}: {w.steps} steps, final size {w.n + len(origin)}, HITs checked {hits_checked}",
           flush=True)
 
