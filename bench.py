@@ -1,7 +1,7 @@
 #!/usr/bin/env python3
 """Throughput of the LaCache two-stage lookahead lookup on GB300.
 
-    python bench.py [--gpus N --steps K --warmup W] [--workload large-16m] [--stage1 auto|tensor|simt]
+    python bench.py [--gpus N --steps K --warmup W] [--workload large-16m] [--stage1 auto|tensor|stream]
     python bench.py --impl reference ...        # the fp64 oracle on the host cores, a bounded sample per step
 
 A step is one lookup: stage 1 (key check with fused threshold + top-c) and stage 2 (merge, lookahead check,
@@ -37,7 +37,7 @@ sys.path.insert(0, ROOT)
 METRIC = "lookups/sec at 1 GB300 (N entries, batch B, k) + % of HBM or bf16 roofline"
 UNIT = "queries/s"
 FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
-STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "tensor-pair": "stage1_tensor.cu", "simt": "stage1_simt.cu",
+STAGE1_SOURCES = {"tensor": "stage1_tensor.cu", "tensor-pair": "stage1_tensor.cu", "stream": "stage1_stream.cu",
                   "lsh": "lsh.cu", "lsh-tensor": "lsh_tc.cu"}
 
 
@@ -48,7 +48,7 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="large-16m")
-    ap.add_argument("--stage1", choices=["auto", "tensor", "simt", "lsh"], default="auto")
+    ap.add_argument("--stage1", choices=["auto", "tensor", "stream", "lsh"], default="auto")
     ap.add_argument("--lsh-bits", type=int, default=256, help="SimHash signature bits for --stage1 lsh")
     ap.add_argument("--batches", type=int, default=8, help="distinct query batches cycled through")
     ap.add_argument("--e2e-steps", type=int, default=500)
@@ -77,25 +77,6 @@ def launch_ranks(n: int, argv: list[str]) -> int:
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={n}",
            "--master-addr", "127.0.0.1", "--master-port", str(port), os.path.abspath(__file__), *argv]
     return subprocess.call(cmd)
-
-
-def read_peak_gbs() -> float:
-    """A read-only streaming rate of this GPU's HBM: the best of five CUDA-event-timed torch.sum reductions over a
-    4 GiB fp32 buffer. The peaks file's HBM figure is a copy, which reads and writes; a scan only reads."""
-    import torch
-    x = torch.ones(1 << 30, dtype=torch.float32, device="cuda")
-    best = float("inf")
-    for i in range(6):
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record()
-        x.sum()
-        e1.record()
-        torch.cuda.synchronize()
-        if i:
-            best = min(best, e0.elapsed_time(e1))
-    del x
-    torch.cuda.empty_cache()
-    return (1 << 32) / (best / 1e3) / 1e9
 
 
 def load_peaks():
@@ -302,7 +283,7 @@ def run_ours(args, w):
     if world > 1:
         dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
     build.build()
-    stage1 = {"auto": L.LACACHE_STAGE1_AUTO, "tensor": L.LACACHE_STAGE1_TENSOR, "simt": L.LACACHE_STAGE1_SIMT,
+    stage1 = {"auto": L.LACACHE_STAGE1_AUTO, "tensor": L.LACACHE_STAGE1_TENSOR, "stream": L.LACACHE_STAGE1_STREAM,
               "lsh": L.LACACHE_STAGE1_LSH}
     # A workload with a step count is a serve loop (Algorithm 1 batch by batch): every timed step looks up a fresh
     # batch and then appends its misses, so the store grows while it is timed; the capacity holds that growth.
@@ -347,7 +328,7 @@ def run_ours(args, w):
     cache.sync()
     n_timed_begin = cache.size
     kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_TENSOR_PAIR: "tensor-pair",
-                   L.LACACHE_STAGE1_SIMT: "simt", L.LACACHE_STAGE1_LSH: "lsh",
+                   L.LACACHE_STAGE1_STREAM: "stream", L.LACACHE_STAGE1_LSH: "lsh",
                    L.LACACHE_STAGE1_LSH_TENSOR: "lsh-tensor"}[cache.last_launch()[1]]
     if world > 1:
         dist.barrier()
@@ -478,11 +459,6 @@ def run_ours(args, w):
         roof = {"bound": "tensor", "achieved": flops / t1_avg_s / 1e12, "peak": peak, "unit": "TFLOP/s",
                 "peak_source": f"{peak_src} ({'sustained' if sustained else 'burst'} bf16 dense)"}
     roof["frac"] = roof["achieved"] / roof["peak"]
-    if roof["bound"] == "hbm":
-        # secondary: the same bytes against a read-only streaming rate measured here (a scan only reads)
-        rp = read_peak_gbs()
-        roof |= {"read_peak_gbs": rp, "frac_of_read_peak": roof["achieved"] / rp,
-                 "read_peak_source": "measured live: best of 5 torch.sum over a 4 GiB fp32 buffer, CUDA events"}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
@@ -675,7 +651,7 @@ def run_sharded(args, w):
                 "unit": "TFLOP/s", "peak_source": f"{peak_src} (burst bf16 dense)"}
     roof["frac"] = roof["achieved"] / roof["peak"]
     kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_TENSOR_PAIR: "tensor-pair",
-                   L.LACACHE_STAGE1_SIMT: "simt", L.LACACHE_STAGE1_LSH: "lsh"}[cache.last_launch()[1]]
+                   L.LACACHE_STAGE1_STREAM: "stream", L.LACACHE_STAGE1_LSH: "lsh"}[cache.last_launch()[1]]
     line = {
         "metric": METRIC, "value": w.batch * args.steps / (elapsed_ms / 1e3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps,

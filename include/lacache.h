@@ -60,10 +60,11 @@ typedef enum { LACACHE_BF16 = 0, LACACHE_F32 = 1 } lacache_dtype;
 
 /* Which stage-1 kernel lookups run. */
 typedef enum {
-  LACACHE_STAGE1_AUTO = 0,   /* the tensor-core scan at every batch size: even one query keeps the scan bound by
-                                HBM, where the CUDA-core scan is bound by FFMA issue from a few queries up */
+  LACACHE_STAGE1_AUTO = 0,   /* the streaming scan for at most 4 queries against at most 32 MB of keys (a store L2
+                                holds, where its stage 1 has the shorter latency); the tensor-core scan otherwise,
+                                which holds the HBM roofline at every batch size once keys stream from HBM */
   LACACHE_STAGE1_TENSOR = 1, /* tcgen05 tensor-core scan (TMA-fed, TMEM accumulators) */
-  LACACHE_STAGE1_SIMT = 2,   /* CUDA-core FFMA scan */
+  LACACHE_STAGE1_STREAM = 2, /* streaming CUDA-core scan: warp per key tile, 128-bit key loads, packed fp32 FMA */
   LACACHE_STAGE1_LSH = 3,    /* SimHash index, then the exact key check (requires lacache_enable_lsh) */
   LACACHE_STAGE1_TENSOR_PAIR = 4, /* reported by lacache_last_launch only, not a configuration value: the tensor
                                      scan on two-CTA clusters (one M=256 MMA per pair of SMs), chosen for batches
@@ -123,8 +124,8 @@ typedef struct {
 } lacache_result;
 
 /* Create a cache on cfg->device with an empty store of cfg->capacity entries. Allocates the store
- * (capacity * (2d + 2 * prefix row + 4k) bytes), the stage-1 scratch (2 * SMs * max_batch * (8 * top_c + 4)
- * bytes) and host staging.
+ * (capacity * (2d + 2 * prefix row + 4k) bytes), the stage-1 scratch (S * max_batch * (8 * top_c + 4) bytes for
+ * S = 2 x SMs partial lists, or up to 4 x SMs while S * max_batch * top_c * 8 stays within 1 GiB) and host staging.
  * On success *out is a new handle; on failure *out is NULL and nothing stays allocated. */
 lacache_status lacache_create(const lacache_config* cfg, lacache_t** out);
 
@@ -285,8 +286,8 @@ lacache_status lacache_inject_stall(lacache_t* h, int32_t lookups);
  * The stage-1 scratch lives in an 8 MiB file-scope device array of the library, which every GPU that loads the
  * library holds until the process exits. 512 bytes of it hold a status word and alignment padding, so a batch
  * fits only if B * (8 * top_c + 4) <= 8 MiB - 512 bytes (for top_c = 32, B <= 32261); larger batches return
- * LACACHE_ERR_UNSUPPORTED and nothing runs. stage1 = LACACHE_STAGE1_AUTO runs the tensor-core scan, or the CUDA-core
- * scan if the driver offers no TMA descriptor encoder; an explicit LACACHE_STAGE1_TENSOR then gives
+ * LACACHE_ERR_UNSUPPORTED and nothing runs. stage1 = LACACHE_STAGE1_AUTO chooses as for a handle, and runs the
+ * streaming scan if the driver offers no TMA descriptor encoder; an explicit LACACHE_STAGE1_TENSOR then gives
  * LACACHE_ERR_CUDA. The first call on a device does a one-time set-up (it looks up the
  * array's device address), so make that first call before any stream capture. All calls on a device share the
  * array: calls that overlap on the GPU (other streams, other host threads) race and give undefined results, so

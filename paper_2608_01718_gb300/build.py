@@ -21,7 +21,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "liblacache.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-SOURCES = ["api.cu", "stage1_simt.cu", "stage1_tensor.cu", "stage2.cu", "noalloc.cu", "calibrate.cu", "lsh.cu",
+SOURCES = ["api.cu", "stage1_stream.cu", "stage1_tensor.cu", "stage2.cu", "noalloc.cu", "calibrate.cu", "lsh.cu",
            "lsh_tc.cu", "speculative.cu", "shards.cu"]
 
 

@@ -322,7 +322,7 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
     a.part_best = h->part_best;
     a.dev_status = h->dev_status;
     a.inputs_from_previous = gathered ? 1 : 0;
-    kernel = c.stage1 == LACACHE_STAGE1_AUTO ? LACACHE_STAGE1_TENSOR : c.stage1;
+    kernel = c.stage1 == LACACHE_STAGE1_AUTO ? lc::auto_stage1(h->n, c.d, B) : c.stage1;
     if (h->inject_stall > 0 && kernel == LACACHE_STAGE1_TENSOR) {
       a.inject_stall = 1;
       --h->inject_stall;
@@ -349,7 +349,7 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
         }
       }
     } else {
-      e = lc::launch_stage1_simt(a, h->num_sms, h->max_splits, st, &splits);
+      e = lc::launch_stage1_stream(a, h->num_sms, h->max_splits, st, &splits);
     }
     if (e != cudaSuccess) return LACACHE_ERR_CUDA;
   }
@@ -455,7 +455,7 @@ lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_
     delete h;
     return LACACHE_ERR_CUDA;
   }
-  h->max_splits = lc::max_splits_for(h->num_sms);
+  h->max_splits = lc::max_splits_for(h->num_sms, c.max_batch, c.top_c);
   const size_t cap = (size_t)c.capacity;
   bool ok = cudaMalloc(&h->key, cap * c.d * 2) == cudaSuccess &&
             cudaMalloc(&h->prefix, cap * pd * 2) == cudaSuccess &&

@@ -114,7 +114,8 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 // Launchers (host). Each returns the CUDA error of the launch. `splits` is the number of partial lists written.
-cudaError_t launch_stage1_simt(const Stage1Args& a, int num_sms, int max_splits, cudaStream_t st, int* splits);
+// The streaming CUDA-core scan (warp per key tile); batches past its shared-memory budget take several launches.
+cudaError_t launch_stage1_stream(const Stage1Args& a, int num_sms, int max_splits, cudaStream_t st, int* splits);
 // Encodes its own TMA descriptors for a.q and a.keys with `encode`.
 // *paired (if not null) is set when the batch ran on CTA pairs.
 cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int num_sms, int max_splits,
@@ -150,8 +151,27 @@ size_t lsh_index_bytes(int64_t capacity, int bits);
 cudaError_t launch_expand_signatures(const uint32_t* sig, int64_t first, int64_t n, int bits, uint8_t* index,
                                      int num_sms, cudaStream_t st);
 
-// Largest split count any stage-1 launcher uses for a given SM count (sizes the scratch): the SimHash scan runs two
-// CTAs per SM, the other kernels at most one split per SM.
-inline int max_splits_for(int num_sms) { return 2 * num_sms; }
+// LACACHE_STAGE1_AUTO's choice for a lookup of B queries against n keys of d elements. Once the keys stream from
+// HBM, the tensor-core scan holds the copy bandwidth at every batch size (measured 1.05-1.09 of it from 1 to 128
+// queries), and the streaming scan is level with it for one or two queries and slower from four. A store of at most
+// 32 MB of keys sits in L2 and the scan is bound by latency; there the streaming scan's stage 1 is the shorter one
+// for up to four queries (9.8 against 13.3 us at 4,096 x 768).
+constexpr int64_t kStreamAutoKeyBytes = (int64_t)32 << 20;
+constexpr int kStreamAutoMaxBatch = 4;
+inline int auto_stage1(int64_t n, int d, int B) {
+  return (B <= kStreamAutoMaxBatch && n * d * 2 <= kStreamAutoKeyBytes) ? LACACHE_STAGE1_STREAM
+                                                                        : LACACHE_STAGE1_TENSOR;
+}
+
+// Largest split count the stage-1 launchers may use on a handle (sizes its partial-list scratch). The SimHash scan
+// runs two CTAs per SM and the single-CTA kernels one split per SM. The CTA-pair schedule wants small splits, so
+// that the pairs sharing a key range read it from L2 (about 600 for 6 GB of keys); it may use up to 4 per SM while
+// the scratch of max_batch x top_c candidates per split stays within 1 GiB.
+inline int max_splits_for(int num_sms, int max_batch, int top_c) {
+  const int64_t per_split = (int64_t)max_batch * top_c * 8;
+  const int64_t budget = ((int64_t)1 << 30) / per_split;
+  const int64_t more = budget < 4 * (int64_t)num_sms ? budget : 4 * (int64_t)num_sms;
+  return more > 2 * num_sms ? (int)more : 2 * num_sms;
+}
 
 }  // namespace lc

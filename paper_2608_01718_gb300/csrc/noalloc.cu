@@ -77,7 +77,7 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
   const lacache_config c = *cfg;
   if (c.d <= 0 || c.k <= 0 || c.top_c <= 0 || isnan(c.tau_c) || isnan(c.tau_a)) return LACACHE_ERR_INVALID_ARG;
   if (c.check_mode < LACACHE_CHECK_EMB || c.check_mode > LACACHE_CHECK_BOTH) return LACACHE_ERR_INVALID_ARG;
-  if (c.stage1 < LACACHE_STAGE1_AUTO || c.stage1 > LACACHE_STAGE1_SIMT) return LACACHE_ERR_INVALID_ARG;
+  if (c.stage1 < LACACHE_STAGE1_AUTO || c.stage1 > LACACHE_STAGE1_STREAM) return LACACHE_ERR_INVALID_ARG;
   if (c.token_match_min > c.k) return LACACHE_ERR_INVALID_ARG;
   if (c.d % 8 != 0 || c.d > lc::kMaxD || c.k > lc::kMaxK || c.top_c > lc::kMaxTopC) return LACACHE_ERR_UNSUPPORTED;
   if (n > (int64_t)INT32_MAX) return LACACHE_ERR_UNSUPPORTED;
@@ -127,16 +127,16 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
       a.part_cand = part_cand;
       a.part_best = part_best;
       a.dev_status = status;
-      // AUTO takes the tensor-core scan, or the CUDA-core scan where the driver gives no TMA descriptor encoder;
-      // an explicit TENSOR request without the encoder is an error
-      int kernel = c.stage1 == LACACHE_STAGE1_AUTO ? LACACHE_STAGE1_TENSOR : c.stage1;
-      if (c.stage1 == LACACHE_STAGE1_AUTO && !s.encode) kernel = LACACHE_STAGE1_SIMT;
+      // AUTO chooses as for a handle, and takes the streaming CUDA-core scan where the driver gives no TMA descriptor
+      // encoder; an explicit TENSOR request without the encoder is an error
+      int kernel = c.stage1 == LACACHE_STAGE1_AUTO ? lc::auto_stage1(n, c.d, B) : c.stage1;
+      if (c.stage1 == LACACHE_STAGE1_AUTO && !s.encode) kernel = LACACHE_STAGE1_STREAM;
       cudaError_t e;
       if (kernel == LACACHE_STAGE1_TENSOR) {
         e = s.encode ? lc::launch_stage1_tensor(a, s.encode, s.num_sms, max_splits, st, &splits)
                      : cudaErrorInvalidValue;
       } else {
-        e = lc::launch_stage1_simt(a, s.num_sms, max_splits, st, &splits);
+        e = lc::launch_stage1_stream(a, s.num_sms, max_splits, st, &splits);
       }
       if (e != cudaSuccess) result = LACACHE_ERR_CUDA;
     }

@@ -15,7 +15,7 @@ LACACHE_OK, LACACHE_ERR_INVALID_ARG, LACACHE_ERR_CAPACITY, LACACHE_ERR_OOM = 0, 
 LACACHE_ERR_CUDA, LACACHE_ERR_DEVICE_TIMEOUT, LACACHE_ERR_UNSUPPORTED, LACACHE_ERR_IO = 4, 5, 6, 7
 LACACHE_CHECK_EMB, LACACHE_CHECK_TOKENS, LACACHE_CHECK_BOTH = 0, 1, 2
 LACACHE_BF16, LACACHE_F32 = 0, 1
-LACACHE_STAGE1_AUTO, LACACHE_STAGE1_TENSOR, LACACHE_STAGE1_SIMT, LACACHE_STAGE1_LSH = 0, 1, 2, 3
+LACACHE_STAGE1_AUTO, LACACHE_STAGE1_TENSOR, LACACHE_STAGE1_STREAM, LACACHE_STAGE1_LSH = 0, 1, 2, 3
 LACACHE_STAGE1_TENSOR_PAIR = 4   # reported by lacache_last_launch only
 LACACHE_STAGE1_LSH_TENSOR = 5    # reported by lacache_last_launch only
 LACACHE_MISS_KEY, LACACHE_HIT, LACACHE_REJECT = 0, 1, 2

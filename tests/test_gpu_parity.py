@@ -1,6 +1,6 @@
 """GPU parity: the CUDA lookup (through the C ABI) against the fp64 oracle on the same seeded bytes.
 
-Both stage-1 kernels are covered (the tcgen05 tensor-core scan and the CUDA-core scan). Cases span several key
+Both stage-1 kernels are covered (the tcgen05 tensor-core scan and the streaming CUDA-core scan). Cases span several key
 tiles with a ragged tail, ragged query tiles and ragged k-steps, the empty cache, exact duplicates, inclusive
 thresholds, top_c = 1 and 32, every check mode, host-buffer lookups and the serve loop with appends.
 """
@@ -20,7 +20,7 @@ from parity import (TOL, Report, compare, fill, gpu_lookup, log_report, new_cach
 
 pytestmark = pytest.mark.gpu
 
-PATHS = [pytest.param(L.LACACHE_STAGE1_TENSOR, id="tensor"), pytest.param(L.LACACHE_STAGE1_SIMT, id="simt")]
+PATHS = [pytest.param(L.LACACHE_STAGE1_TENSOR, id="tensor"), pytest.param(L.LACACHE_STAGE1_STREAM, id="stream")]
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -86,6 +86,38 @@ def test_dimension_and_window_extremes(stage1, d, k, batch):
     w = wl.WORKLOADS["mid-1m"].scaled(n=3_000, d=d, k=k, batch=batch, clusters=30, vocab=5)
     rep = run_parity(w, stage1, steps=(0, 1))
     assert rep.exact + rep.band == 2 * w.batch
+
+
+@pytest.mark.parametrize("d", [384, 768, 1024])
+@pytest.mark.parametrize("batch", [1, 2, 3, 5, 8, 9, 17])
+def test_stream_query_groups_and_load_phases(d, batch):
+    """The streaming scan's shapes: query groups of 1, 2, 4 and 8 (the batch rounded up; several groups past 8),
+    one or two load phases per row, lanes without a chunk (d = 384), and a store that is not a whole number of
+    warp tiles or splits."""
+    w = wl.WORKLOADS["mid-1m"].scaled(n=20_011, d=d, batch=batch)
+    rep = run_parity(w, L.LACACHE_STAGE1_STREAM)
+    assert rep.exact + rep.band == w.batch and rep.band <= 1
+
+
+def test_auto_takes_the_stream_scan_only_for_small_batches_on_stores_l2_holds():
+    """LACACHE_STAGE1_AUTO: the streaming scan for at most 4 queries against at most 32 MB of keys, the tensor-core
+    scan otherwise (and its results agree with the explicit kernels')."""
+    small = wl.WORKLOADS["mid-1m"].scaled(n=10_000, batch=8)      # 15 MB of keys
+    large = wl.WORKLOADS["mid-1m"].scaled(n=30_000, batch=8)      # 46 MB of keys
+    for w, want in ((small, {1: L.LACACHE_STAGE1_STREAM, 4: L.LACACHE_STAGE1_STREAM, 5: L.LACACHE_STAGE1_TENSOR}),
+                    (large, {1: L.LACACHE_STAGE1_TENSOR, 4: L.LACACHE_STAGE1_TENSOR})):
+        st = oracle_store(w)
+        with new_cache(w, L.LACACHE_STAGE1_AUTO) as cache:
+            fill(cache, w)
+            full = wl.batch(w, 0, device="cuda")
+            for B, kernel in want.items():
+                q = {k: full[k][:B].contiguous() for k in ("emb", "prefix", "ids")}
+                g = gpu_lookup(cache, q)
+                assert cache.last_launch()[1] == kernel, (w.n, B)
+                p = params(w)
+                oq = oracle_queries(q)
+                rep = compare(g, oracle.lookup(st, oq, p), p, pair_scores=pair_scores_fn(st, oq))
+                assert rep.exact + rep.band == B
 
 
 @pytest.mark.parametrize("stage1", PATHS)
@@ -365,14 +397,15 @@ def test_two_handles_look_up_concurrently_on_two_streams(batch):
                     assert np.array_equal(v.cpu().numpy(), g[k], equal_nan=True), k
 
 
-def test_back_to_back_lookups_of_mixed_sizes_match_lookups_run_alone():
+@pytest.mark.parametrize("stage1", PATHS)
+def test_back_to_back_lookups_of_mixed_sizes_match_lookups_run_alone(stage1):
     # A lookup's stage 1 scans while the previous lookup's stage 2 finishes, and both use the handle's partial-list
     # scratch and schedule counters. Lookups of changing batch size (single CTAs on the dynamic schedule and CTA
     # pairs, growing and shrinking the scratch they cover), enqueued back to back with no synchronization, must
     # each give the result of the same lookup run alone.
     w = wl.WORKLOADS["mid-1m"].scaled(n=60_000, batch=200)
     sizes = [32, 7, 200, 64, 1, 130, 32, 200, 5]
-    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+    with new_cache(w, stage1) as cache:
         fill(cache, w)
         full = [wl.batch(w, i, device="cuda") for i in range(len(sizes))]
         qs = [{k: full[i][k][:b].contiguous() for k in ("emb", "prefix", "ids")} for i, b in enumerate(sizes)]
@@ -453,10 +486,11 @@ def test_candidate_list_sizes(top_c, batch):
 
 
 @pytest.mark.parametrize("batch", [32, 200], ids=["dynamic-schedule", "cta-pairs"])
-def test_lookup_captured_in_a_cuda_graph_replays_like_eager_lookups(batch):
+@pytest.mark.parametrize("stage1", PATHS)
+def test_lookup_captured_in_a_cuda_graph_replays_like_eager_lookups(stage1, batch):
     # the stage-1 schedule keeps no host-side state between launches, so one captured lookup can be replayed
     w = wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch)
-    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+    with new_cache(w, stage1) as cache:
         fill(cache, w)
         q0, q1 = wl.batch(w, 0, device="cuda"), wl.batch(w, 1, device="cuda")
         eager = []

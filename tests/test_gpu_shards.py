@@ -40,7 +40,7 @@ def fill_range(cache, w, a, b):
 
 CASES = {
     "tiny-2": (wl.WORKLOADS["tiny-4k"], (0, 2048, 4096), L.LACACHE_STAGE1_TENSOR, oracle.CHECK_EMB),
-    "tiny-empty-simt": (wl.WORKLOADS["tiny-4k"], (0, 700, 700, 2901, 4096), L.LACACHE_STAGE1_SIMT, oracle.CHECK_EMB),
+    "tiny-empty-stream": (wl.WORKLOADS["tiny-4k"], (0, 700, 700, 2901, 4096), L.LACACHE_STAGE1_STREAM, oracle.CHECK_EMB),
     "tiny-16": (wl.WORKLOADS["tiny-4k"], tuple(range(0, 4097, 256)), L.LACACHE_STAGE1_TENSOR, oracle.CHECK_EMB),
     "tiny-tokens": (wl.WORKLOADS["tiny-4k"].scaled(n=3000, k=4, vocab=3, batch=48), (0, 1100, 3000),
                     L.LACACHE_STAGE1_TENSOR, oracle.CHECK_TOKENS),

@@ -46,7 +46,7 @@ def _same(a: dict, b: dict):
 
 
 @pytest.mark.parametrize("batch", [96, 256], ids=["one-tile", "cta-pairs"])
-@pytest.mark.parametrize("stage1", [L.LACACHE_STAGE1_TENSOR, L.LACACHE_STAGE1_SIMT], ids=["tensor", "simt"])
+@pytest.mark.parametrize("stage1", [L.LACACHE_STAGE1_TENSOR, L.LACACHE_STAGE1_STREAM], ids=["tensor", "stream"])
 def test_noalloc_lookup_matches_the_handle_lookup(stage1, batch):
     w = wl.WORKLOADS["mid-1m"].scaled(n=50_000, batch=batch)
     key, pre, ids = _rows(w)
@@ -64,11 +64,11 @@ def test_noalloc_lookup_matches_the_handle_lookup(stage1, batch):
 
 @pytest.mark.parametrize("mode,tmin,top_c,stage1", [
     (L.LACACHE_CHECK_TOKENS, 12, 8, L.LACACHE_STAGE1_TENSOR),
-    (L.LACACHE_CHECK_BOTH, 12, 8, L.LACACHE_STAGE1_SIMT),
+    (L.LACACHE_CHECK_BOTH, 12, 8, L.LACACHE_STAGE1_STREAM),
     (L.LACACHE_CHECK_EMB, 0, 1, L.LACACHE_STAGE1_AUTO),
     (L.LACACHE_CHECK_EMB, 0, 32, L.LACACHE_STAGE1_AUTO),
-    (L.LACACHE_CHECK_TOKENS, 12, 32, L.LACACHE_STAGE1_SIMT),
-], ids=["tokens-12", "both-12", "top1-auto", "top32-auto", "tokens-top32-simt"])
+    (L.LACACHE_CHECK_TOKENS, 12, 32, L.LACACHE_STAGE1_STREAM),
+], ids=["tokens-12", "both-12", "top1-auto", "top32-auto", "tokens-top32-stream"])
 def test_noalloc_modes_and_list_sizes(mode, tmin, top_c, stage1):
     """The check modes with a partial token match, the smallest and largest candidate lists, and AUTO: each filled
     into stage 2's arguments by the no-alloc entry point itself, against the handle's lookup."""
