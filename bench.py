@@ -59,6 +59,8 @@ def parse_args():
                          "the same batches, one all-gather and a merge per lookup (strong scaling)")
     ap.add_argument("--entries", type=int, default=0,
                     help="store size override: a smaller case of the workload (profiling captures)")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="batch size override: a batch-size case of the workload (kernel crossover measurements)")
     return ap.parse_args()
 
 
@@ -425,7 +427,8 @@ def run_ours(args, w):
     w_alg = w.scaled(n=n_timed_end) if serve else w
     s1_bytes, s2_bytes, flops = algorithmic(w_alg, w.batch)
     t1_avg_s = t1_ms / max(1, timed) / 1e3
-    traffic = None if args.entries else kernel_traffic(kernel_name, w.name, f"-b{lsh['bits']}" if lsh else "")
+    traffic = None if args.entries or args.batch else kernel_traffic(kernel_name, w.name,
+                                                                      f"-b{lsh['bits']}" if lsh else "")
     value = job["value"]
     # the stage-1 kernel is bound by HBM below the ridge (flops per byte of the measured peaks), else by the
     # tensor pipe; a kernel timed back to back for over a second is compared with the sustained bf16 peak
@@ -735,6 +738,8 @@ def main():
     w = wl.WORKLOADS[args.workload]
     if args.entries:
         w = w.scaled(n=args.entries)
+    if args.batch:
+        w = w.scaled(batch=args.batch)
     if args.impl == "reference":
         return run_reference(args, w)
     if args.mode == "shard":

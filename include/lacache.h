@@ -124,7 +124,7 @@ typedef struct {
 } lacache_result;
 
 /* Create a cache on cfg->device with an empty store of cfg->capacity entries. Allocates the store
- * (capacity * (2d + 2 * prefix row + 4k) bytes), the stage-1 scratch (S * max_batch * (8 * top_c + 4) bytes for
+ * (capacity * (2d + 2 * prefix row + 4k) bytes), the stage-1 scratch (S * max_batch * (8 * top_c + 8) bytes for
  * S = 2 x SMs partial lists, or up to 4 x SMs while S * max_batch * top_c * 8 stays within 1 GiB) and host staging.
  * On success *out is a new handle; on failure *out is NULL and nothing stays allocated. */
 lacache_status lacache_create(const lacache_config* cfg, lacache_t** out);
@@ -285,7 +285,7 @@ lacache_status lacache_inject_stall(lacache_t* h, int32_t lookups);
  * d, k, tau_c, tau_a, top_c, token_match_min, check_mode, device and stage1; capacity and max_batch are ignored.
  * The stage-1 scratch lives in an 8 MiB file-scope device array of the library, which every GPU that loads the
  * library holds until the process exits. 512 bytes of it hold a status word and alignment padding, so a batch
- * fits only if B * (8 * top_c + 4) <= 8 MiB - 512 bytes (for top_c = 32, B <= 32261); larger batches return
+ * fits only if B * (8 * top_c + 8) <= 8 MiB - 512 bytes (for top_c = 32, B <= 31773); larger batches return
  * LACACHE_ERR_UNSUPPORTED and nothing runs. stage1 = LACACHE_STAGE1_AUTO chooses as for a handle, and runs the
  * streaming scan if the driver offers no TMA descriptor encoder; an explicit LACACHE_STAGE1_TENSOR then gives
  * LACACHE_ERR_CUDA. The first call on a device does a one-time set-up (it looks up the

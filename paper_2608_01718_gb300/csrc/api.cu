@@ -23,7 +23,7 @@ struct lacache {
   __nv_bfloat16* prefix;     // [capacity x pd]
   int32_t* ids;              // [capacity x k]
   uint64_t* part_cand;       // [max_splits x max_batch x top_c]
-  float* part_best;          // [max_splits x max_batch]
+  lc::PartMeta* part_meta;   // [max_splits x max_batch]
   unsigned int* dev_status;  // device status word
   int32_t* append_dst;       // [max_batch] destination rank of each appended query
   int32_t* append_count;     // device count of appended rows
@@ -287,7 +287,7 @@ void free_all(lacache* h) {
   cudaFree(h->prefix);
   cudaFree(h->ids);
   cudaFree(h->part_cand);
-  cudaFree(h->part_best);
+  cudaFree(h->part_meta);
   cudaFree(h->dev_status);
   cudaFree(h->append_dst);
   cudaFree(h->append_count);
@@ -319,7 +319,7 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
     a.tau_c = c.tau_c;
     a.top_c = c.top_c;
     a.part_cand = h->part_cand;
-    a.part_best = h->part_best;
+    a.part_meta = h->part_meta;
     a.dev_status = h->dev_status;
     a.inputs_from_previous = gathered ? 1 : 0;
     kernel = c.stage1 == LACACHE_STAGE1_AUTO ? lc::auto_stage1(h->n, c.d, B) : c.stage1;
@@ -356,7 +356,7 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
   Stage2Args b{};
   b.n = h->n;
   b.part_cand = h->part_cand;
-  b.part_best = h->part_best;
+  b.part_meta = h->part_meta;
   b.splits = splits;
   b.B = B;
   b.pd = h->pd;
@@ -461,7 +461,7 @@ lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_
             cudaMalloc(&h->prefix, cap * pd * 2) == cudaSuccess &&
             cudaMalloc(&h->ids, cap * c.k * 4) == cudaSuccess &&
             cudaMalloc(&h->part_cand, (size_t)h->max_splits * c.max_batch * c.top_c * 8) == cudaSuccess &&
-            cudaMalloc(&h->part_best, (size_t)h->max_splits * c.max_batch * 4) == cudaSuccess &&
+            cudaMalloc(&h->part_meta, (size_t)h->max_splits * c.max_batch * sizeof(lc::PartMeta)) == cudaSuccess &&
             cudaMalloc(&h->dev_status, 4) == cudaSuccess &&
             cudaMalloc(&h->append_dst, (size_t)c.max_batch * 4) == cudaSuccess &&
             cudaMalloc(&h->append_count, 4) == cudaSuccess &&

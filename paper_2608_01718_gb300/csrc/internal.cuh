@@ -65,8 +65,15 @@ __host__ __device__ __forceinline__ uint64_t pack_cand(float s, uint32_t j) {
 __host__ __device__ __forceinline__ float cand_score(uint64_t c) { return score_of_order((uint32_t)(c >> 32)); }
 __host__ __device__ __forceinline__ uint32_t cand_id(uint64_t c) { return ~(uint32_t)c; }
 
-// Stage-1 output: per split s and query q, the split's top_c candidates (sorted, 0-padded) and its best score.
-//   part_cand[(s * B + q) * top_c + i], part_best[s * B + q]
+// Stage-1 output, per split s and query q: a record of the split's best key score (over all its entries: a miss
+// reports the best over the store) and of how many candidates its partial list holds, and the list itself, sorted,
+// in its first `count` slots (later slots are not written: most lists hold few candidates, or none).
+//   part_meta[s * B + q], part_cand[(s * B + q) * top_c + i] for i < count
+struct __align__(8) PartMeta {
+  float best;
+  uint32_t count;
+};
+
 struct Stage1Args {
   const __nv_bfloat16* keys;  // [n x d] store keys
   int64_t n;
@@ -76,7 +83,7 @@ struct Stage1Args {
   float tau_c;
   int top_c;
   uint64_t* part_cand;
-  float* part_best;
+  PartMeta* part_meta;
   unsigned int* dev_status;
   int inject_stall;           // test support: CTA 0 of the tensor kernel withholds one load (see lacache.h)
   int* tile_ctr;              // tensor kernel, one query tile: dynamic tile schedule on these two counters
@@ -89,7 +96,7 @@ struct Stage1Args {
 struct Stage2Args {
   int64_t n;                     // valid entries: candidate ids at or past n are dropped
   const uint64_t* part_cand;
-  const float* part_best;
+  const PartMeta* part_meta;
   int splits;
   int B;
   int pd;                        // prefix row length: sum of the models' dimensions

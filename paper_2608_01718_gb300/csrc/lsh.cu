@@ -250,11 +250,17 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
       }
     }
     flush(sh, a, q0, qn);
+    // the lists' candidates (a sorted list holds them in its first slots, then zeros) and each list's record
     for (int i = threadIdx.x; i < qn * C; i += kThreads) {
       const int qq = i / C;
-      a.part_cand[((int64_t)s * a.B + q0 + qq) * C + (i - qq * C)] = sh.list[qq][i - qq * C];
+      const uint64_t x = sh.list[qq][i - qq * C];
+      if (x) a.part_cand[((int64_t)s * a.B + q0 + qq) * C + (i - qq * C)] = x;
     }
-    if (threadIdx.x < qn) a.part_best[(int64_t)s * a.B + q0 + threadIdx.x] = score_of_order(sh.best[threadIdx.x]);
+    if (threadIdx.x < qn) {
+      uint32_t count = 0;
+      while ((int)count < C && sh.list[threadIdx.x][count]) ++count;
+      a.part_meta[(int64_t)s * a.B + q0 + threadIdx.x] = PartMeta{score_of_order(sh.best[threadIdx.x]), count};
+    }
     __syncthreads();
   }
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");

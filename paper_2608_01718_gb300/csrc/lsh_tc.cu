@@ -571,11 +571,16 @@ __global__ void __launch_bounds__(kThreads, 1) lsh_tc_kernel(Stage1Args a, LshAr
     if (__syncthreads_or(*abort_flag != 0)) break;
     if (warp < kEpiWarps) {
       const int et = threadIdx.x;
+      // the lists' candidates (a sorted list holds them in its first slots, then zeros) and each list's record
       for (int i = et; i < qn * C; i += kEpiWarps * 32) {
         const int qq = i / C;
-        a.part_cand[((int64_t)s * a.B + q0 + qq) * C + (i - qq * C)] = lists[i];
+        if (lists[i]) a.part_cand[((int64_t)s * a.B + q0 + qq) * C + (i - qq * C)] = lists[i];
       }
-      for (int i = et; i < qn; i += kEpiWarps * 32) a.part_best[(int64_t)s * a.B + q0 + i] = score_of_order(t.best[i]);
+      for (int i = et; i < qn; i += kEpiWarps * 32) {
+        uint32_t count = 0;
+        while ((int)count < C && lists[(size_t)i * C + count]) ++count;
+        a.part_meta[(int64_t)s * a.B + q0 + i] = PartMeta{score_of_order(t.best[i]), count};
+      }
     }
     __syncthreads();
   }

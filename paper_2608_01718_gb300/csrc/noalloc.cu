@@ -22,7 +22,7 @@ constexpr size_t kNoAllocScratchBytes = (size_t)8 << 20;   // the stated maximum
 constexpr size_t kStatusBytes = 256;                         // device status word, first 256 bytes
 constexpr int kMaxDevices = 64;
 
-// The scratch: [status word | partial candidate lists | partial best scores]. In host code this name is only a
+// The scratch: [status word | partial candidate lists | partial-list records]. In host code this name is only a
 // host-side stand-in; kernels receive the device address found by cudaGetSymbolAddress below.
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
@@ -89,7 +89,7 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
       !out->n_cand)
     return LACACHE_ERR_INVALID_ARG;
   // The batch must fit the fixed scratch with at least one partial list per query.
-  const size_t per_split = (size_t)B * ((size_t)8 * c.top_c + 4);
+  const size_t per_split = (size_t)B * ((size_t)8 * c.top_c + sizeof(lc::PartMeta));
   const size_t room = kNoAllocScratchBytes - kStatusBytes - 256;
   if (per_split > room) return LACACHE_ERR_UNSUPPORTED;
 
@@ -110,7 +110,7 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
     unsigned int* status = reinterpret_cast<unsigned int*>(s.scratch);
     uint64_t* part_cand = reinterpret_cast<uint64_t*>(s.scratch + kStatusBytes);
     const size_t cand_bytes = ((size_t)max_splits * B * c.top_c * 8 + 255) & ~(size_t)255;
-    float* part_best = reinterpret_cast<float*>(s.scratch + kStatusBytes + cand_bytes);
+    lc::PartMeta* part_meta = reinterpret_cast<lc::PartMeta*>(s.scratch + kStatusBytes + cand_bytes);
     // Only the status word must start at zero; the stage-1 kernels write every partial entry they later read.
     if (cudaMemsetAsync(status, 0, sizeof(unsigned int), st) != cudaSuccess) result = LACACHE_ERR_CUDA;
 
@@ -125,7 +125,7 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
       a.tau_c = c.tau_c;
       a.top_c = c.top_c;
       a.part_cand = part_cand;
-      a.part_best = part_best;
+      a.part_meta = part_meta;
       a.dev_status = status;
       // AUTO chooses as for a handle, and takes the streaming CUDA-core scan where the driver gives no TMA descriptor
       // encoder; an explicit TENSOR request without the encoder is an error
@@ -144,7 +144,7 @@ extern "C" lacache_status lacache_lookup_noalloc(const lacache_config* cfg, int6
       lc::Stage2Args b{};
       b.n = n;
       b.part_cand = part_cand;
-      b.part_best = part_best;
+      b.part_meta = part_meta;
       b.splits = splits;
       b.B = B;
       b.pd = c.d;

@@ -46,7 +46,7 @@ struct StreamParams {
   int top_c;
   int splits;
   uint64_t* part_cand;
-  float* part_best;
+  PartMeta* part_meta;
   int wait_first;     // the queries are written by the grid launched just before: wait before reading them
 };
 
@@ -246,7 +246,8 @@ __global__ void __launch_bounds__(kThreads, 1) stage1_stream_kernel(const Stream
       b = fmaxf(b, best[w * qpad + t]);
     }
     uint64_t* dst = p.part_cand + ((int64_t)blockIdx.x * p.B + p.q0 + t) * C;
-    for (int i = 0; i < C; ++i) {
+    int count = 0;
+    for (; count < C; ++count) {
       uint64_t mx = 0;
       int mw = -1;
       for (int w = 0; w < kWarps; ++w) {
@@ -256,10 +257,11 @@ __global__ void __launch_bounds__(kThreads, 1) stage1_stream_kernel(const Stream
           mw = w;
         }
       }
-      dst[i] = mx;
-      if (mw >= 0) ++head[mw];
+      if (mw < 0) break;   // every warp's list is exhausted
+      dst[count] = mx;
+      ++head[mw];
     }
-    p.part_best[(int64_t)blockIdx.x * p.B + p.q0 + t] = b;
+    p.part_meta[(int64_t)blockIdx.x * p.B + p.q0 + t] = PartMeta{b, (uint32_t)count};
   }
 }
 
@@ -334,7 +336,7 @@ cudaError_t launch_stage1_stream(const Stage1Args& a, int num_sms, int max_split
   if (s < 1) s = 1;
   p.splits = (int)s;
   p.part_cand = a.part_cand;
-  p.part_best = a.part_best;
+  p.part_meta = a.part_meta;
   *splits = p.splits;
   for (int q0 = 0; q0 < a.B; q0 += qc) {
     p.q0 = q0;

@@ -86,7 +86,7 @@ struct TcParams {
   uint32_t* sig;     // signature mode: [n x sig_words] output words
   int sig_words;
   uint64_t* part_cand;
-  float* part_best;
+  PartMeta* part_meta;
   unsigned int* dev_status;
 };
 
@@ -522,8 +522,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint64_t* dst = p.part_cand + ((int64_t)sp * p.B + q) * p.top_c;
 #pragma unroll
       for (int i = 0; i < CPAD; ++i)
-        if (i < p.top_c) dst[i] = i < top.count ? pack_cand(top.s[i], top.j[i]) : 0ull;
-      p.part_best[(int64_t)sp * p.B + q] = best;
+        if (i < top.count) dst[i] = pack_cand(top.s[i], top.j[i]);
+      p.part_meta[(int64_t)sp * p.B + q] = PartMeta{best, (uint32_t)top.count};
     };
     if (dyn) {
       const bool active = row < p.B;
@@ -763,7 +763,7 @@ cudaError_t launch_stage1_tensor(const Stage1Args& a, EncodeTiledFn encode, int 
   p.n_tiles = (a.n + BN - 1) / BN;
   p.k_steps = (a.d + BK - 1) / BK;
   p.part_cand = a.part_cand;
-  p.part_best = a.part_best;
+  p.part_meta = a.part_meta;
   p.dev_status = a.dev_status;
   p.inject_stall = a.inject_stall;
   p.wait_first = a.inputs_from_previous;

@@ -1,10 +1,10 @@
 // Candidate merge, stage 2 (the lookahead check) and the decision, fused in one kernel.
 //
 // One CTA (8 warps) per query:
-//  1. merge the stage-1 partial lists (splits x top_c packed candidates) into C_q, the top_c candidates by
-//     (key score desc, entry id asc): every thread keeps a sorted top-c of the entries it reads (loads issued
-//     eight at a time), each warp reduces its lanes' lists by top_c rounds of a warp-wide max, and warp 0 merges
-//     the eight warp lists the same way;
+//  1. merge the stage-1 partial lists (per split a record of its best score and candidate count, and that many
+//     packed candidates) into C_q, the top_c candidates by (key score desc, entry id asc): every thread keeps a
+//     sorted top-c of the candidates it reads (four splits in flight), each warp reduces its lanes' lists by top_c
+//     rounds of a warp-wide max, and warp 0 merges the eight warp lists the same way;
 //  2. the candidates are checked in parallel, one warp per candidate: r = <p_q, P_j> (the prefix-embedding cosine
 //     sim(f_k(x), f_k(x'))) in fp32, each lane's 8-element chunks in order, then a butterfly sum (every lane ends
 //     with the same bits); m = number of positions i < k with equal token ids;
@@ -82,40 +82,43 @@ __global__ void __launch_bounds__(kThreads) stage2_kernel(Stage2Args a) {
   // The next lookup's stage 1 may be scheduled now; it too waits for this grid before touching memory.
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-  // 1a + 1b. The splits' best scores and their partial lists, loaded together (one memory round trip for the
-  // common case of at most 2 x kThreads splits and U x kThreads list entries); then the maximum of the best
-  // scores, and every thread's sorted top-c of the entries it read.
+  // 1a + 1b. Every thread takes splits tid, tid + kThreads, ...: a split's record (best score, candidate count) and
+  // the first two slots of its list are loaded together, before the count is known, so lists of at most two
+  // candidates (the common case) take one memory round trip; longer ones load their other slots after it. Then the
+  // maximum of the best scores, and every thread's sorted top-c of the candidates it read.
   uint64_t loc[CPAD];
 #pragma unroll
   for (int i = 0; i < CPAD; ++i) loc[i] = 0;
-  const int total = a.splits * C;
-  constexpr int U = CPAD <= 16 ? 8 : 4;   // loads in flight per thread (one pass for 152 splits x 8)
+  constexpr int U = 4;   // splits in flight per thread
   float best = -INFINITY;
-  {
-    const int s0 = threadIdx.x, s1 = threadIdx.x + kThreads;
-    const float b0 = s0 < a.splits ? a.part_best[(int64_t)s0 * a.B + q] : -INFINITY;
-    const float b1 = s1 < a.splits ? a.part_best[(int64_t)s1 * a.B + q] : -INFINITY;
-    best = fmaxf(b0, b1);
-  }
-  for (int e0 = threadIdx.x; e0 < total; e0 += U * kThreads) {
-    uint64_t x[U];
+  auto take = [&](uint64_t x) {
+    if ((int64_t)cand_id(x) >= a.n) x = 0;   // never gather outside the store
+    keep(loc, x);
+  };
+  for (int s0 = threadIdx.x; s0 < a.splits; s0 += U * kThreads) {
+    PartMeta m[U];
+    uint64_t x0[U], x1[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const int e = e0 + u * kThreads;
-      x[u] = 0;
-      if (e < total) {
-        const int s = e / C;
-        x[u] = a.part_cand[((int64_t)s * a.B + q) * C + (e - s * C)];
+      const int sp = s0 + u * kThreads;
+      m[u] = PartMeta{-INFINITY, 0u};
+      x0[u] = x1[u] = 0;
+      if (sp < a.splits) {
+        const int64_t r = (int64_t)sp * a.B + q;
+        m[u] = a.part_meta[r];
+        x0[u] = a.part_cand[r * C];
+        if (C > 1) x1[u] = a.part_cand[r * C + 1];
       }
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      if (x[u] != 0 && (int64_t)cand_id(x[u]) >= a.n) x[u] = 0;   // never gather outside the store
-      keep(loc, x[u]);
+      best = fmaxf(best, m[u].best);
+      const int cnt = (int)m[u].count < C ? (int)m[u].count : C;
+      if (cnt > 0) take(x0[u]);
+      if (cnt > 1) take(x1[u]);
+      for (int i = 2; i < cnt; ++i) take(a.part_cand[((int64_t)(s0 + u * kThreads) * a.B + q) * C + i]);
     }
   }
-  for (int s = threadIdx.x + 2 * kThreads; s < a.splits; s += kThreads)
-    best = fmaxf(best, a.part_best[(int64_t)s * a.B + q]);
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) best = fmaxf(best, __shfl_xor_sync(kFull, best, o));
   if (lane == 0) warp_best[warp] = best;

@@ -96,9 +96,9 @@ def _empty_batch(B, d, k):
 def test_noalloc_empty_cache_and_largest_batch():
     """With no rows (n = 0) stage 1 does not run and stage 2 sees no partial list: every query is a key miss, as
     for an empty handle. The batch is the largest the fixed scratch takes at top_c = 32:
-    B * (8 * top_c + 4) <= 8 MiB - 512 bytes."""
+    B * (8 * top_c + 8) <= 8 MiB - 512 bytes."""
     d, k, top_c = 64, 4, 32
-    B = ((8 << 20) - 512) // (8 * top_c + 4)
+    B = ((8 << 20) - 512) // (8 * top_c + 8)
     q, qi = _empty_batch(B, d, k)
     cfg = L.make_config(d, k, 1, 0.9, 0.8, top_c, max_batch=B)
     for _ in range(2):
@@ -118,7 +118,7 @@ def test_noalloc_empty_cache_and_largest_batch():
 def test_noalloc_refuses_a_batch_larger_than_its_scratch():
     d, top_c = 64, 32
     cfg = L.make_config(d, 4, 1, 0.9, 0.8, top_c, max_batch=1)
-    B = ((8 << 20) - 512) // (8 * top_c + 4) + 1    # one query more than fits the 8 MiB scratch
+    B = ((8 << 20) - 512) // (8 * top_c + 8) + 1    # one query more than fits the 8 MiB scratch
     q = torch.zeros((B, d), dtype=torch.bfloat16, device="cuda")
     qi = torch.zeros((B, 4), dtype=torch.int32, device="cuda")
     out = L.alloc_result(B, top_c, "cuda", candidates=False)
