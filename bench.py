@@ -81,6 +81,74 @@ def launch_ranks(n: int, argv: list[str]) -> int:
     return subprocess.call(cmd)
 
 
+def peaks_lib():
+    """The measurement kernels (libpeaks.so, built beside the lookup library)."""
+    from paper_2608_01718_gb300 import build
+    lib = ctypes.CDLL(build.PEAKS_LIB)
+    lib.lcpeaks_read.argtypes = [ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p]
+    lib.lcpeaks_popc.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.c_int,
+                                 ctypes.c_void_p]
+    return lib
+
+
+def timed_best(launch, reps: int = 5) -> float:
+    """Best CUDA-event time (ms) of `launch` on the current stream, over reps runs after one warm-up run."""
+    import torch
+    best = float("inf")
+    for i in range(reps + 1):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        launch()
+        e1.record()
+        torch.cuda.synchronize()
+        if i:
+            best = min(best, e0.elapsed_time(e1))
+    return best
+
+
+def read_peak_gbs() -> float:
+    """HBM read rate of a kernel that only reads: the best of 5 CUDA-event-timed passes of lcpeaks_read (128-bit
+    loads, four in flight per thread) over a 4 GiB buffer."""
+    import torch
+    lib = peaks_lib()
+    nbytes = 1 << 32
+    buf = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
+    sink = torch.zeros(1, dtype=torch.int32, device="cuda")
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    stream = torch.cuda.current_stream().cuda_stream
+
+    def launch():
+        if lib.lcpeaks_read(buf.data_ptr(), nbytes, sink.data_ptr(), sms, stream):
+            raise RuntimeError("lcpeaks_read failed")
+    ms = timed_best(launch)
+    del buf
+    torch.cuda.empty_cache()
+    return nbytes / (ms / 1e3) / 1e9
+
+
+def popc_peak(words: int, radius: int) -> dict:
+    """The SimHash scan's distance arithmetic with no memory traffic (lcpeaks_popc), timed with CUDA events while
+    nvidia-smi samples the SM clock: signature words compared per second, and per clock and SM."""
+    import torch
+    lib = peaks_lib()
+    sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+    sink = torch.zeros(1, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream().cuda_stream
+    steps = 4096 * 8 // words
+    clocks = ClockSampler(torch.cuda.current_device())
+    clocks.start()
+
+    def launch():
+        if lib.lcpeaks_popc(words, steps, radius, sink.data_ptr(), sms, stream):
+            raise RuntimeError("lcpeaks_popc failed")
+    ms = timed_best(launch, reps=10)
+    clk = clocks.stop()
+    total = 2 * sms * 512 * steps * 32 * words
+    rate = total / (ms / 1e3)
+    mhz = clk.get("sm_mhz") or 2070.0
+    return {"words_per_s": rate, "words_per_clock_per_sm": rate / (sms * mhz * 1e6), "sm_mhz": mhz}
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -444,14 +512,22 @@ def run_ours(args, w):
         # lookup. Population count runs at 16 per clock per SM (the CUDA arithmetic-throughput table), the logic
         # and integer operations at 64. The scan's carry-save adders fold 8 words into 5 popcounts (4 into 3), whose
         # 19 (10) other operations fit under the popcount time on the 64-wide pipe. So the derived ceiling is
-        # 16 x 8 / 5 words (16 x 4 / 3 at 128 bits) per clock per SM x SMs x the maximum SM clock.
+        # 16 x 8 / 5 words (16 x 4 / 3 at 128 bits) per clock per SM x SMs x the maximum SM clock. Beside it, the
+        # same arithmetic measured with no memory traffic (lcpeaks_popc), scaled to the scan's median SM clock.
         sms = torch.cuda.get_device_properties(local_rank).multi_processor_count
         words = w.batch * w.n * (lsh["bits"] // 32)
         per_clock = 16 * (8 / 5 if (lsh["bits"] // 32) % 8 == 0 else 4 / 3)
-        roof = {"bound": "alu", "achieved": words / t1_avg_s / 1e12,
+        achieved = words / t1_avg_s / 1e12
+        mp = popc_peak(lsh["bits"] // 32, lsh["radius"])
+        measured = mp["words_per_clock_per_sm"] * sms * (clock.get("sm_mhz") or mp["sm_mhz"]) * 1e6 / 1e12
+        roof = {"bound": "alu", "achieved": achieved,
                 "peak": per_clock * sms * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12, "unit": "Twords/s",
                 "peak_source": f"derived: {per_clock:.1f} signature words/clock/SM (popcounts at 16/clock after "
                                f"carry-save folding) x {sms} SMs x max SM clock",
+                "measured_peak": measured, "frac_of_measured_peak": achieved / measured,
+                "measured_peak_source": "lcpeaks_popc: the scan's XOR / carry-save / popcount / compare arithmetic "
+                                        f"on register and shared data, {mp['words_per_clock_per_sm']:.2f} words/clock"
+                                        "/SM measured, x SMs x the scan's median SM clock",
                 "algorithmic_word_comparisons_per_launch": words}
     elif flops / s1_bytes < ridge:
         roof = {"bound": "hbm", "achieved": s1_bytes / t1_avg_s / 1e9, "peak": peaks["hbm_gbs"], "unit": "GB/s",
@@ -462,6 +538,11 @@ def run_ours(args, w):
         roof = {"bound": "tensor", "achieved": flops / t1_avg_s / 1e12, "peak": peak, "unit": "TFLOP/s",
                 "peak_source": f"{peak_src} ({'sustained' if sustained else 'burst'} bf16 dense)"}
     roof["frac"] = roof["achieved"] / roof["peak"]
+    if roof["bound"] == "hbm":
+        # beside the copy peak (which reads and writes every byte), the rate of a kernel that only reads
+        rp = read_peak_gbs()
+        roof |= {"read_peak_gbs": rp, "frac_of_read_peak": roof["achieved"] / rp,
+                 "read_peak_source": "measured live: lcpeaks_read, best of 5 reads of a 4 GiB buffer, CUDA events"}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,

@@ -2,7 +2,8 @@
 
     python -m paper_2608_01718_gb300.build [-v]
 
-Output: paper_2608_01718_gb300/_build/liblacache.so (git-ignored). No cmake; nvcc and a C++ host compiler only.
+Output: paper_2608_01718_gb300/_build/liblacache.so, and libpeaks.so (the benchmark's measurement kernels, not part
+of the lookup library), both git-ignored. No cmake; nvcc and a C++ host compiler only.
 """
 from __future__ import annotations
 
@@ -19,6 +20,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "liblacache.so")
+PEAKS_LIB = os.path.join(BUILD, "libpeaks.so")
+PEAKS_SOURCE = "peaks.cu"
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 SOURCES = ["api.cu", "stage1_stream.cu", "stage1_tensor.cu", "stage2.cu", "noalloc.cu", "calibrate.cu", "lsh.cu",
@@ -57,24 +60,34 @@ def _build_locked(verbose: bool, force: bool) -> str:
     srcs = [os.path.join(CSRC, s) for s in SOURCES]
     deps = srcs + [os.path.join(CSRC, h) for h in ("internal.cuh", "tcgen05.cuh")]
     deps += [os.path.join(INCLUDE, "lacache.h"), __file__]
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= max(os.path.getmtime(p) for p in deps):
+    peaks_src = os.path.join(CSRC, PEAKS_SOURCE)
+    lib_ok = os.path.exists(LIB) and os.path.getmtime(LIB) >= max(os.path.getmtime(p) for p in deps)
+    peaks_ok = os.path.exists(PEAKS_LIB) and os.path.getmtime(PEAKS_LIB) >= max(os.path.getmtime(peaks_src),
+                                                                                   os.path.getmtime(__file__))
+    if not force and lib_ok and peaks_ok:
         return LIB
     tool = nvcc()
     objs, procs = [], []
+    fd, peaks_tmp = tempfile.mkstemp(suffix=".so", dir=BUILD)
+    os.close(fd)
+    peaks = subprocess.Popen([tool, *flags(verbose), "-shared", peaks_src, "-o", peaks_tmp], stdout=subprocess.PIPE,
+                             stderr=subprocess.STDOUT, text=True)
     for src in srcs:
         obj = os.path.join(BUILD, os.path.basename(src).replace(".cu", ".o"))
         objs.append(obj)
         cmd = [tool, *flags(verbose), "-c", src, "-o", obj]
         procs.append((src, subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.STDOUT, text=True)))
     failed = []
-    for src, proc in procs:
+    for src, proc in procs + [(peaks_src, peaks)]:
         out, _ = proc.communicate()
         if verbose or proc.returncode:
             sys.stderr.write(out)
         if proc.returncode:
             failed.append(src)
     if failed:
+        os.unlink(peaks_tmp)
         raise RuntimeError(f"nvcc failed for {failed}")
+    os.replace(peaks_tmp, PEAKS_LIB)
     fd, tmp = tempfile.mkstemp(suffix=".so", dir=BUILD)
     os.close(fd)
     link = [tool, *ARCH, "-shared", "-Xcompiler", "-fPIC", "-o", tmp, *objs]
