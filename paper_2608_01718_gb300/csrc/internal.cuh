@@ -136,6 +136,12 @@ cudaError_t launch_signatures(const __nv_bfloat16* rows, int64_t n, int d, const
                               int bits, uint32_t* sig, unsigned int* dev_status, EncodeTiledFn encode, int num_sms,
                               cudaStream_t st, bool rows_from_previous = false);
 
+// Query signatures of a batch of B < kLshTensorMinBatch queries on the CUDA cores, in the bit layout of
+// launch_signatures (one CTA per query and 32-bit word). q_from_previous: the queries are written by the grid
+// launched just before.
+cudaError_t launch_sign_queries(const __nv_bfloat16* q, int B, int d, const __nv_bfloat16* hyperplanes, int bits,
+                                uint32_t* qsig, cudaStream_t st, bool q_from_previous);
+
 // The SimHash-indexed key check: entries whose signature is within `radius` of the query's get the exact key
 // check (threshold + top-c partial lists, as the other stage-1 kernels).
 struct LshArgs {

@@ -266,7 +266,59 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
-// The scan is a programmatic dependent launch of the query-signature GEMM: its CTAs may be scheduled while the
+// Query signatures of a small batch on the CUDA cores. The tensor-core GEMM that signs entries at insert runs only
+// bits / 128 CTAs with a dozen dependent k-steps each, about 11.5 us whatever the batch; here one CTA per (query,
+// 32-hyperplane word) takes one memory round trip. Warp i computes hyperplanes 32w + 4i .. 32w + 4i + 3: lane l reads
+// the rows' 16-byte chunks l, l + 32, ... (coalesced), accumulates in fp32 (each lane's chunks in order), and a
+// butterfly reduce-scatter of the four sums leaves hyperplane 4i + l / 8's dot in lanes l. Bit h of word w is set
+// iff <hyperplane 32w + h, query> >= 0, as for the entries' signatures.
+__global__ void __launch_bounds__(256) sign_queries_kernel(const __nv_bfloat16* __restrict__ q, int d,
+                                                           const __nv_bfloat16* __restrict__ hyper, int words,
+                                                           uint32_t* __restrict__ qsig, int wait_first) {
+  __shared__ uint32_t part[8];
+  if (wait_first) asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int w = blockIdx.x % words, qi = blockIdx.x / words;
+  const int dc = d / 8;
+  const uint4* qrow = reinterpret_cast<const uint4*>(q + (int64_t)qi * d);
+  const uint4* hrow = reinterpret_cast<const uint4*>(hyper + (int64_t)(32 * w + 4 * warp) * d);
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+  for (int c = lane; c < dc; c += 32) {
+    const uint4 qv = __ldg(qrow + c);
+    uint4 hv[4];
+#pragma unroll
+    for (int h = 0; h < 4; ++h) hv[h] = __ldg(hrow + (int64_t)h * dc + c);
+#pragma unroll
+    for (int h = 0; h < 4; ++h) acc[h] = dot8(hv[h], qv, acc[h]);
+  }
+  // reduce-scatter of four values: after two halving steps lane l holds value l / 8's sum over 4 lanes, and three
+  // more steps add across the lanes that share it
+  const bool hi16 = (lane & 16) != 0, hi8 = (lane & 8) != 0;
+  float x0 = (hi16 ? acc[2] : acc[0]) + __shfl_xor_sync(kFull, hi16 ? acc[0] : acc[2], 16);
+  float x1 = (hi16 ? acc[3] : acc[1]) + __shfl_xor_sync(kFull, hi16 ? acc[1] : acc[3], 16);
+  float v = (hi8 ? x1 : x0) + __shfl_xor_sync(kFull, hi8 ? x0 : x1, 8);
+#pragma unroll
+  for (int o = 4; o >= 1; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  const unsigned ballot = __ballot_sync(kFull, (lane & 7) == 0 && v >= 0.f);
+  if (lane == 0) {
+    uint32_t b = 0;
+#pragma unroll
+    for (int h = 0; h < 4; ++h) b |= ((ballot >> (8 * h)) & 1u) << h;
+    part[warp] = b << (4 * warp);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    uint32_t word = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) word |= part[i];
+    asm volatile("griddepcontrol.wait;" ::: "memory");   // the previous lookup's scan has read qsig
+    qsig[(int64_t)qi * words + w] = word;
+  }
+}
+
+// The scan is a programmatic dependent launch of the query-signature kernel: its CTAs may be scheduled while the
 // signatures are computed and wait in griddepcontrol.wait, which hides the launch gap.
 template <int W>
 cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStream_t st) {
@@ -287,6 +339,21 @@ cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStre
 }
 
 }  // namespace
+
+cudaError_t launch_sign_queries(const __nv_bfloat16* q, int B, int d, const __nv_bfloat16* hyperplanes, int bits,
+                                uint32_t* qsig, cudaStream_t st, bool q_from_previous) {
+  const int words = bits / 32;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)(B * words));
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, sign_queries_kernel, q, d, hyperplanes, words, qsig, q_from_previous ? 1 : 0);
+}
 
 cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits, cudaStream_t st,
                               int* splits) {
