@@ -133,3 +133,16 @@ def test_a_missing_library_raises_instead_of_falling_back(monkeypatch, tmp_path)
         lacache.lacache_create(lacache.make_config(64, 8, 1024, 0.9, 0.8, 8, max_batch=16))
     with pytest.raises(RuntimeError, match="is missing"):
         lacache.status_string(lacache.LACACHE_OK)
+
+
+def test_candidate_packing_orders_scores_then_ids(tmp_path):
+    """The stage-1 kernels' packed (score, id) candidates, compiled for the host from the same header: their
+    unsigned order is (score descending, id ascending), and -0.0 ties with +0.0."""
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    src = os.path.join(root, "tests", "c_client", "pack_order_check.cu")
+    exe = tmp_path / "pack_order_check"
+    res = subprocess.run([build.nvcc(), "-std=c++17", "-I", os.path.join(root, "include"), "-I", build.CSRC,
+                          src, "-o", str(exe)], capture_output=True, text=True)
+    assert res.returncode == 0, res.stdout + res.stderr
+    run = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert run.returncode == 0, run.stderr
