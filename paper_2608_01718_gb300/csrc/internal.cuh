@@ -164,16 +164,20 @@ size_t lsh_index_bytes(int64_t capacity, int bits);
 cudaError_t launch_expand_signatures(const uint32_t* sig, int64_t first, int64_t n, int bits, uint8_t* index,
                                      int num_sms, cudaStream_t st);
 
-// LACACHE_STAGE1_AUTO's choice for a lookup of B queries against n keys of d elements. Once the keys stream from
-// HBM, the tensor-core scan holds the copy bandwidth at every batch size (measured 1.05-1.09 of it from 1 to 128
-// queries), and the streaming scan is level with it for one or two queries and slower from four. A store of at most
-// 32 MB of keys sits in L2 and the scan is bound by latency; there the streaming scan's stage 1 is the shorter one
-// for up to four queries (9.8 against 13.3 us at 4,096 x 768).
+// LACACHE_STAGE1_AUTO's choice for a lookup of B queries against n keys of d elements, from measurements of both
+// kernels. Once the keys stream from HBM, the tensor-core scan holds the copy bandwidth at every batch size (1.05-1.09
+// of it from 1 to 128 queries). The streaming scan matches or passes it for one or two queries at d = 1024, where
+// every lane has its whole share of a row, four 16-byte chunks, in flight per tile (585.6 against 590.9 us at
+// 2M x 1024 and one query), and falls behind with fewer chunks per lane, several phases or more queries (d = 800,
+// 896 and 1280 trail by 1-2 %). A store of at most 32 MB of keys sits in L2 and the scan is bound by
+// latency; there the streaming scan's stage 1 is the shorter one for up to four queries (10.1 against 13.3 us at
+// 4,096 x 768).
 constexpr int64_t kStreamAutoKeyBytes = (int64_t)32 << 20;
 constexpr int kStreamAutoMaxBatch = 4;
 inline int auto_stage1(int64_t n, int d, int B) {
-  return (B <= kStreamAutoMaxBatch && n * d * 2 <= kStreamAutoKeyBytes) ? LACACHE_STAGE1_STREAM
-                                                                        : LACACHE_STAGE1_TENSOR;
+  if (B <= kStreamAutoMaxBatch && n * d * 2 <= kStreamAutoKeyBytes) return LACACHE_STAGE1_STREAM;
+  if (B <= 2 && d == 1024) return LACACHE_STAGE1_STREAM;
+  return LACACHE_STAGE1_TENSOR;
 }
 
 // Largest split count the stage-1 launchers may use on a handle (sizes its partial-list scratch). The SimHash scan

@@ -100,12 +100,14 @@ def test_stream_query_groups_and_load_phases(d, batch):
 
 
 def test_auto_takes_the_stream_scan_only_for_small_batches_on_stores_l2_holds():
-    """LACACHE_STAGE1_AUTO: the streaming scan for at most 4 queries against at most 32 MB of keys, the tensor-core
-    scan otherwise (and its results agree with the explicit kernels')."""
+    """LACACHE_STAGE1_AUTO: the streaming scan for at most 4 queries against at most 32 MB of keys and for 1 or 2
+    queries at d = 1024, the tensor-core scan otherwise (and the oracle agrees with its results)."""
     small = wl.WORKLOADS["mid-1m"].scaled(n=10_000, batch=8)      # 15 MB of keys
     large = wl.WORKLOADS["mid-1m"].scaled(n=30_000, batch=8)      # 46 MB of keys
+    wide = wl.WORKLOADS["large-16m"].scaled(n=30_000, batch=8)    # d = 1024, 61 MB of keys
     for w, want in ((small, {1: L.LACACHE_STAGE1_STREAM, 4: L.LACACHE_STAGE1_STREAM, 5: L.LACACHE_STAGE1_TENSOR}),
-                    (large, {1: L.LACACHE_STAGE1_TENSOR, 4: L.LACACHE_STAGE1_TENSOR})):
+                    (large, {1: L.LACACHE_STAGE1_TENSOR, 4: L.LACACHE_STAGE1_TENSOR}),
+                    (wide, {1: L.LACACHE_STAGE1_STREAM, 2: L.LACACHE_STAGE1_STREAM, 3: L.LACACHE_STAGE1_TENSOR})):
         st = oracle_store(w)
         with new_cache(w, L.LACACHE_STAGE1_AUTO) as cache:
             fill(cache, w)
