@@ -4,24 +4,26 @@
 //
 // Warp per key tile. A warp takes KT consecutive keys at a time. Each key row is cut into 16-byte chunks (8 bf16),
 // and lane l owns chunks l, l + 32, l + 64, ...: for one key the 32 lanes read 512 contiguous bytes per 128-bit
-// load (ld.global.nc.v4), so every load instruction of the warp is fully coalesced. All KT x CPL loads of a tile are
-// issued before any arithmetic. The row goes in phases of PH chunks per lane, so KT x PH 128-bit loads (32
-// registers, 4 KB per warp, 64 KB per SM) are in flight together and the rest of the register budget holds the sums.
+// load (ld.global.nc.v4), so every load instruction of the warp is fully coalesced. The row goes in phases of PH
+// chunks per lane, and all KT x PH loads of a phase are issued before any arithmetic. For one or two queries a phase
+// is a whole row of up to 1024 elements (KT = 4 keys x PH = 4 chunks: 16 loads, 8 KB per warp in flight; KT = 8 for
+// rows of at most 512 elements and one query); for 4 or 8 queries, 8 loads per phase, leaving registers for the sums.
 //
 // The queries of the launch sit in shared memory as fp32, split into the low and high halves of each chunk, so
 // that lane l's reads of chunk l are contiguous across the warp (conflict-free 128-bit loads). They are taken QB
 // at a time (a query group); each lane converts its key chunks to fp32 once per group and accumulates element
 // pairs with packed fp32 FMAs (fma.rn.f32x2) into KT x QB partial sums.
 //
-// Reduction: one butterfly reduce-scatter over the warp turns the 32 lanes' KT x QB partials into full scores, lane
-// l ending with score (key l / (32 / (KT QB)) / QB, query ... % QB): KT QB - 1 shuffles instead of 5 per score.
-// Every score is summed in the same order (each lane's chunks in order, then the same butterfly tree), so equal
-// keys give bit-equal scores.
+// Reduction: one butterfly reduce-scatter over the warp turns the 32 lanes' V = KT x QB partials into full scores:
+// lane l ends with value v = l / (32 / V), i.e. key v / QB of the tile and query v % QB of the group, after V - 1 +
+// log2(32 / V) shuffles instead of 5 per score. Every score is summed in the same order (each lane's chunks in
+// order, then the same butterfly tree), so equal keys give bit-equal scores.
 //
 // Threshold + top_c: every warp keeps, per query, a sorted list of packed (score, id) candidates in shared memory
 // and a running threshold max(tau_c, c-th best). A lane whose score clears it inserts, one lane at a time
 // (ballot order); the packed order makes the list independent of the order of arrival. At the end the CTA merges its
-// warps' lists into the split's partial list. Grid: one CTA of 16 warps per SM, each CTA one split of the key range.
+// warps' lists into the split's partial list (a record of its best score and candidate count, then the candidates).
+// Grid: one CTA of 16 warps per SM, each CTA one contiguous split of the key range.
 #include "internal.cuh"
 
 namespace lc {
