@@ -30,12 +30,15 @@ def library():
     L.load()
 
 
-def _check_streamed(w, per_class):
+def _check_streamed(w, per_class, pairs_of_queries=False):
+    """The full-size lookup of the whole batch (AUTO: the tensor-core scan), and with pairs_of_queries the same
+    queries looked up two at a time (AUTO: the streaming scan at d = 1024), against the streamed oracle."""
     q = wl.batch(w, 0, device="cuda")
     sample = stratified_sample(q["class"], per_class)
     p = params(w)
     so = StreamedOracle(w, q, sample, p)
-    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+    small = None
+    with new_cache(w, L.LACACHE_STAGE1_AUTO) as cache:
         so.fill(cache)
         assert cache.size == w.n
         out = cache.lookup(q["emb"], q["prefix"], q["ids"])
@@ -44,9 +47,22 @@ def _check_streamed(w, per_class):
         # batches of more than one query tile run on CTA pairs
         assert cache.last_launch()[1] == (L.LACACHE_STAGE1_TENSOR_PAIR if w.batch > 128 else L.LACACHE_STAGE1_TENSOR)
         g = {k: v.cpu().numpy() for k, v in out.items()}
+        if pairs_of_queries:
+            parts = []
+            for i in range(0, w.batch, 2):
+                qq = {k: q[k][i:i + 2].contiguous() for k in ("emb", "prefix", "ids")}
+                parts.append(cache.lookup(qq["emb"], qq["prefix"], qq["ids"]))
+                assert cache.last_launch()[1] == L.LACACHE_STAGE1_STREAM
+            torch.cuda.synchronize()
+            cache.sync()
+            small = {k: torch.cat([o[k] for o in parts]).cpu().numpy() for k in parts[0]}
     res = so.result()
     rep = compare(g, res, p, rows=sample, pair_scores=so.pair_scores)
     log_report(f"{w.name} full size, sampled", rep)
+    if small is not None:
+        rep2 = compare(small, res, p, rows=sample, pair_scores=so.pair_scores)
+        log_report(f"{w.name} full size, two queries per lookup (streaming scan)", rep2)
+        assert rep2.exact + rep2.band == len(sample) and rep2.band <= max(1, len(sample) // 50)
     assert rep.exact + rep.band == len(sample)
     assert rep.band <= max(1, len(sample) // 50)
     assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
@@ -60,7 +76,7 @@ def _check_streamed(w, per_class):
 
 def test_large_cache_near_hbm_capacity():
     """16,777,216 entries x 1024 dims (34 GB of keys), B = 128, Zipf(1.1) targets: every query of the batch."""
-    rep = _check_streamed(wl.WORKLOADS["large-16m"], per_class=128)
+    rep = _check_streamed(wl.WORKLOADS["large-16m"], per_class=128, pairs_of_queries=True)
     assert rep.queries == 128
 
 
