@@ -46,6 +46,9 @@ MUTATIONS = [
      "res.prefix_score[b] = r[0]", PINS),
     ("margin-drops-threshold-gap", "lookup.py", "gaps.append(cs[served] - tau_c)",
      "gaps.append(np.inf)", PINS),
+    ("literal-margin-drops-top-two-gap", "lookup.py", "lit.append(s_sorted[0] - s_sorted[1])", "pass", PINS),
+    ("literal-margin-drops-threshold-distance", "lookup.py",
+     "lit = [abs(kc.best[b] - tau_c)] if np.isfinite(kc.best[b]) else []", "lit = []", PINS),
     ("margin-push-out-only-from-the-last-slot", "lookup.py",
      "            if n_above > c:\n                # j* pushed past the cut",
      "            if n_above > c and served == c - 1:\n                # j* pushed past the cut", PINS),

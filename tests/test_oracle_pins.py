@@ -251,6 +251,29 @@ def test_margin_terms():
     assert r.status[0] == HIT and r.margin[0] == 1.0 - 0.984375
 
 
+def test_literal_margin_is_the_threshold_distance_or_the_top_two_gap():
+    """The north-star's literal band: min(|best score - tau_c|, s_(1) - s_(2)), from dyadic scores."""
+    q = np.array([1.0, 0, 0, 0])
+    keys = [[0.875, 0, 0, 0], [0.75, 0, 0, 0], [0.5, 0, 0, 0]]
+    st = store_of(keys, [E[1]] * 3, [[0]] * 3)
+    # best 0.875 is 0.125 above tau_c = 0.75; the top two (0.875, 0.75) are 0.125 apart: both terms 0.125
+    r = oracle.lookup(st, queries_of(q, E[1], [0]), Params(0.75, 0.5, 2))
+    assert r.literal_margin[0] == 0.125
+    # tau_c = 0.8125: the best is 0.0625 above it; only one entry clears it, so no top-two gap
+    r = oracle.lookup(st, queries_of(q, E[1], [0]), Params(0.8125, 0.5, 2))
+    assert r.n_above[0] == 1 and r.literal_margin[0] == 0.0625
+    # tau_c = 0.25: the best is 0.625 above it, and the top-two gap 0.125 is smaller
+    r = oracle.lookup(st, queries_of(q, E[1], [0]), Params(0.25, 0.5, 3))
+    assert r.literal_margin[0] == 0.125
+    # nothing clears tau_c = 0.9375: the distance of the best score (0.875) below it
+    r = oracle.lookup(st, queries_of(q, E[1], [0]), Params(0.9375, 0.5, 2))
+    assert r.status[0] == MISS_KEY and r.literal_margin[0] == 0.0625
+    # an empty cache has no score at all: no band
+    empty = Store.of(np.zeros((0, 4), np.uint16), np.zeros((0, 4), np.uint16), np.zeros((0, 1), np.int32))
+    r = oracle.lookup(empty, queries_of(q, E[1], [0]), Params(0.5, 0.5, 2))
+    assert r.literal_margin[0] == math.inf
+
+
 def test_margin_counts_changes_from_outside_the_examined_candidates():
     q = np.array([1.0, 0, 0, 0])
     # a passing entry just past the cut could rise above the served entry and be served instead
