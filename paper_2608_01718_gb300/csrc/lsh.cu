@@ -204,26 +204,28 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
       for (int w = 0; w < W; ++w) e[w] = nxt[w];
       load_sig<W>(l.sig, j + kTile, j_end, nxt);
       // every query's distance first, as a mask of the admitted queries (the queue stores below could alias the
-      // query signatures for the compiler); groups of 8 queries, as many as the pass has (the padding rows of the
-      // last group are masked out below)
+      // query signatures for the compiler): whole groups of 8 queries unrolled, then the pass's remaining queries
+      // (a uniform count), so a pass of one query computes one distance
       unsigned pend = 0;
-      for (int g = 0; g < qn; g += 8) {
+      auto test_query = [&](int qq) {
+        const uint4* qs = reinterpret_cast<const uint4*>(sh.qsig[qq]);
+        uint32_t x[W];
 #pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int qq = g + u;
-          const uint4* qs = reinterpret_cast<const uint4*>(sh.qsig[qq]);
-          uint32_t x[W];
-#pragma unroll
-          for (int w = 0; w < W / 4; ++w) {
-            const uint4 v = qs[w];
-            x[4 * w] = e[4 * w] ^ v.x;
-            x[4 * w + 1] = e[4 * w + 1] ^ v.y;
-            x[4 * w + 2] = e[4 * w + 2] ^ v.z;
-            x[4 * w + 3] = e[4 * w + 3] ^ v.w;
-          }
-          pend |= (hamming<W>(x) <= l.radius ? 1u : 0u) << qq;
+        for (int w = 0; w < W / 4; ++w) {
+          const uint4 v = qs[w];
+          x[4 * w] = e[4 * w] ^ v.x;
+          x[4 * w + 1] = e[4 * w + 1] ^ v.y;
+          x[4 * w + 2] = e[4 * w + 2] ^ v.z;
+          x[4 * w + 3] = e[4 * w + 3] ^ v.w;
         }
+        pend |= (hamming<W>(x) <= l.radius ? 1u : 0u) << qq;
+      };
+      const int whole = qn & ~7;
+      for (int g = 0; g < whole; g += 8) {
+#pragma unroll
+        for (int u = 0; u < 8; ++u) test_query(g + u);
       }
+      for (int qq = whole; qq < qn; ++qq) test_query(qq);
       pend = j < j_end ? pend & qmask : 0u;
       // Queue the admitted pairs; flush while the queue is past kFlushAt or a pair found it full. Every round of
       // this loop either queues all pending pairs or fills the queue, so it ends.
