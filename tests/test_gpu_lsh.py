@@ -55,10 +55,12 @@ def _expected_lsh_kernel(batch):
     return L.LACACHE_STAGE1_LSH_TENSOR if batch >= 40 else L.LACACHE_STAGE1_LSH
 
 
+# popcount-1 / -2: a pass of fewer queries than one group of 8 (only their distances are computed);
 # popcount-36: two passes of 32 queries (the handle's max_batch is below the tensor scan's minimum, so it keeps no
 # expanded index); tensor-200: two passes of 128 queries at 128 and 256 bits, four of 64 at 512, ragged last pass
-@pytest.mark.parametrize("batch", [5, 32, 36, 40, 64, 200],
-                         ids=["popcount-5", "popcount-32", "popcount-36", "tensor-40", "tensor-64", "tensor-200"])
+@pytest.mark.parametrize("batch", [1, 2, 5, 32, 36, 40, 64, 200],
+                         ids=["popcount-1", "popcount-2", "popcount-5", "popcount-32", "popcount-36", "tensor-40",
+                              "tensor-64", "tensor-200"])
 @pytest.mark.parametrize("bits", [128, 256, 512])
 def test_lsh_lookup_matches_the_oracle(bits, batch):
     _check_lsh_lookup(wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch), bits)

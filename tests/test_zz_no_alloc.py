@@ -86,6 +86,23 @@ def test_noalloc_modes_and_list_sizes(mode, tmin, top_c, stage1):
             _same(out, ref)
 
 
+def test_noalloc_auto_on_a_small_store_takes_the_streaming_scan():
+    """AUTO chooses as for a handle: two queries against 15 MB of keys take the streaming scan, in both entry
+    points, and give the same results."""
+    w = wl.WORKLOADS["mid-1m"].scaled(n=10_000, batch=2)
+    key, pre, ids = _rows(w)
+    with L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch) as cache:
+        cache.insert(key, pre, ids)
+        for step in (0, 1):
+            q = wl.batch(w, step, device="cuda")
+            ref = cache.lookup(q["emb"], q["prefix"], q["ids"])
+            assert cache.last_launch()[1] == L.LACACHE_STAGE1_STREAM
+            out = L.alloc_result(w.batch, w.top_c, "cuda")
+            L.lacache_lookup_noalloc(cache.cfg, key, pre, ids, q["emb"], q["prefix"], q["ids"], out)
+            torch.cuda.synchronize()
+            _same(out, ref)
+
+
 def _empty_batch(B, d, k):
     g = torch.Generator(device="cuda").manual_seed(B)
     q = torch.randn((B, d), generator=g, device="cuda").to(torch.bfloat16)
