@@ -337,12 +337,13 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
       e = lc::launch_stage1_tensor(a, h->encode, h->num_sms, h->max_splits, st, &splits, &paired);
       if (paired) kernel = LACACHE_STAGE1_TENSOR_PAIR;
     } else if (kernel == LACACHE_STAGE1_LSH) {
-      // the popcount scan's small batches sign their queries on the CUDA cores; the tensor-core scan's batches of
-      // 40 and more with the tensor-core GEMM that signs the entries
-      const bool tc_scan = B >= lc::kLshTensorMinBatch && h->sig_index;
-      e = tc_scan ? lc::launch_signatures(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, h->dev_status, h->encode,
-                                          h->num_sms, st, gathered)
-                  : lc::launch_sign_queries(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, st, gathered);
+      // batches of up to kSignCudaCoreMaxBatch queries are signed on the CUDA cores (one CTA per query and word,
+      // about one memory round trip), larger ones by the tensor-core GEMM that signs the entries: the CUDA-core
+      // kernel reads each 32-hyperplane block once per query, which costs more than the GEMM beyond that
+      e = B > lc::kSignCudaCoreMaxBatch
+              ? lc::launch_signatures(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, h->dev_status, h->encode,
+                                      h->num_sms, st, gathered)
+              : lc::launch_sign_queries(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, st, gathered);
       if (e == cudaSuccess) {
         lc::LshArgs l{h->sig, h->qsig, h->lsh_bits / 32, h->lsh_radius, h->sig_index};
         if (B >= lc::kLshTensorMinBatch && h->sig_index) {
