@@ -8,8 +8,10 @@ A step is one lookup: stage 1 (key check with fused threshold + top-c) and stage
 decision) for one batch of B synthetic queries against a resident cache of N entries. The default workload is the
 largest single-GPU one: 16,777,216 entries of d = 1024 (34.4 GB of keys, 69.8 GB of store) and batches of 128
 queries. The inputs are resident in HBM before timing starts. Every step reads the whole key store, far larger
-than L2, so no L2 flush is needed between steps. The device time is taken with CUDA events on the launching
-stream, between barriers, as the max over ranks.
+than L2, so no L2 flush is needed between steps. Where a step streams less than twice the L2 (the SimHash index of a
+1M-entry store, a 4k-entry store), a write of four times the L2 runs between timed steps, every step is timed on its
+own and the end-to-end calls are timed one by one after a flush (`L2Flush`). The device time is taken with CUDA
+events on the launching stream, between barriers, as the max over ranks.
 
 With N > 1 GPUs, one process runs per GPU. Under torchrun (WORLD_SIZE set) this script is one of the ranks;
 otherwise `--gpus N` builds the library once and starts N ranks through torch.distributed.run itself. Every rank
@@ -89,6 +91,53 @@ def peaks_lib():
     lib.lcpeaks_popc.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_void_p, ctypes.c_int,
                                  ctypes.c_void_p]
     return lib
+
+
+class L2Flush:
+    """Keeps a step's inputs out of L2 between timed steps when they would fit in it. A step that streams fewer
+    than twice the L2's bytes (streamed_bytes) gets a write of four times the L2 before it: a fill of a device
+    buffer, on the current stream, outside the step's own events. Otherwise the flush does nothing."""
+
+    def __init__(self, streamed_bytes: int, what: str):
+        import torch
+        props = torch.cuda.get_device_properties(torch.cuda.current_device())
+        self.l2 = int(getattr(props, "L2_cache_size", 0) or 129 * 10**6)
+        self.on = streamed_bytes < 2 * self.l2
+        self.buf = torch.empty(4 * self.l2, dtype=torch.uint8, device="cuda") if self.on else None
+        self.fills = 0
+        self.note = (f"flush: the {what} read per step ({streamed_bytes / 1e6:.1f} MB) fit in the "
+                     f"{self.l2 / 1e6:.0f} MB L2, so a {4 * self.l2 / 1e6:.0f} MB write runs before every timed step "
+                     "(outside its events) and before every timed end-to-end call (outside its clock)"
+                     if self.on else
+                     f"no flush: the {what} read per step ({streamed_bytes / 1e9:.2f} GB) exceed twice the "
+                     f"{self.l2 / 1e6:.0f} MB L2")
+
+    def __call__(self):
+        if self.on:
+            self.fills += 1
+            self.buf.fill_(self.fills & 0xFF)
+
+
+def device_steps_ms(step, steps: int, stream, flush: L2Flush) -> float:
+    """Device time (ms) of steps 0 .. steps-1 on `stream`: one event pair around the whole loop, or, with the L2
+    flush on, one pair around each step with the flush between them, summed."""
+    import torch
+    if not flush.on:
+        ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        ev0.record(stream)
+        for i in range(steps):
+            step(i)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        return ev0.elapsed_time(ev1)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for i in range(steps):
+        flush()
+        evs[i][0].record(stream)
+        step(i)
+        evs[i][1].record(stream)
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in evs)
 
 
 def timed_best(launch, reps: int = 5) -> float:
@@ -306,7 +355,8 @@ def run_reference(args, w):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(w) | {"parallelism": "single"},
+            "config": workload_config(w) | {"parallelism": "single",
+                                            "l2": "not applicable: the oracle runs on the host cores"},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -336,7 +386,6 @@ def workload_config(w):
     else:
         cfg |= {"prefix_dims": list(w.prefix_dims), "tau_a_models": list(w.tau_a_models),
                 "mix_near_random_collision_mimic": list(w.mix)}
-    cfg["l2"] = f"no flush: the keys read per step ({w.n * w.d * 2 / 1e9:.2f} GB) exceed the 129 MB L2"
     return cfg
 
 
@@ -400,28 +449,29 @@ def run_ours(args, w):
     kernel_name = {L.LACACHE_STAGE1_TENSOR: "tensor", L.LACACHE_STAGE1_TENSOR_PAIR: "tensor-pair",
                    L.LACACHE_STAGE1_STREAM: "stream", L.LACACHE_STAGE1_LSH: "lsh",
                    L.LACACHE_STAGE1_LSH_TENSOR: "lsh-tensor"}[cache.last_launch()[1]]
+    # what a step streams: the SimHash index (bits / 8 bytes an entry for the popcount scan, bits bytes for the
+    # tensor-core scan's expanded copy) or the keys
+    if lsh:
+        flush = L2Flush(w.n * lsh["bits"] // (1 if kernel_name == "lsh-tensor" else 8), "SimHash index bytes")
+    else:
+        flush = L2Flush(w.n * w.d * 2, "keys")
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     clocks = ClockSampler(torch.cuda.current_device())
     clocks.start()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    ev0.record(stream)
-    for i in range(args.steps):
-        serve_step(warm + i) if serve else step(i)
-    ev1.record(stream)
-    torch.cuda.synchronize()
+    elapsed_ms = device_steps_ms(lambda i: serve_step(warm + i) if serve else step(i), args.steps, stream, flush)
     if world > 1:
         dist.barrier()
     clock = clocks.stop()
     cache.sync()
-    elapsed_ms = ev0.elapsed_time(ev1)
     n_timed_end = cache.size
     # Second pass over the same steps with the library's stage events (recorded on the lookup's stream around
     # each kernel) for the per-kernel times of the roofline. The events sit between the two kernels, so this pass
     # is kept out of the throughput measurement above.
     L.lacache_stage_timing(cache.h, args.steps)
     for i in range(args.steps):
+        flush()
         step(i)
     t1_ms, t2_ms, timed = L.lacache_stage_times(cache.h)
     L.lacache_stage_timing(cache.h, 0)
@@ -459,19 +509,27 @@ def run_ours(args, w):
             raise RuntimeError("lacache_lookup_host_async failed")
         return served
 
-    def run_sync(n: int) -> None:
-        bad = 0
+    def run_sync(n: int) -> float:
+        """Seconds of n synchronous calls; with the L2 flush on, each call is timed alone after a flush that has
+        finished, and the calls' times are summed."""
+        bad, total = 0, 0.0
+        t0 = time.perf_counter()
         for i in range(n):
+            if flush.on:
+                flush()
+                torch.cuda.synchronize()
+                t0 = time.perf_counter()
             bad |= lib.lacache_lookup_host(*calls[i % nb][i % depth])
+            if flush.on:
+                total += time.perf_counter() - t0
         if bad:
             raise RuntimeError("lacache_lookup_host failed")
+        return total if flush.on else time.perf_counter() - t0
 
     run_sync(max(3, args.warmup))
     if world > 1:
         dist.barrier()
-    t0 = time.perf_counter()
-    run_sync(args.e2e_steps)
-    e2e_sync_s = time.perf_counter() - t0
+    e2e_sync_s = run_sync(args.e2e_steps)
     sync_status = [o["status"].clone() for o in hout]
     run_async(max(3, args.warmup))
     if world > 1:
@@ -479,6 +537,11 @@ def run_ours(args, w):
     t0 = time.perf_counter()
     run_async(args.e2e_steps)
     e2e_s = time.perf_counter() - t0
+    if flush.on:
+        # the pipelined loop overlaps calls, so a flush between them cannot be kept out of its clock: the
+        # end-to-end figure is then the synchronous calls', each from a flushed L2 (the loop above still checks
+        # that pipelined lookups decide as the synchronous ones)
+        e2e_s = e2e_sync_s
     # both timed loops ran the same e2e_steps steps, so each output slot's last batch is the same in both: the
     # pipelined lookups must have written the same decisions as the synchronous ones
     for slot in range(depth):
@@ -547,7 +610,8 @@ def run_ours(args, w):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": workload_config(w) | {"parallelism": f"replicas{world}" if world > 1 else "single"} |
+        "config": workload_config(w) | {"parallelism": f"replicas{world}" if world > 1 else "single",
+                                        "l2": flush.note} |
                   ({"serve_loop": {"steps_timed": args.steps, "entries_at_start": n_timed_begin,
                                    "entries_at_end": n_timed_end,
                                    "step": "lookup, then append of the batch's misses (lacache_append_misses)"}}
@@ -565,7 +629,9 @@ def run_ours(args, w):
         "stage_ms": {"stage1": t1_ms / max(1, timed), "stage2": t2_ms / max(1, timed), "timed_lookups": timed},
         "e2e": {"value": job["e2e_value"], "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": args.e2e_steps,
-                "api": f"lacache_lookup_host_async (mapped pinned host buffers, {depth} lookups in flight)"},
+                "api": ("lacache_lookup_host (pinned host buffers, one synchronous call per step, each timed alone "
+                        "after an L2 flush)") if flush.on else
+                       f"lacache_lookup_host_async (mapped pinned host buffers, {depth} lookups in flight)"},
         "e2e_sync": {"value": sync_job["e2e_value"], "unit": UNIT, "steps": args.e2e_steps,
                      "api": "lacache_lookup_host (pinned host buffers, one synchronous call per step)"},
         "gpu_launches": ((3 if lsh else 2) + (2 if serve else 0)) * args.steps,
@@ -672,24 +738,20 @@ def run_sharded(args, w):
         step(i)
     torch.cuda.synchronize()
     cache.sync()
+    flush = L2Flush(max(1, b - a) * w.d * 2, "shard's keys")
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
     clocks = ClockSampler(torch.cuda.current_device())
     clocks.start()
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    ev0.record(stream)
-    for i in range(args.steps):
-        step(i)
-    ev1.record(stream)
-    torch.cuda.synchronize()
+    elapsed_ms = device_steps_ms(step, args.steps, stream, flush)
     if world > 1:
         dist.barrier()
     clock = clocks.stop()
     cache.sync()
-    elapsed_ms = ev0.elapsed_time(ev1)
     L.lacache_stage_timing(cache.h, args.steps)
     for i in range(args.steps):
+        flush()
         step(i)
     t1_ms, t2_ms, timed = L.lacache_stage_times(cache.h)
     L.lacache_stage_timing(cache.h, 0)
@@ -713,10 +775,18 @@ def run_sharded(args, w):
         e2e_step(i)
     if world > 1:
         dist.barrier()
+    e2e_s = 0.0
     t0 = time.perf_counter()
     for i in range(args.e2e_steps):
+        if flush.on:   # each synchronous step timed alone after a finished flush
+            flush()
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
         e2e_step(i)
-    e2e_s = time.perf_counter() - t0
+        if flush.on:
+            e2e_s += time.perf_counter() - t0
+    if not flush.on:
+        e2e_s = time.perf_counter() - t0
     times = torch.tensor([elapsed_ms, e2e_s], dtype=torch.float64, device="cuda")
     if world > 1:
         dist.all_reduce(times, op=dist.ReduceOp.MAX)
@@ -740,7 +810,8 @@ def run_sharded(args, w):
         "metric": METRIC, "value": w.batch * args.steps / (elapsed_ms / 1e3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": elapsed_ms / args.steps,
         "higher_is_better": True, "scaling": "strong", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-        "config": workload_config(w) | {"parallelism": f"entry-shards{world}", "shard_entries": b - a},
+        "config": workload_config(w) | {"parallelism": f"entry-shards{world}", "shard_entries": b - a,
+                                        "l2": flush.note},
         "stage1_kernel": kernel_name,
         "roofline": roof | {"traffic": None, "kernel": f"stage1_{kernel_name} (one shard)",
                             "algorithmic_bytes_per_launch": s1_bytes, "algorithmic_flops_per_launch": flops,
