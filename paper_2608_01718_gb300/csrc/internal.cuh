@@ -171,9 +171,10 @@ cudaError_t launch_expand_signatures(const uint32_t* sig, int64_t first, int64_t
 // of it from 1 to 128 queries). The streaming scan matches or passes it for one or two queries at d = 1024, where
 // every lane has its whole share of a row, four 16-byte chunks, in flight per tile (585.6 against 590.9 us at
 // 2M x 1024 and one query), and falls behind with fewer chunks per lane, several phases or more queries (d = 800,
-// 896 and 1280 trail by 1-2 %). A store of at most 32 MB of keys sits in L2 and the scan is bound by
-// latency; there the streaming scan's stage 1 is the shorter one for up to four queries (10.1 against 13.3 us at
-// 4,096 x 768).
+// 896 and 1280 trail by 1-2 %). On a store of at most 32 MB of keys the scan is bound by latency; there the
+// streaming scan's stage 1 is the shorter one for up to four queries, with the keys left in L2 by the previous
+// lookup (10.1 against 13.3 us at 4,096 x 768) and from a flushed L2 (10.0 against 14.3 us; 22.3 against 25.9 us at
+// 43,690 x 768).
 constexpr int64_t kStreamAutoKeyBytes = (int64_t)32 << 20;
 constexpr int kStreamAutoMaxBatch = 4;
 inline int auto_stage1(int64_t n, int d, int B) {
