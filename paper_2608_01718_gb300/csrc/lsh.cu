@@ -1,9 +1,16 @@
 // Stage 1 through the SimHash index (Eq. 1; Algorithm 1's "search semantic cache with key h(x)"): the key check
 // sim(x, x') >= tau_c applied only to the entries whose signature is within `radius` bits of the query's.
 //
-// One CTA per contiguous split of the entries (two per SM); one entry per thread per tile of 512. A thread loads
-// its entry's signature (16-byte loads, one tile ahead, into registers) and counts the differing bits against each
-// of up to 32 query signatures held in shared memory. Admitted (query, entry) pairs are queued in shared memory.
+// One CTA per contiguous split of the entries (two per SM); one entry per thread per tile of 512. A thread counts
+// the differing bits of its entry's signature against each of up to 32 query signatures held in shared memory. The
+// signatures arrive in one of two ways (bulk_ring() picks one per launch):
+//  - registers: each thread loads its entry's words with 16-byte loads one tile ahead. The fewest instructions
+//    around the distance arithmetic, so the form for the ALU-bound scans (several queries at 128 or 256 bits).
+//  - a ring of tile-sized shared-memory stages, one bulk copy (cp.async.bulk) per tile, issued by thread 0 and
+//    completed on the stage's mbarrier; a stage is refilled after the tile's CTA barrier, so kStages - 1 tiles are
+//    in flight while one is counted. Twice the bytes in flight, and W registers free: the form for the scans bound
+//    by memory (one query on a large store) and for 512-bit signatures.
+// Admitted (query, entry) pairs are queued in shared memory.
 // When the queue passes three quarters of its capacity, and at the end of the split, all warps take queue items two
 // at a time and compute the exact fp32 score over the gathered key row (each lane's 8-element chunks in order,
 // then a butterfly sum). The warp of each query then folds the scores that clear tau_c into that query's top-c
@@ -11,6 +18,7 @@
 // that finds the queue full stays in its thread's pending mask and is queued again after the next flush. The
 // partial lists have the format of the other stage-1 kernels, so stage 2 is shared.
 #include "internal.cuh"
+#include "tcgen05.cuh"
 
 namespace lc {
 namespace {
@@ -19,9 +27,19 @@ constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
 constexpr int kTile = kThreads;     // entries per tile, one per thread
 constexpr int kQC = 32;             // queries per pass over the entries (one bit each in a thread's masks)
-constexpr int kCap = 8192;          // queue capacity
-constexpr int kFlushAt = kCap - kCap / 4;   // a tile that leaves more items than this is followed by a flush
 constexpr unsigned kFull = 0xffffffffu;
+
+// Per signature width (W words) and form: the queue capacity and the depth of the signature ring. Two CTAs share an
+// SM's 228 KB. Without a ring the queue takes 8,192 items (12 bytes each); with one, the queue and the ring
+// (kTile * W * 4 bytes a stage: 8 / 16 / 32 KB at W = 4 / 8 / 16) split about 100 KB, and kStages - 1 tiles, 40 /
+// 32 / 32 KB, are in flight per CTA while one is counted.
+template <int W, bool Bulk>
+struct Geo {
+  static constexpr int kCap = !Bulk ? 8192 : W == 16 ? 2048 : 4096;
+  static constexpr int kStages = !Bulk ? 1 : W == 4 ? 6 : W == 8 ? 3 : 2;
+  static constexpr int kFlushAt = kCap - kCap / 4;   // a tile that leaves more items than this is followed by a flush
+  static constexpr int kRingWords = Bulk ? kTile * W : 4;   // a stage (a placeholder without the ring)
+};
 
 struct Item {
   int32_t j;      // entry id
@@ -47,19 +65,26 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// The ring and the query signatures are read as 16-byte vectors (and the ring is a bulk-copy destination), so
+// both sit on 16-byte boundaries (checked in launch_w).
+template <int W, bool Bulk>
 struct Shared {
-  uint32_t qsig[kQC][16];
+  using G = Geo<W, Bulk>;
+  alignas(16) uint32_t ring[G::kStages][G::kRingWords];   // entry t of a tile at words [t W, t W + W) of its stage
+  alignas(16) uint32_t qsig[kQC][W];
+  uint64_t bar[G::kStages];       // stage full: thread 0's arrive with the bytes, then the copy's
   uint64_t list[kQC][kMaxTopC];   // per query: sorted packed candidates of this split, 0 = empty
   unsigned int best[kQC];         // score_order of the best admitted score
   int count;                      // queued items
-  Item items[kCap];
-  float score[kCap];
+  Item items[G::kCap];
+  float score[G::kCap];
 };
 
 // Exact scores of the queued items, then each query's warp folds its items into the query's list.
-__device__ void flush(Shared& sh, const Stage1Args& a, int q0, int qn) {
+template <int W, bool Bulk>
+__device__ void flush(Shared<W, Bulk>& sh, const Stage1Args& a, int q0, int qn) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int total = min(sh.count, kCap);   // pairs that found the queue full were not stored
+  const int total = min(sh.count, Geo<W, Bulk>::kCap);   // pairs that found the queue full were not stored
   const int v = a.d / 8;
   for (int base = warp * 2; base < total; base += kWarps * 2) {
     float acc0 = 0.f, acc1 = 0.f;
@@ -174,16 +199,55 @@ __device__ __forceinline__ void load_sig(const uint32_t* sig, int64_t j, int64_t
   }
 }
 
+// Thread 0: tile `ti` of the split (entries j_begin + ti * kTile ..., at most j_end) into stage `st`, as one bulk
+// copy completing on the stage's barrier. The split's signatures are contiguous and 16-byte aligned (W >= 4 words an
+// entry), and a tile's byte count is a multiple of 16.
 template <int W>
+__device__ __forceinline__ void fetch_tile(Shared<W, true>& sh, const uint32_t* sig, int64_t j_begin, int64_t j_end,
+                                           int64_t ti, int st) {
+  const int64_t t0 = j_begin + ti * kTile;
+  const uint32_t bytes = (uint32_t)min((int64_t)kTile, j_end - t0) * W * 4;
+  const uint32_t bar = smem_u32(&sh.bar[st]);
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // the stage's last generic reads come first
+  mbar_expect_tx(bar, bytes);
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
+               ::"r"(smem_u32(sh.ring[st])), "l"(sig + t0 * W), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
+template <int W, bool Bulk>
 __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, LshArgs l, int splits) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  Shared& sh = *reinterpret_cast<Shared*>(smem_raw);
+  using G = Geo<W, Bulk>;
+  Shared<W, Bulk>& sh = *reinterpret_cast<Shared<W, Bulk>*>(smem_raw);
+  constexpr int S = G::kStages;
+  if (Bulk && threadIdx.x == 0) {
+    for (int st = 0; st < S; ++st) mbar_init(smem_u32(&sh.bar[st]), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const int s = blockIdx.x;
   const int64_t j_begin = a.n * s / splits, j_end = a.n * (s + 1) / splits;
+  const int64_t tiles = (j_end - j_begin + kTile - 1) / kTile;
   const int C = a.top_c;
+  // Ring form: stage uses are numbered across the passes: use u sits in stage u % S, and its copy completes the stage
+  // barrier's phase of parity (u / S) & 1. A thread whose wait for a tile runs out (about a second) records the
+  // timeout and reads no further tiles, but keeps to the CTA's barriers, so every pass still ends and writes its
+  // lists (the host reads the timeout from the status word). Thread 0 then issues no further copies and, before the
+  // CTA exits, waits (again with a limit) for the copies it had issued past the tile it gave up on.
+  uint32_t u0 = 0;           // first use of this pass
+  bool live = true;
+  int64_t issued = 0;        // thread 0: copies issued in this pass
+  uint32_t drain_first = 0;  // thread 0, once it gave up: the first use still in flight, and how many
+  int64_t drain_count = 0;
   for (int q0 = 0; q0 < a.B; q0 += kQC) {
     const int qn = min(kQC, a.B - q0);
+    if constexpr (Bulk) {
+      if (threadIdx.x == 0 && live) {
+        for (issued = 0; issued < min((int64_t)S, tiles); ++issued)
+          fetch_tile<W>(sh, l.sig, j_begin, j_end, issued, (int)((u0 + issued) % S));
+      }
+    }
     for (int i = threadIdx.x; i < kQC * W; i += kThreads) {
       const int qq = i / W;
       sh.qsig[qq][i % W] = qq < qn ? l.qsig[(int64_t)(q0 + qq) * W + i % W] : 0u;
@@ -192,17 +256,43 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
     if (threadIdx.x < kQC) sh.best[threadIdx.x] = score_order(-INFINITY);
     if (threadIdx.x == 0) sh.count = 0;
     __syncthreads();
-    // The next tile's signatures are loaded before the current tile is counted, so the load latency is hidden
-    // behind the popcounts.
-    uint32_t nxt[W];
-    load_sig<W>(l.sig, j_begin + threadIdx.x, j_end, nxt);
     const unsigned qmask = qn >= 32 ? kFull : (1u << qn) - 1u;
-    for (int64_t t0 = j_begin; t0 < j_end; t0 += kTile) {
-      const int64_t j = t0 + threadIdx.x;
+    // register form: the next tile's signatures are loaded before the current tile is counted
+    uint32_t nxt[W];
+    if constexpr (!Bulk) load_sig<W>(l.sig, j_begin + threadIdx.x, j_end, nxt);
+    for (int64_t ti = 0; ti < tiles; ++ti) {
+      const int64_t j = j_begin + ti * kTile + threadIdx.x;
+      const uint32_t use = u0 + (uint32_t)ti;
+      const int st = (int)(use % S);
+      bool ok = true;
       uint32_t e[W];
+      if constexpr (Bulk) {
+        ok = false;
+        if (live) {
+          ok = mbar_wait(smem_u32(&sh.bar[st]), (use / S) & 1u, nullptr);
+          if (!ok) {
+            live = false;
+            atomicOr(a.dev_status, kDevTimeout);
+            if (threadIdx.x == 0) {   // tiles ti .. issued - 1 of this pass may still be in flight
+              drain_first = use;
+              drain_count = issued - ti;
+            }
+          }
+        }
+        const uint4* src = reinterpret_cast<const uint4*>(&sh.ring[st][threadIdx.x * W]);
 #pragma unroll
-      for (int w = 0; w < W; ++w) e[w] = nxt[w];
-      load_sig<W>(l.sig, j + kTile, j_end, nxt);
+        for (int c = 0; c < W / 4; ++c) {
+          const uint4 v = ok ? src[c] : make_uint4(0u, 0u, 0u, 0u);
+          e[4 * c] = v.x;
+          e[4 * c + 1] = v.y;
+          e[4 * c + 2] = v.z;
+          e[4 * c + 3] = v.w;
+        }
+      } else {
+#pragma unroll
+        for (int w = 0; w < W; ++w) e[w] = nxt[w];
+        load_sig<W>(l.sig, j + kTile, j_end, nxt);
+      }
       // every query's distance first, as a mask of the admitted queries (the queue stores below could alias the
       // query signatures for the compiler): whole groups of 8 queries unrolled, then the pass's remaining queries
       // (a uniform count), so a pass of one query computes one distance
@@ -226,7 +316,7 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
         for (int u = 0; u < 8; ++u) test_query(g + u);
       }
       for (int qq = whole; qq < qn; ++qq) test_query(qq);
-      pend = j < j_end ? pend & qmask : 0u;
+      pend = ok && j < j_end ? pend & qmask : 0u;
       // Queue the admitted pairs; flush while the queue is past kFlushAt or a pair found it full. Every round of
       // this loop either queues all pending pairs or fills the queue, so it ends.
       int top = -1;   // the highest queue slot this thread took in this round
@@ -236,7 +326,7 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
           const int qq = __ffs(pend) - 1;
           pend &= pend - 1;
           const int slot = atomicAdd(&sh.count, 1);
-          if (slot < kCap) {
+          if (slot < G::kCap) {
             sh.items[slot] = Item{(int32_t)j, qq};
             top = slot;
           } else {
@@ -246,12 +336,20 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
         pend = full;
         // the barrier's OR gives every thread the same answer (a read of the count after a plain barrier
         // could already see the next tile's items in some threads)
-        if (!__syncthreads_or(pend != 0 || top >= kFlushAt)) break;
-        flush(sh, a, q0, qn);
+        if (!__syncthreads_or(pend != 0 || top >= G::kFlushAt)) break;
+        flush<W, Bulk>(sh, a, q0, qn);
         top = -1;
       }
+      if constexpr (Bulk) {
+        // every thread has read stage st (the barrier above): thread 0 refills it with the tile S ahead
+        if (threadIdx.x == 0 && live && ti + S < tiles) {
+          fetch_tile<W>(sh, l.sig, j_begin, j_end, ti + S, st);
+          ++issued;
+        }
+      }
     }
-    flush(sh, a, q0, qn);
+    u0 += (uint32_t)tiles;
+    flush<W, Bulk>(sh, a, q0, qn);
     // the lists' candidates (a sorted list holds them in its first slots, then zeros) and each list's record
     for (int i = threadIdx.x; i < qn * C; i += kThreads) {
       const int qq = i / C;
@@ -264,6 +362,12 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
       a.part_meta[(int64_t)s * a.B + q0 + threadIdx.x] = PartMeta{score_of_order(sh.best[threadIdx.x]), count};
     }
     __syncthreads();
+  }
+  if (threadIdx.x == 0) {
+    for (int64_t k = 0; k < drain_count; ++k) {
+      const uint32_t u = drain_first + (uint32_t)k;
+      if (!mbar_wait(smem_u32(&sh.bar[u % S]), (u / S) & 1u, nullptr)) break;
+    }
   }
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
@@ -322,10 +426,16 @@ __global__ void __launch_bounds__(256) sign_queries_kernel(const __nv_bfloat16* 
 
 // The scan is a programmatic dependent launch of the query-signature kernel: its CTAs may be scheduled while the
 // signatures are computed and wait in griddepcontrol.wait, which hides the launch gap.
-template <int W>
+template <int W, bool Bulk>
 cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStream_t st) {
-  const size_t smem = sizeof(Shared);
-  cudaError_t e = cudaFuncSetAttribute(lsh_scan_kernel<W>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  using Sh = Shared<W, Bulk>;
+  static_assert(offsetof(Sh, ring) % 16 == 0 && offsetof(Sh, qsig) % 16 == 0 &&
+                    (sizeof(uint32_t) * Geo<W, Bulk>::kRingWords) % 16 == 0 && offsetof(Sh, bar) % 8 == 0,
+                "16-byte vector reads and bulk copies need 16-byte aligned rows; mbarriers 8 bytes");
+  static_assert(2 * (sizeof(Sh) + 1024) <= 228 * 1024, "two CTAs per SM");
+  const size_t smem = sizeof(Sh);
+  cudaError_t e = cudaFuncSetAttribute(lsh_scan_kernel<W, Bulk>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(splits);
@@ -337,7 +447,18 @@ cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStre
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, lsh_scan_kernel<W>, a, l, splits);
+  return cudaLaunchKernelEx(&cfg, lsh_scan_kernel<W, Bulk>, a, l, splits);
+}
+
+// The ring form for scans bound by memory, the register form for those bound by the distance arithmetic. Measured
+// per lookup step, both forms forced, mid-1m (1M entries) from a flushed L2 and large-16m (16.7M entries):
+//  - 512-bit signatures: the ring is faster at every batch tried (1 to 32 queries; 177 against 223 us at one query
+//    on large-16m), its 16 free registers counting as much as the bytes in flight;
+//  - 128 and 256 bits: the ring is faster only for one query on a store of at least 16 tiles per split (86 against
+//    101 us at 256 bits on large-16m, 82 against 90 at 128); at two or more queries, or on mid-1m's 7 tiles per
+//    split, the register form is as fast or faster (up to 10 %).
+bool bulk_ring(int words, int B, int64_t n, int splits) {
+  return words == 16 || (B == 1 && n / splits >= 16 * (int64_t)kTile);
 }
 
 }  // namespace
@@ -364,10 +485,11 @@ cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms
   if (s > max_splits) s = max_splits;
   if (s < 1) s = 1;
   *splits = s;
+  const bool bulk = bulk_ring(l.words, a.B, a.n, s);
   switch (l.words) {   // 128, 256 or 512-bit signatures (16-byte loads)
-    case 4: return launch_w<4>(a, l, s, st);
-    case 8: return launch_w<8>(a, l, s, st);
-    case 16: return launch_w<16>(a, l, s, st);
+    case 4: return bulk ? launch_w<4, true>(a, l, s, st) : launch_w<4, false>(a, l, s, st);
+    case 8: return bulk ? launch_w<8, true>(a, l, s, st) : launch_w<8, false>(a, l, s, st);
+    case 16: return bulk ? launch_w<16, true>(a, l, s, st) : launch_w<16, false>(a, l, s, st);
     default: return cudaErrorInvalidValue;
   }
 }

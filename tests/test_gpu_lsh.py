@@ -66,6 +66,14 @@ def test_lsh_lookup_matches_the_oracle(bits, batch):
     _check_lsh_lookup(wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch), bits)
 
 
+@pytest.mark.parametrize("bits", [128, 256])
+def test_single_query_lookups_on_a_large_store_match_the_oracle(bits):
+    # 2.6M entries of d = 64: 304 splits of about 8,553 entries (17 tiles, the last one ragged). One-query lookups
+    # on splits of at least 16 tiles stream the signatures through the scan's shared-memory ring (at 512 bits every
+    # lookup does, and the cases above cover it); eight such lookups, compared as one batch
+    _check_lsh_lookup(wl.WORKLOADS["mid-1m"].scaled(n=2_600_000, d=64, batch=8), bits, one_at_a_time=True)
+
+
 @pytest.mark.parametrize("top_c", [1, 32])
 @pytest.mark.parametrize("batch", [16, 64], ids=["popcount", "tensor"])
 def test_lsh_top_c_extremes_match_the_oracle(batch, top_c):
@@ -73,7 +81,7 @@ def test_lsh_top_c_extremes_match_the_oracle(batch, top_c):
     _check_lsh_lookup(wl.WORKLOADS["mid-1m"].scaled(n=40_000, batch=batch, top_c=top_c), 256)
 
 
-def _check_lsh_lookup(w, bits):
+def _check_lsh_lookup(w, bits, one_at_a_time=False):
     batch = w.batch
     radius = wl.lsh_radius(w.tau_c, bits)
     R = wl.hyperplanes(bits, w.d, device="cuda")
@@ -82,8 +90,15 @@ def _check_lsh_lookup(w, bits):
         fill(cache, w)
         L.lacache_enable_lsh(cache.h, bits, radius, R)
         q = wl.batch(w, 0, device="cuda")
-        g = gpu_lookup(cache, q)
-        assert cache.last_launch()[1] == _expected_lsh_kernel(batch)
+        if one_at_a_time:
+            parts = []
+            for i in range(batch):
+                parts.append(gpu_lookup(cache, {k: q[k][i:i + 1] for k in ("emb", "prefix", "ids")}))
+                assert cache.last_launch()[1] == L.LACACHE_STAGE1_LSH
+            g = {k: np.concatenate([r[k] for r in parts]) for k in parts[0]}
+        else:
+            g = gpu_lookup(cache, q)
+            assert cache.last_launch()[1] == _expected_lsh_kernel(batch)
     oq = oracle_queries(q)
     p = params(w)
     res, amb = oracle.lookup_lsh(st, oq, p, wl.bf16_bits(R), radius)
