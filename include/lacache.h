@@ -270,6 +270,10 @@ lacache_status lacache_stage_times(lacache_t* h, double* stage1_ms, double* stag
  * issuer's bounded wait (about one second) runs out. The kernel then records LACACHE_ERR_DEVICE_TIMEOUT, its other
  * roles stop, its issued copies and MMAs drain, TMEM is freed and it exits. The context stays usable: the next
  * lacache_sync reports the timeout and later lookups run normally. The affected lookup's outputs are undefined.
+ * Lookups through the SimHash index take the injection when the popcount scan runs its shared-memory ring form
+ * (512-bit signatures, or one query on a store of at least 16 tiles of 512 entries per split): its first CTA
+ * withholds the bulk copy of its first tile, every thread's bounded wait for that tile runs out, the CTA still
+ * ends its passes and waits (bounded) for its issued copies, and the timeout is recorded the same way.
  * On CTA pairs (B > 128) the first CTA is the leader of the first pair; its abort stops its peer too. A single
  * query tile (B <= 128) runs on a dynamic schedule: the stall happens only if the first CTA claims a key tile, which
  * is certain when the store holds many more 256-key tiles than the GPU has SMs. 0 cancels. */

@@ -327,6 +327,8 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
       a.inject_stall = 1;
       --h->inject_stall;
     }
+    // the SimHash scan takes the injection only in its ring form (the launcher reports which form ran)
+    if (h->inject_stall > 0 && kernel == LACACHE_STAGE1_LSH) a.inject_stall = 1;
     cudaError_t e;
     if (kernel == LACACHE_STAGE1_TENSOR) {
       if (!h->encode) return LACACHE_ERR_CUDA;
@@ -350,7 +352,9 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
           e = lc::launch_stage1_lsh_tc(a, l, h->num_sms, h->max_splits, st, &splits);
           kernel = LACACHE_STAGE1_LSH_TENSOR;
         } else {
-          e = lc::launch_stage1_lsh(a, l, h->num_sms, h->max_splits, st, &splits);
+          bool ring = false;
+          e = lc::launch_stage1_lsh(a, l, h->num_sms, h->max_splits, st, &splits, &ring);
+          if (ring && a.inject_stall) --h->inject_stall;
         }
       }
     } else {

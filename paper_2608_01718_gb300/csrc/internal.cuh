@@ -85,7 +85,8 @@ struct Stage1Args {
   uint64_t* part_cand;
   PartMeta* part_meta;
   unsigned int* dev_status;
-  int inject_stall;           // test support: CTA 0 of the tensor kernel withholds one load (see lacache.h)
+  int inject_stall;           // test support: CTA 0 of the tensor kernel, or of the SimHash scan's ring form,
+                              // withholds one load (see lacache.h)
   int* tile_ctr;              // tensor kernel, one query tile: dynamic tile schedule on these two counters
                               // [next tile, CTAs done], zero at launch and zero again when the grid ends
                               // (nullptr: static schedule)
@@ -155,8 +156,10 @@ struct LshArgs {
 };
 // Popcount scan (small batches) and the tensor-core scan over the expanded index (batches of at least
 // kLshTensorMinBatch queries).
+// *ring: the launch runs the scan's shared-memory ring form (the only form with bounded waits, so the only one a
+// stall injection, a.inject_stall, acts on).
 cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits, cudaStream_t st,
-                              int* splits);
+                              int* splits, bool* ring);
 cudaError_t launch_stage1_lsh_tc(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits,
                                  cudaStream_t st, int* splits);
 constexpr int kLshTensorMinBatch = 40;

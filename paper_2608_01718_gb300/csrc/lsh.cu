@@ -244,8 +244,12 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
     const int qn = min(kQC, a.B - q0);
     if constexpr (Bulk) {
       if (threadIdx.x == 0 && live) {
+        // test support: CTA 0 withholds the copy of its first tile (no arrive either), so every thread's wait for
+        // it runs out; the withheld copy counts as issued, and the drain below waits for it in vain (bounded)
+        const bool withhold = a.inject_stall && blockIdx.x == 0 && q0 == 0;
         for (issued = 0; issued < min((int64_t)S, tiles); ++issued)
-          fetch_tile<W>(sh, l.sig, j_begin, j_end, issued, (int)((u0 + issued) % S));
+          if (!(withhold && issued == 0))
+            fetch_tile<W>(sh, l.sig, j_begin, j_end, issued, (int)((u0 + issued) % S));
       }
     }
     for (int i = threadIdx.x; i < kQC * W; i += kThreads) {
@@ -364,9 +368,11 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
     __syncthreads();
   }
   if (threadIdx.x == 0) {
+    // each pending copy gets its own bounded wait: one that never arrives does not cut short the wait for the
+    // others, which may still be writing this CTA's shared memory
     for (int64_t k = 0; k < drain_count; ++k) {
       const uint32_t u = drain_first + (uint32_t)k;
-      if (!mbar_wait(smem_u32(&sh.bar[u % S]), (u / S) & 1u, nullptr)) break;
+      mbar_wait(smem_u32(&sh.bar[u % S]), (u / S) & 1u, nullptr);
     }
   }
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -479,13 +485,14 @@ cudaError_t launch_sign_queries(const __nv_bfloat16* q, int B, int d, const __nv
 }
 
 cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits, cudaStream_t st,
-                              int* splits) {
+                              int* splits, bool* ring) {
   const int64_t tiles = (a.n + kTile - 1) / kTile;
   int s = (int)(tiles < 2 * (int64_t)num_sms ? tiles : 2 * (int64_t)num_sms);
   if (s > max_splits) s = max_splits;
   if (s < 1) s = 1;
   *splits = s;
   const bool bulk = bulk_ring(l.words, a.B, a.n, s);
+  *ring = bulk;
   switch (l.words) {   // 128, 256 or 512-bit signatures (16-byte loads)
     case 4: return bulk ? launch_w<4, true>(a, l, s, st) : launch_w<4, false>(a, l, s, st);
     case 8: return bulk ? launch_w<8, true>(a, l, s, st) : launch_w<8, false>(a, l, s, st);

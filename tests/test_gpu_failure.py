@@ -6,6 +6,10 @@ and exits, and lacache_sync reports LACACHE_ERR_DEVICE_TIMEOUT. The context must
 matches the one taken before the injection. With B = 256 the batch runs on CTA pairs: the withholding CTA is the
 leader of the first pair, whose abort also stops its peer; both CTAs still meet at the cluster barrier before
 freeing the pair's TMEM.
+
+The SimHash popcount scan's ring form (always taken at 512 bits) has the same test: its first CTA withholds the
+bulk copy of its first tile, every thread's bounded wait for it runs out, and the CTA ends its pass, waits (bounded)
+for the copies it did issue, and exits.
 """
 import pytest
 import torch
@@ -49,3 +53,30 @@ def test_stage1_wait_timeout_is_reported_and_the_context_stays_usable(batch):
         cache.sync()
         for k in ("status", "entry_id", "cand_id", "n_cand"):
             assert torch.equal(after[k], before[k]), k
+
+
+def test_simhash_ring_wait_timeout_is_reported_and_the_context_stays_usable():
+    w = wl.WORKLOADS["mid-1m"].scaled(n=40_000, batch=8)
+    bits = 512
+    with L.LaCache(w.d, w.k, w.n, w.tau_c, w.tau_a, w.top_c, max_batch=w.batch,
+                   stage1=L.LACACHE_STAGE1_LSH) as cache:
+        for ch in wl.iter_store(w, "cuda"):
+            cache.insert(ch["key"], ch["prefix"], ch["ids"])
+        L.lacache_enable_lsh(cache.h, bits, wl.lsh_radius(w.tau_c, bits), wl.hyperplanes(bits, w.d, device="cuda"))
+        q = wl.batch(w, 0, device="cuda")
+        before = {k: v.clone() for k, v in cache.lookup(q["emb"], q["prefix"], q["ids"]).items()}
+        cache.sync()
+        L.lacache_inject_stall(cache.h, 1)
+        cache.lookup(q["emb"], q["prefix"], q["ids"])
+        assert cache.last_launch()[1] == L.LACACHE_STAGE1_LSH
+        with pytest.raises(L.LacacheError) as e:
+            cache.sync()
+        assert e.value.status == L.LACACHE_ERR_DEVICE_TIMEOUT
+        cache.sync()
+        after = cache.lookup(q["emb"], q["prefix"], q["ids"])
+        cache.sync()
+        for k in ("status", "entry_id", "cand_id", "n_cand"):
+            assert torch.equal(after[k], before[k]), k
+        # the injection was taken by that lookup: the next one runs clean
+        cache.lookup(q["emb"], q["prefix"], q["ids"])
+        cache.sync()
