@@ -10,6 +10,11 @@
 //    completed on the stage's mbarrier; a stage is refilled after the tile's CTA barrier, so kStages - 1 tiles are
 //    in flight while one is counted. Twice the bytes in flight, and W registers free: the form for the scans bound
 //    by memory (one query on a large store) and for 512-bit signatures.
+// The distance test first counts the differing bits of a prefix of P of the W words (the kernel's P parameter): a
+// pair whose prefix distance already exceeds the radius is out, since the prefix distance never exceeds the whole
+// one. With the radii the thresholds give, nearly every pair of unrelated signatures is out after the prefix
+// (prefix_words() picks P from the binomial tail of a random pair's distance), and the few left in each thread's
+// mask get the whole distance in a loop over that mask. P = W tests the whole signature at once.
 // Admitted (query, entry) pairs are queued in shared memory.
 // When the queue passes three quarters of its capacity, and at the end of the split, all warps take queue items two
 // at a time and compute the exact fp32 score over the gathered key row (each lane's 8-element chunks in order,
@@ -17,6 +22,8 @@
 // list. A tile can admit more pairs than the queue has room for (up to 512 x 32, e.g. with radius = bits): a pair
 // that finds the queue full stays in its thread's pending mask and is queued again after the next flush. The
 // partial lists have the format of the other stage-1 kernels, so stage 2 is shared.
+#include <cmath>
+
 #include "internal.cuh"
 #include "tcgen05.cuh"
 
@@ -151,17 +158,19 @@ __device__ __forceinline__ void csa(uint32_t& hi, uint32_t& lo, uint32_t a, uint
   hi = (a & b) | (u & c);
 }
 
-// Number of set bits in x[0..W). Population count runs at 16 per clock per SM, the logic operations at 64, so
-// carry-save adders first fold words into sum and carry words, each group of 8 words into 5 popcounts (3 adders):
+// Number of set bits in x[0..N) (N = 4, 8 or 16). Population count runs at 16 per clock per SM, the logic
+// operations at 64, so carry-save adders first fold words into sum and carry words, each group of 8 words into 5
+// popcounts (3 adders):
 //   x0 + x1 + x2 = sa + 2 ca,  x3 + x4 + x5 = sb + 2 cb,  sa + sb + x6 = sc + 2 cc,
 //   |x0..x7| = |sc| + |x7| + 2 (|ca| + |cb| + |cc|);
 // a group of 4 words into 3 (one adder). The count is exact.
-template <int W>
+template <int N, int W>
 __device__ __forceinline__ int hamming(const uint32_t (&x)[W]) {
+  static_assert(N <= W, "a prefix of the signature");
   int h = 0;
-  if constexpr (W % 8 == 0) {
+  if constexpr (N % 8 == 0) {
 #pragma unroll
-    for (int g = 0; g < W; g += 8) {
+    for (int g = 0; g < N; g += 8) {
       uint32_t ca, sa, cb, sb, cc, sc;
       csa(ca, sa, x[g], x[g + 1], x[g + 2]);
       csa(cb, sb, x[g + 3], x[g + 4], x[g + 5]);
@@ -169,15 +178,35 @@ __device__ __forceinline__ int hamming(const uint32_t (&x)[W]) {
       h += __popc(sc) + __popc(x[g + 7]) + 2 * (__popc(ca) + __popc(cb) + __popc(cc));
     }
   } else {
-    static_assert(W % 4 == 0, "signature words come in groups of 4");
+    static_assert(N % 4 == 0, "signature words come in groups of 4");
 #pragma unroll
-    for (int g = 0; g < W; g += 4) {
+    for (int g = 0; g < N; g += 4) {
       uint32_t c, s;
       csa(c, s, x[g], x[g + 1], x[g + 2]);
       h += __popc(s) + __popc(x[g + 3]) + 2 * __popc(c);
     }
   }
   return h;
+}
+
+// Number of set bits in x[0..N) for a prefix of N = 3 or 5 words (one or two carry-save adders):
+//   N = 3: x0 + x1 + x2 = s + 2 c;                        |x| = |s| + 2 |c|
+//   N = 5: x0 + x1 + x2 = s1 + 2 c1, s1 + x3 + x4 = s2 + 2 c2;  |x| = |s2| + 2 (|c1| + |c2|)
+// and hamming() for N = 4, 8 or 16.
+template <int N, int W>
+__device__ __forceinline__ int prefix_count(const uint32_t (&x)[W]) {
+  if constexpr (N == 3) {
+    uint32_t c, s;
+    csa(c, s, x[0], x[1], x[2]);
+    return __popc(s) + 2 * __popc(c);
+  } else if constexpr (N == 5) {
+    uint32_t c1, s1, c2, s2;
+    csa(c1, s1, x[0], x[1], x[2]);
+    csa(c2, s2, s1, x[3], x[4]);
+    return __popc(s2) + 2 * (__popc(c1) + __popc(c2));
+  } else {
+    return hamming<N, W>(x);
+  }
 }
 
 // Signature words of entry j into e (zeros past the split's end).
@@ -215,7 +244,7 @@ __device__ __forceinline__ void fetch_tile(Shared<W, true>& sh, const uint32_t* 
                : "memory");
 }
 
-template <int W, bool Bulk>
+template <int W, bool Bulk, int P>
 __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, LshArgs l, int splits) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   using G = Geo<W, Bulk>;
@@ -299,20 +328,23 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
       }
       // every query's distance first, as a mask of the admitted queries (the queue stores below could alias the
       // query signatures for the compiler): whole groups of 8 queries unrolled, then the pass's remaining queries
-      // (a uniform count), so a pass of one query computes one distance
-      unsigned pend = 0;
+      // (a uniform count), so a pass of one query computes one distance. With a prefix test (P < W) the loop
+      // leaves the queries within the radius on the first P words in `cand`, and each gets its whole distance
+      // after it.
+      unsigned pend = 0, cand = 0;
       auto test_query = [&](int qq) {
         const uint4* qs = reinterpret_cast<const uint4*>(sh.qsig[qq]);
         uint32_t x[W];
 #pragma unroll
-        for (int w = 0; w < W / 4; ++w) {
+        for (int w = 0; w < (P + 3) / 4; ++w) {
           const uint4 v = qs[w];
           x[4 * w] = e[4 * w] ^ v.x;
-          x[4 * w + 1] = e[4 * w + 1] ^ v.y;
-          x[4 * w + 2] = e[4 * w + 2] ^ v.z;
-          x[4 * w + 3] = e[4 * w + 3] ^ v.w;
+          if (4 * w + 1 < P) x[4 * w + 1] = e[4 * w + 1] ^ v.y;
+          if (4 * w + 2 < P) x[4 * w + 2] = e[4 * w + 2] ^ v.z;
+          if (4 * w + 3 < P) x[4 * w + 3] = e[4 * w + 3] ^ v.w;
         }
-        pend |= (hamming<W>(x) <= l.radius ? 1u : 0u) << qq;
+        const unsigned bit = (prefix_count<P, W>(x) <= l.radius ? 1u : 0u) << qq;
+        if constexpr (P == W) pend |= bit; else cand |= bit;
       };
       const int whole = qn & ~7;
       for (int g = 0; g < whole; g += 8) {
@@ -320,6 +352,23 @@ __global__ void __launch_bounds__(kThreads, 2) lsh_scan_kernel(Stage1Args a, Lsh
         for (int u = 0; u < 8; ++u) test_query(g + u);
       }
       for (int qq = whole; qq < qn; ++qq) test_query(qq);
+      if constexpr (P < W) {
+        while (cand) {   // this thread's few candidates, each with its whole distance
+          const int qq = __ffs(cand) - 1;
+          cand &= cand - 1;
+          const uint4* qs = reinterpret_cast<const uint4*>(sh.qsig[qq]);
+          uint32_t x[W];
+#pragma unroll
+          for (int w = 0; w < W / 4; ++w) {
+            const uint4 v = qs[w];
+            x[4 * w] = e[4 * w] ^ v.x;
+            x[4 * w + 1] = e[4 * w + 1] ^ v.y;
+            x[4 * w + 2] = e[4 * w + 2] ^ v.z;
+            x[4 * w + 3] = e[4 * w + 3] ^ v.w;
+          }
+          pend |= (hamming<W, W>(x) <= l.radius ? 1u : 0u) << qq;
+        }
+      }
       pend = ok && j < j_end ? pend & qmask : 0u;
       // Queue the admitted pairs; flush while the queue is past kFlushAt or a pair found it full. Every round of
       // this loop either queues all pending pairs or fills the queue, so it ends.
@@ -432,7 +481,7 @@ __global__ void __launch_bounds__(256) sign_queries_kernel(const __nv_bfloat16* 
 
 // The scan is a programmatic dependent launch of the query-signature kernel: its CTAs may be scheduled while the
 // signatures are computed and wait in griddepcontrol.wait, which hides the launch gap.
-template <int W, bool Bulk>
+template <int W, bool Bulk, int P>
 cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStream_t st) {
   using Sh = Shared<W, Bulk>;
   static_assert(offsetof(Sh, ring) % 16 == 0 && offsetof(Sh, qsig) % 16 == 0 &&
@@ -440,7 +489,7 @@ cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStre
                 "16-byte vector reads and bulk copies need 16-byte aligned rows; mbarriers 8 bytes");
   static_assert(2 * (sizeof(Sh) + 1024) <= 228 * 1024, "two CTAs per SM");
   const size_t smem = sizeof(Sh);
-  cudaError_t e = cudaFuncSetAttribute(lsh_scan_kernel<W, Bulk>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(lsh_scan_kernel<W, Bulk, P>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)smem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -453,7 +502,7 @@ cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStre
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, lsh_scan_kernel<W, Bulk>, a, l, splits);
+  return cudaLaunchKernelEx(&cfg, lsh_scan_kernel<W, Bulk, P>, a, l, splits);
 }
 
 // The ring form for scans bound by memory, the register form for those bound by the distance arithmetic. Measured
@@ -465,6 +514,37 @@ cudaError_t launch_w(const Stage1Args& a, const LshArgs& l, int splits, cudaStre
 //    split, the register form is as fast or faster (up to 10 %).
 bool bulk_ring(int words, int B, int64_t n, int splits) {
   return words == 16 || (B == 1 && n / splits >= 16 * (int64_t)kTile);
+}
+
+// Probability that two independent uniformly random n-bit strings differ in at most r positions.
+double random_pair_within(int n, int r) {
+  if (r >= n) return 1.0;
+  double p = 0.0;
+  for (int i = 0; i <= r; ++i) p += std::exp(std::lgamma(n + 1.0) - std::lgamma(i + 1.0) - std::lgamma(n - i + 1.0));
+  return p * std::exp(-n * std::log(2.0));
+}
+
+// The distance test's prefix: 3, 5 or 8 words at W = 4, 8 or 16 (96, 160 or 256 bits) when at most 2 % of
+// unrelated pairs (whose distance is about that of random strings) stay within the radius on it, else the whole
+// signature. At the radii the thresholds give (35, 60 and 106 bits at tau_c = 0.9) the prefix keeps 0.5 %, 0.1 %
+// and 0.4 % of them.
+template <int W>
+constexpr int kPrefixWords = W == 4 ? 3 : W == 8 ? 5 : 8;
+template <int W>
+bool use_prefix(int radius) {
+  return random_pair_within(32 * kPrefixWords<W>, radius) <= 0.02;
+}
+
+template <int W>
+cudaError_t launch_form(bool bulk, const Stage1Args& a, const LshArgs& l, int splits, cudaStream_t st) {
+  constexpr int P = kPrefixWords<W>;
+  const bool prefix = use_prefix<W>(l.radius);
+  if constexpr (W == 16) {   // 512-bit signatures always take the ring form
+    return prefix ? launch_w<W, true, P>(a, l, splits, st) : launch_w<W, true, W>(a, l, splits, st);
+  } else {
+    if (prefix) return bulk ? launch_w<W, true, P>(a, l, splits, st) : launch_w<W, false, P>(a, l, splits, st);
+    return bulk ? launch_w<W, true, W>(a, l, splits, st) : launch_w<W, false, W>(a, l, splits, st);
+  }
 }
 
 }  // namespace
@@ -494,9 +574,9 @@ cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms
   const bool bulk = bulk_ring(l.words, a.B, a.n, s);
   *ring = bulk;
   switch (l.words) {   // 128, 256 or 512-bit signatures (16-byte loads)
-    case 4: return bulk ? launch_w<4, true>(a, l, s, st) : launch_w<4, false>(a, l, s, st);
-    case 8: return bulk ? launch_w<8, true>(a, l, s, st) : launch_w<8, false>(a, l, s, st);
-    case 16: return bulk ? launch_w<16, true>(a, l, s, st) : launch_w<16, false>(a, l, s, st);
+    case 4: return launch_form<4>(bulk, a, l, s, st);
+    case 8: return launch_form<8>(bulk, a, l, s, st);
+    case 16: return launch_form<16>(bulk, a, l, s, st);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -66,6 +66,14 @@ def test_lsh_lookup_matches_the_oracle(bits, batch):
     _check_lsh_lookup(wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch), bits)
 
 
+@pytest.mark.parametrize("batch", [1, 5])
+@pytest.mark.parametrize("bits", [128, 256, 512])
+def test_lsh_lookup_at_a_low_threshold_matches_the_oracle(bits, batch):
+    # tau_c = 0.8 gives radii of 45, 79 and 142 bits, too wide for the scan's prefix test to reject unrelated
+    # pairs: it tests whole signatures (at 512 bits through its shared-memory ring)
+    _check_lsh_lookup(wl.WORKLOADS["mid-1m"].scaled(n=70_000, batch=batch, tau_c=0.8), bits)
+
+
 @pytest.mark.parametrize("bits", [128, 256])
 def test_single_query_lookups_on_a_large_store_match_the_oracle(bits):
     # 2.6M entries of d = 64: 304 splits of about 8,553 entries (17 tiles, the last one ragged). One-query lookups
