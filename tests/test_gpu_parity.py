@@ -100,12 +100,16 @@ def test_stream_query_groups_and_load_phases(d, batch):
 
 
 def test_auto_takes_the_stream_scan_only_for_small_batches_on_stores_l2_holds():
-    """LACACHE_STAGE1_AUTO: the streaming scan for at most 4 queries against at most 32 MB of keys and for 1 or 2
+    """LACACHE_STAGE1_AUTO: the streaming scan against at most 32 MB of keys while n d B <= 2^25, and for 1 or 2
     queries at d = 1024, the tensor-core scan otherwise (and the oracle agrees with its results)."""
-    small = wl.WORKLOADS["mid-1m"].scaled(n=10_000, batch=8)      # 15 MB of keys
+    tiny = wl.WORKLOADS["tiny-4k"].scaled(batch=22)                # 4,096 x 384: n d = 1,572,864
+    small = wl.WORKLOADS["mid-1m"].scaled(n=10_000, batch=8)      # 15 MB of keys, n d = 7,680,000
+    mid = wl.WORKLOADS["mid-1m"].scaled(n=20_000, batch=3)        # 30.7 MB of keys, n d = 15,360,000
     large = wl.WORKLOADS["mid-1m"].scaled(n=30_000, batch=8)      # 46 MB of keys
     wide = wl.WORKLOADS["large-16m"].scaled(n=30_000, batch=8)    # d = 1024, 61 MB of keys
-    for w, want in ((small, {1: L.LACACHE_STAGE1_STREAM, 4: L.LACACHE_STAGE1_STREAM, 5: L.LACACHE_STAGE1_TENSOR}),
+    for w, want in ((tiny, {16: L.LACACHE_STAGE1_STREAM, 21: L.LACACHE_STAGE1_STREAM, 22: L.LACACHE_STAGE1_TENSOR}),
+                    (small, {1: L.LACACHE_STAGE1_STREAM, 4: L.LACACHE_STAGE1_STREAM, 5: L.LACACHE_STAGE1_TENSOR}),
+                    (mid, {2: L.LACACHE_STAGE1_STREAM, 3: L.LACACHE_STAGE1_TENSOR}),
                     (large, {1: L.LACACHE_STAGE1_TENSOR, 4: L.LACACHE_STAGE1_TENSOR}),
                     (wide, {1: L.LACACHE_STAGE1_STREAM, 2: L.LACACHE_STAGE1_STREAM, 3: L.LACACHE_STAGE1_TENSOR})):
         st = oracle_store(w)
