@@ -60,11 +60,10 @@ typedef enum { LACACHE_BF16 = 0, LACACHE_F32 = 1 } lacache_dtype;
 
 /* Which stage-1 kernel lookups run. */
 typedef enum {
-  LACACHE_STAGE1_AUTO = 0,   /* the streaming scan for stores of at most 32 MB of keys (n x d x 2 bytes, a store
-                                L2 holds) when n x d x B <= 2^25 (few enough multiply-adds that its latency is
-                                the shorter), and for 1 or 2 queries at d = 1024 (where it matches the tensor-core
-                                scan from HBM); the tensor-core scan otherwise, which holds the HBM roofline at
-                                every batch size */
+  LACACHE_STAGE1_AUTO = 0,   /* the streaming scan when n x d x B <= 2^25 (few enough multiply-adds that its
+                                latency is the shorter: at most 64 MiB of keys at one query) and for 1 or 2
+                                queries at d = 1024 (where it matches the tensor-core scan from HBM); the
+                                tensor-core scan otherwise, which holds the HBM roofline at every batch size */
   LACACHE_STAGE1_TENSOR = 1, /* tcgen05 tensor-core scan (TMA-fed, TMEM accumulators) */
   LACACHE_STAGE1_STREAM = 2, /* streaming CUDA-core scan: warp per key tile, 128-bit key loads, packed fp32 FMA */
   LACACHE_STAGE1_LSH = 3,    /* SimHash index, then the exact key check (requires lacache_enable_lsh) */

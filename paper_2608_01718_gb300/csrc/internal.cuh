@@ -174,18 +174,17 @@ cudaError_t launch_expand_signatures(const uint32_t* sig, int64_t first, int64_t
 // of it from 1 to 128 queries). The streaming scan matches or passes it for one or two queries at d = 1024, where
 // every lane has its whole share of a row, four 16-byte chunks, in flight per tile (585.6 against 590.9 us at
 // 2M x 1024 and one query), and falls behind with fewer chunks per lane, several phases or more queries (d = 800,
-// 896 and 1280 trail by 1-2 %). On a store of at most 32 MB of keys the scan is bound by latency: the tensor-core
+// 896 and 1280 trail by 1-2 %). On stores of up to some tens of MB the scan is bound by latency: the tensor-core
 // scan takes a nearly flat 9-16 us a lookup, while the streaming scan's time grows with its multiply-adds, n d B.
-// Back-to-back lookups (store in L2) cross over at about 2^25 of them: 4,096 x 384, B = 16: 13.7 against 14.0 us a
-// lookup; 16,384 x 768, B = 2: 8.9 against 8.9, B = 4: 10.4 against 8.9; 43,690 x 768, B = 1: 10.6 against 13.3,
-// B = 2: 13.6 against 13.1. A single lookup on an idle device crosses later (16,384 x 768, B = 4: 18.2 against
-// 21.2 us), and from a flushed L2 the streaming scan's stage 1 is also the shorter one up to that size (22.3
-// against 25.9 us at 43,690 x 768, B = 1). So the streaming scan takes the stores of at most 32 MB of keys when
-// n d B <= 2^25.
-constexpr int64_t kStreamAutoKeyBytes = (int64_t)32 << 20;
+// Back-to-back lookups cross over at about 2^25 of them: 4,096 x 384, B = 16: 13.7 against 14.0 us a lookup;
+// 16,384 x 768, B = 2: 8.9 against 8.9, B = 4: 10.4 against 8.9; 43,690 x 768 (67 MB of keys), B = 1: 10.6 against
+// 13.3, B = 2: 13.6 against 13.1. A single lookup on an idle device crosses later (16,384 x 768, B = 4: 18.2
+// against 21.2 us), and from a flushed L2 the streaming scan's stage 1 is also the shorter one at that size (22.3
+// against 25.9 us at 43,690 x 768, B = 1). So the streaming scan takes the lookups with n d B <= 2^25 (at most
+// 64 MiB of keys, at one query).
 constexpr int64_t kStreamAutoMacs = (int64_t)1 << 25;
 inline int auto_stage1(int64_t n, int d, int B) {
-  if (n * d * 2 <= kStreamAutoKeyBytes && n * d * B <= kStreamAutoMacs) return LACACHE_STAGE1_STREAM;
+  if (n * d * B <= kStreamAutoMacs) return LACACHE_STAGE1_STREAM;
   if (B <= 2 && d == 1024) return LACACHE_STAGE1_STREAM;
   return LACACHE_STAGE1_TENSOR;
 }

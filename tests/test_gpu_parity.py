@@ -100,17 +100,19 @@ def test_stream_query_groups_and_load_phases(d, batch):
 
 
 def test_auto_takes_the_stream_scan_only_for_small_batches_on_stores_l2_holds():
-    """LACACHE_STAGE1_AUTO: the streaming scan against at most 32 MB of keys while n d B <= 2^25, and for 1 or 2
-    queries at d = 1024, the tensor-core scan otherwise (and the oracle agrees with its results)."""
+    """LACACHE_STAGE1_AUTO: the streaming scan while n d B <= 2^25, and for 1 or 2 queries at d = 1024, the
+    tensor-core scan otherwise (and the oracle agrees with its results)."""
     tiny = wl.WORKLOADS["tiny-4k"].scaled(batch=22)                # 4,096 x 384: n d = 1,572,864
     small = wl.WORKLOADS["mid-1m"].scaled(n=10_000, batch=8)      # 15 MB of keys, n d = 7,680,000
     mid = wl.WORKLOADS["mid-1m"].scaled(n=20_000, batch=3)        # 30.7 MB of keys, n d = 15,360,000
-    large = wl.WORKLOADS["mid-1m"].scaled(n=30_000, batch=8)      # 46 MB of keys
+    large = wl.WORKLOADS["mid-1m"].scaled(n=30_000, batch=8)      # 46 MB of keys, n d = 23,040,000
+    over = wl.WORKLOADS["mid-1m"].scaled(n=44_000, batch=2)       # 68 MB of keys, n d = 33,792,000 > 2^25
     wide = wl.WORKLOADS["large-16m"].scaled(n=30_000, batch=8)    # d = 1024, 61 MB of keys
     for w, want in ((tiny, {16: L.LACACHE_STAGE1_STREAM, 21: L.LACACHE_STAGE1_STREAM, 22: L.LACACHE_STAGE1_TENSOR}),
                     (small, {1: L.LACACHE_STAGE1_STREAM, 4: L.LACACHE_STAGE1_STREAM, 5: L.LACACHE_STAGE1_TENSOR}),
                     (mid, {2: L.LACACHE_STAGE1_STREAM, 3: L.LACACHE_STAGE1_TENSOR}),
-                    (large, {1: L.LACACHE_STAGE1_TENSOR, 4: L.LACACHE_STAGE1_TENSOR}),
+                    (large, {1: L.LACACHE_STAGE1_STREAM, 2: L.LACACHE_STAGE1_TENSOR, 4: L.LACACHE_STAGE1_TENSOR}),
+                    (over, {1: L.LACACHE_STAGE1_TENSOR}),
                     (wide, {1: L.LACACHE_STAGE1_STREAM, 2: L.LACACHE_STAGE1_STREAM, 3: L.LACACHE_STAGE1_TENSOR})):
         st = oracle_store(w)
         with new_cache(w, L.LACACHE_STAGE1_AUTO) as cache:
