@@ -28,7 +28,8 @@ struct lacache {
   int32_t* append_dst;       // [max_batch] destination rank of each appended query
   int32_t* append_count;     // device count of appended rows
   int32_t* append_count_host;  // pinned
-  unsigned char* stage_in;   // device staging for lookup_host inputs
+  unsigned char* stage_in;   // device staging for lookup_host inputs: two slots, used in turn
+  int stage_slot;            // the slot the next host lookup's inputs go to
   unsigned char* stage_out;  // device staging for lookup_host results
   unsigned char* stage_host; // pinned host staging of lookup_host results (mapped: the kernels write it directly)
   unsigned char* stage_host_dev; // device address of stage_host, or nullptr if the device cannot map it
@@ -136,8 +137,13 @@ __global__ void append_rows_kernel(const uint4* __restrict__ q_emb, const uint4*
 
 // lookup_host's inputs, read by the device straight from mapped pinned host memory (NVLink-C2C on Grace) into the
 // device staging: one launch for the three arrays instead of one DMA copy each. Segments with zero bytes are
-// skipped; 16-byte vectors where both ends are aligned, bytes otherwise. Lets the stage-1 grid (a programmatic
-// dependent) start its set-up at once; that grid is launched to wait for this one before reading anything.
+// skipped; 16-byte vectors where both ends are aligned, bytes otherwise.
+// The kernel is a programmatic dependent of the previous lookup's stage 2, so it copies while that stage runs:
+// host lookups use the two staging slots in turn, and the lookup that last used this slot (two host lookups back)
+// has completed. Before it exits it waits for the grids before it, so its completion also means the previous
+// lookup has ended (the stage-1 grid after it, which waits for it, then overwrites the partial lists the previous
+// stage 2 read). Lets the stage-1 grid (a programmatic dependent too) start its set-up at once; that grid waits for
+// this one before reading anything.
 struct GatherSeg {
   const unsigned char* src;
   unsigned char* dst;
@@ -158,6 +164,7 @@ __global__ void gather_host_kernel(GatherArgs g) {
     for (size_t i = tid; i < nv; i += nth) dv[i] = sv[i];
     for (size_t i = nv * 16 + tid; i < e.bytes; i += nth) e.dst[i] = e.src[i];
   }
+  asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
 // The address through which the current device can read host pointer p, or nullptr when it has none (pageable
@@ -190,21 +197,37 @@ struct HostInputs {
   unsigned char* dst[3];
   size_t bytes[3];
 };
+size_t stage_in_bytes(const lacache_config& c, int pd);
+// Distance between the two staging slots: a slot's bytes rounded up to 256, so that both slots' arrays keep the
+// alignment the kernels and the TMA descriptors need (a slot ends with B * k * 4 bytes of token ids).
+size_t stage_in_stride(const lacache_config& c, int pd) { return (stage_in_bytes(c, pd) + 255) & ~(size_t)255; }
+
+// The inputs go to the handle's current staging slot; a host lookup that enqueues work then moves the handle to
+// the other slot (next_stage_slot), so consecutive host lookups alternate.
 HostInputs host_inputs(const lacache* h, int B, const void* emb, const void* pre, const int32_t* ids) {
   const lacache_config& c = h->cfg;
   HostInputs in{{emb, pre, ids}, {}, {(size_t)B * c.d * 2, (size_t)B * h->pd * 2, (size_t)B * c.k * 4}};
-  in.dst[0] = h->stage_in;
+  in.dst[0] = h->stage_in + (size_t)h->stage_slot * stage_in_stride(c, h->pd);
   in.dst[1] = in.dst[0] + (size_t)c.max_batch * c.d * 2;
   in.dst[2] = in.dst[1] + (size_t)c.max_batch * h->pd * 2;
   return in;
 }
 
-// One gather kernel for the segments of g, `bytes` in all.
+void next_stage_slot(lacache* h) { h->stage_slot ^= 1; }
+
+// One gather kernel for the segments of g, `bytes` in all (a programmatic dependent launch).
 cudaError_t launch_gather(const lacache* h, const GatherArgs& g, size_t bytes, cudaStream_t st) {
   const size_t vec = (bytes + 15) / 16;
-  const int grid = (int)std::min<size_t>((vec + 255) / 256, (size_t)2 * h->num_sms);
-  gather_host_kernel<<<grid, 256, 0, st>>>(g);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)std::min<size_t>((vec + 255) / 256, (size_t)2 * h->num_sms));
+  cfg.blockDim = dim3(256);
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, gather_host_kernel, g);
 }
 
 // A handle set to the SimHash stage can look up only once its index is enabled.
@@ -478,7 +501,7 @@ lacache_status lacache_create_ensemble(const lacache_config* cfg, const lacache_
             cudaMalloc(&h->counters, 3 * sizeof(unsigned long long)) == cudaSuccess &&
             cudaMemset(h->counters, 0, 3 * sizeof(unsigned long long)) == cudaSuccess &&
             cudaMemset(h->tile_ctr, 0, 2 * sizeof(int)) == cudaSuccess &&
-            cudaMalloc(&h->stage_in, stage_in_bytes(c, pd)) == cudaSuccess &&
+            cudaMalloc(&h->stage_in, 2 * stage_in_stride(c, pd)) == cudaSuccess &&
             cudaMalloc(&h->stage_out, stage_out_bytes(c, ens->m)) == cudaSuccess &&
             cudaMallocHost(&h->append_count_host, 4) == cudaSuccess &&
             cudaHostAlloc((void**)&h->stage_host, stage_out_bytes(c, ens->m), cudaHostAllocMapped) == cudaSuccess &&
@@ -573,6 +596,7 @@ lacache_status lacache_lookup_host(lacache_t* h, int32_t B, const void* q_emb_ho
   cudaStream_t st = (cudaStream_t)cuda_stream;
   const lacache_config& c = h->cfg;
   const HostInputs in = host_inputs(h, B, q_emb_host, q_prefix_host, q_ids_host);
+  next_stage_slot(h);
   // Inputs: arrays in mapped pinned memory are gathered by one kernel; any other array is copied by DMA.
   GatherArgs g{};
   size_t gathered = 0;
@@ -649,6 +673,7 @@ lacache_status lacache_lookup_host_async(lacache_t* h, int32_t B, const void* q_
                       map_output(o.cand_prefix_scores, &dev.cand_prefix_scores);
   if (!mapped) return LACACHE_ERR_INVALID_ARG;
   cudaStream_t st = (cudaStream_t)cuda_stream;
+  next_stage_slot(h);
   if (launch_gather(h, g, gathered, st) != cudaSuccess) return LACACHE_ERR_CUDA;
   return run_lookup(h, B, in.dst[0], in.dst[1], reinterpret_cast<const int32_t*>(in.dst[2]), dev, st, true);
 }

@@ -322,6 +322,33 @@ def test_async_host_lookups_in_flight_match_device_lookups(stage1):
                 assert np.array_equal(v.numpy(), g[k], equal_nan=True), k
 
 
+def test_host_lookups_interleaved_with_device_lookups_keep_their_inputs():
+    # Host lookups stage their inputs in two slots used in turn, and each one's gather may run while the lookup
+    # before it is still in stage 2. Eight lookups are enqueued back to back on one stream, host and device
+    # lookups mixed, each with its own batch; k = 5 makes a slot's size no multiple of 16 bytes.
+    w = wl.WORKLOADS["tiny-4k"].scaled(k=5, batch=48)
+    kinds = ["host", "host", "device", "host", "host", "host", "device", "host"]
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
+        fill(cache, w)
+        qs = [wl.batch(w, i, device="cuda") for i in range(len(kinds))]
+        want = [gpu_lookup(cache, q) for q in qs]
+        stream = torch.cuda.current_stream()
+        outs = []
+        for kind, q in zip(kinds, qs):
+            if kind == "host":
+                hq = {k: _host_copy(q[k], "pinned") for k in ("emb", "prefix", "ids")}
+                o = L.alloc_result(w.batch, w.top_c, "cpu", pinned=True)
+                L.lacache_lookup_host_async(cache.h, hq["emb"], hq["prefix"], hq["ids"], o, stream)
+                outs.append((o, hq))
+            else:
+                outs.append((cache.lookup(q["emb"], q["prefix"], q["ids"], cuda_stream=stream), None))
+        stream.synchronize()
+        cache.sync()
+        for (o, _), g in zip(outs, want):
+            for k, v in o.items():
+                assert np.array_equal(v.cpu().numpy(), g[k], equal_nan=True), k
+
+
 def test_async_host_lookup_refuses_unmapped_or_misaligned_buffers():
     w = wl.WORKLOADS["tiny-4k"]
     with new_cache(w, L.LACACHE_STAGE1_TENSOR) as cache:
