@@ -13,8 +13,8 @@
 // The distance test first counts the differing bits of a prefix of P of the W words (the kernel's P parameter): a
 // pair whose prefix distance already exceeds the radius is out, since the prefix distance never exceeds the whole
 // one. With the radii the thresholds give, nearly every pair of unrelated signatures is out after the prefix
-// (prefix_words() picks P from the binomial tail of a random pair's distance), and the few left in each thread's
-// mask get the whole distance in a loop over that mask. P = W tests the whole signature at once.
+// (use_prefix() keeps the test where the binomial tail of a random pair's prefix distance says so), and the few
+// left in each thread's mask get the whole distance in a loop over that mask. P = W tests the whole signature.
 // Admitted (query, entry) pairs are queued in shared memory.
 // When the queue passes three quarters of its capacity, and at the end of the split, all warps take queue items two
 // at a time and compute the exact fp32 score over the gathered key row (each lane's 8-element chunks in order,
