@@ -82,6 +82,14 @@ def test_single_query_lookups_on_a_large_store_match_the_oracle(bits):
     _check_lsh_lookup(wl.WORKLOADS["mid-1m"].scaled(n=2_600_000, d=64, batch=8), bits, one_at_a_time=True)
 
 
+@pytest.mark.slow
+@pytest.mark.parametrize("bits", [256, 512])
+def test_lsh_lookup_at_full_size_matches_the_oracle(bits):
+    # mid-1m at full size (1,048,576 entries, B = 32), as the benchmark's SimHash line times it: the popcount scan
+    # with its prefix test, in its register form at 256 bits and its shared-memory ring form at 512
+    _check_lsh_lookup(wl.WORKLOADS["mid-1m"], bits)
+
+
 @pytest.mark.parametrize("top_c", [1, 32])
 @pytest.mark.parametrize("batch", [16, 64], ids=["popcount", "tensor"])
 def test_lsh_top_c_extremes_match_the_oracle(batch, top_c):
