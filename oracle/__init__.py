@@ -12,11 +12,11 @@ from .lookup import (CHECK_BOTH, CHECK_EMB, CHECK_TOKENS, HIT, MISS_KEY, REJECT,
                      Store, decide, lookahead, lookup, passes)
 from .serve import ServeLoop
 from .calibrate import calibrate, nearest_rank, pair_similarities
-from .lsh import hamming, lookup_lsh, projections, signatures
+from .lsh import LshKeyCheck, hamming, lookup_lsh, projections, signatures
 from .speculative import accepted_prefix
 from .shards import merge as merge_shards
 
 __all__ = ["round_to_bf16", "widen", "CHECK_BOTH", "CHECK_EMB", "CHECK_TOKENS", "HIT", "MISS_KEY", "REJECT",
            "KeyCheck", "Params", "Result", "Store", "decide", "lookahead", "lookup", "passes", "ServeLoop",
-           "calibrate", "nearest_rank", "pair_similarities", "hamming", "lookup_lsh", "projections", "signatures",
+           "calibrate", "nearest_rank", "pair_similarities", "LshKeyCheck", "hamming", "lookup_lsh", "projections", "signatures",
            "accepted_prefix", "merge_shards"]

@@ -39,10 +39,34 @@ def signatures(rows_bits, hyperplanes_bits, amb: float = AMBIGUOUS):
 
 def hamming(a_bits, b_bits) -> np.ndarray:
     """Hamming distances between every signature of a [n, b] and every one of b [m, b]: [n, m]."""
-    a = np.asarray(a_bits, dtype=np.int64)
-    b = np.asarray(b_bits, dtype=np.int64)
-    # bits differ where exactly one is set: a + b - 2ab summed over the bits
-    return a.sum(axis=1)[:, None] + b.sum(axis=1)[None, :] - 2 * (a @ b.T)
+    a = np.asarray(a_bits, dtype=np.float64)
+    b = np.asarray(b_bits, dtype=np.float64)
+    # bits differ where exactly one is set: a + b - 2ab summed over the bits (counts of at most b bits: integers,
+    # exact in fp64, which lets the product run as a library matrix product)
+    return np.rint(a.sum(axis=1)[:, None] + b.sum(axis=1)[None, :] - 2 * (a @ b.T)).astype(np.int64)
+
+
+class LshKeyCheck:
+    """The key check with the SimHash index as the cache search, fed block by block like KeyCheck: of each block
+    of entries, those whose signature is within `radius` of the query's are admitted to the exact check.
+
+    `kc` is the underlying KeyCheck (decide() takes it); ambiguous[q] is True if ambiguous signature bits of the
+    query or of an entry could move an entry with sim >= tau_c - 2e-3 across the Hamming radius."""
+
+    def __init__(self, q_bits, tau_c: float, hyperplanes_bits, radius: int):
+        self.hyperplanes_bits, self.radius = hyperplanes_bits, radius
+        self.q_sig, self.q_amb = signatures(q_bits, hyperplanes_bits)
+        self.kc = KeyCheck(q_bits, tau_c)
+        self.ambiguous = np.zeros(self.q_sig.shape[0], dtype=bool)
+
+    def add_rows(self, key_bits, j0: int) -> None:
+        e_sig, e_amb = signatures(key_bits, self.hyperplanes_bits)
+        hd = hamming(self.q_sig, e_sig)
+        s = self.kc.q @ widen(key_bits).T
+        slack = self.q_amb.sum(axis=1)[:, None] + e_amb.sum(axis=1)[None, :]
+        near = s >= self.kc.tau_c - 2e-3
+        self.ambiguous |= np.any(near & (slack > 0) & (np.abs(hd - self.radius) <= slack), axis=1)
+        self.kc.add_scores(s, j0, admitted=hd <= self.radius)
 
 
 def lookup_lsh(store: Store, queries: dict, params: Params, hyperplanes_bits, radius: int,
@@ -51,17 +75,9 @@ def lookup_lsh(store: Store, queries: dict, params: Params, hyperplanes_bits, ra
 
     Returns (Result, ambiguous): ambiguous[q] is True if ambiguous signature bits of the query or of an entry
     could move an entry with sim >= tau_c - 2e-3 across the Hamming radius."""
-    q_sig, q_amb = signatures(queries["emb"], hyperplanes_bits)
-    kc = KeyCheck(queries["emb"], params.tau_c)
-    ambiguous = np.zeros(q_sig.shape[0], dtype=bool)
+    lk = LshKeyCheck(queries["emb"], params.tau_c, hyperplanes_bits, radius)
     for j0 in range(0, store.n, block_rows):
-        rows = store.key[j0:min(store.n, j0 + block_rows)]
-        e_sig, e_amb = signatures(rows, hyperplanes_bits)
-        hd = hamming(q_sig, e_sig)
-        s = kc.q @ widen(rows).T
-        slack = q_amb.sum(axis=1)[:, None] + e_amb.sum(axis=1)[None, :]
-        near = s >= params.tau_c - 2e-3
-        ambiguous |= np.any(near & (slack > 0) & (np.abs(hd - radius) <= slack), axis=1)
-        kc.add_scores(s, j0, admitted=hd <= radius)
-    res = decide(kc, queries["prefix"], queries["ids"], params, lambda j: store.prefix[j], lambda j: store.ids[j])
-    return res, ambiguous
+        lk.add_rows(store.key[j0:min(store.n, j0 + block_rows)], j0)
+    res = decide(lk.kc, queries["prefix"], queries["ids"], params, lambda j: store.prefix[j],
+                 lambda j: store.ids[j])
+    return res, lk.ambiguous

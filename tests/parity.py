@@ -209,15 +209,21 @@ class StreamedOracle:
     check (A_q is a union over blocks). The prefix rows and ids of the entries stage 2 and the decision margin
     may need (every entry of each A_q: the margin of a rejection looks past the candidate cut) are then
     regenerated from the generator, never read back from the device. With no cache the store is generated on
-    `device` only for the oracle.
+    `device` only for the oracle. With `lsh` = (hyperplane bits, radius) the cache search is the SimHash index
+    (oracle.LshKeyCheck), and `ambiguous` marks the sampled queries that ambiguous signature bits could change.
     """
 
-    def __init__(self, w: wl.Workload, q: dict, sample, p: oracle.Params):
+    def __init__(self, w: wl.Workload, q: dict, sample, p: oracle.Params, lsh=None):
         self.w, self.q, self.p = w, q, p
         self.sample = np.asarray(sample)
         self.oq = oracle_queries(q, torch.as_tensor(self.sample))
-        self.kc = oracle.KeyCheck(self.oq["emb"], p.tau_c)
+        self.lk = oracle.LshKeyCheck(self.oq["emb"], p.tau_c, *lsh) if lsh is not None else None
+        self.kc = self.lk.kc if self.lk is not None else oracle.KeyCheck(self.oq["emb"], p.tau_c)
         self.device = "cuda"
+
+    @property
+    def ambiguous(self):
+        return self.lk.ambiguous if self.lk is not None else np.zeros(len(self.sample), dtype=bool)
 
     def fill(self, cache: L.LaCache | None, device="cuda") -> None:
         self.device = device
@@ -225,7 +231,7 @@ class StreamedOracle:
         for ch in wl.iter_store(self.w, device):
             if cache is not None:
                 cache.insert(ch["key"], ch["prefix"], ch["ids"], dtype)
-            self.kc.add_rows(_bits(ch["key"], self.w.key_dtype == "f32"), ch["j0"])
+            (self.lk or self.kc).add_rows(_bits(ch["key"], self.w.key_dtype == "f32"), ch["j0"])
             del ch
         if device != "cpu":
             torch.cuda.synchronize()

@@ -1,7 +1,7 @@
 """Parity at the full sizes of the large workloads, in the launch configuration the benchmark uses.
 
-large-16m (70 GB store) checks its whole batch of 128 queries against the streamed oracle, and batch-4m a
-stratified sample of 513 of its 8192 queries. serve-2m runs all 1000 steps. The oracle replays steps 0-2 from its
+large-16m (70 GB store) checks its whole batch of 128 queries against the streamed oracle, through the exact scan
+and through the SimHash index, and batch-4m a stratified sample of 513 of its 8192 queries. serve-2m runs all 1000 steps. The oracle replays steps 0-2 from its
 own state. Five seeded later steps are verified against the store rebuilt from the GPU's append log: every logged
 row is first checked, bit for bit, against the non-HIT query row the GPU reported. Every step is also checked for
 the properties that hold at any size: the append log, bit-exact appended rows, and both checks passing for every
@@ -78,6 +78,37 @@ def test_large_cache_near_hbm_capacity():
     """16,777,216 entries x 1024 dims (34 GB of keys), B = 128, Zipf(1.1) targets: every query of the batch."""
     rep = _check_streamed(wl.WORKLOADS["large-16m"], per_class=128, pairs_of_queries=True)
     assert rep.queries == 128
+
+
+def test_large_cache_through_the_simhash_index():
+    """16,777,216 entries x 1024 looked up through a 256-bit SimHash index (B = 128: the tensor-core Hamming scan
+    over the expanded index), every query of the batch against the streamed oracle. Queries whose outcome an
+    ambiguous signature bit could change are set aside (at most 1 in 50)."""
+    w = wl.WORKLOADS["large-16m"]
+    bits = 256
+    radius = wl.lsh_radius(w.tau_c, bits)
+    R = wl.hyperplanes(bits, w.d, device="cuda")
+    q = wl.batch(w, 0, device="cuda")
+    sample = np.arange(w.batch)
+    p = params(w)
+    so = StreamedOracle(w, q, sample, p, lsh=(wl.bf16_bits(R), radius))
+    with new_cache(w, L.LACACHE_STAGE1_LSH) as cache:
+        so.fill(cache)
+        L.lacache_enable_lsh(cache.h, bits, radius, R)
+        out = cache.lookup(q["emb"], q["prefix"], q["ids"])
+        torch.cuda.synchronize()
+        cache.sync()
+        assert cache.last_launch()[1] == L.LACACHE_STAGE1_LSH_TENSOR
+        g = {k: v.cpu().numpy() for k, v in out.items()}
+    res = so.result()
+    keep = np.nonzero(~so.ambiguous)[0]
+    sub = oracle.Result(**{f: getattr(res, f)[keep] for f in res.__dataclass_fields__})
+    rep = compare(g, sub, p, rows=sample[keep], pair_scores=lambda b, j: so.pair_scores(int(keep[b]), j))
+    log_report(f"{w.name} full size through the SimHash index ({w.batch - len(keep)} queries with ambiguous bits)",
+               rep)
+    assert len(keep) >= w.batch - max(2, w.batch // 50)
+    assert rep.exact + rep.band == len(keep) and rep.band <= max(1, len(keep) // 50)
+    assert rep.hits > 0 and rep.rejects > 0 and rep.misses > 0
 
 
 def test_large_batch_tensor_core_regime():

@@ -82,7 +82,7 @@ MUTATIONS = [
      "widen(rows_bits) @ widen(hyperplanes_bits)[::-1].T", LSH),
     ("signature-sign-strict", "lsh.py", "return p >= 0.0, np.abs(p) < amb", "return p > 0.0, np.abs(p) < amb", LSH),
     ("hamming-drops-factor-two", "lsh.py", "- 2 * (a @ b.T)", "- (a @ b.T)", LSH),
-    ("radius-exclusive", "lsh.py", "admitted=hd <= radius", "admitted=hd < radius", LSH),
+    ("radius-exclusive", "lsh.py", "admitted=hd <= self.radius", "admitted=hd < self.radius", LSH),
     ("nearest-rank-floor", "calibrate.py", "math.ceil(percentile / 100.0 * v.size)",
      "math.floor(percentile / 100.0 * v.size)", CAL),
     ("cap-is-max", "calibrate.py", "return min(cap, p), p", "return max(cap, p), p", CAL),
