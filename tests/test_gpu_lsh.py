@@ -132,17 +132,19 @@ def _check_lsh_lookup(w, bits, one_at_a_time=False):
     assert np.array_equal(res.status, exact.status) and np.array_equal(res.entry_id, exact.entry_id)
 
 
+@pytest.mark.parametrize("bits", [256, 512])
 @pytest.mark.parametrize("batch", [16, 64], ids=["popcount", "tensor"])
-def test_full_radius_equals_the_exact_scan_and_appends_are_signed(batch):
-    # radius = bits admits every pair: the queue overflows on every tile, and appended entries must be signed (in
-    # both the packed and the expanded form) before the next lookup
+def test_full_radius_equals_the_exact_scan_and_appends_are_signed(batch, bits):
+    # radius = bits admits every pair: the queue overflows on every tile (at 512 bits the popcount scan's ring form,
+    # whose queue is a quarter of the register form's), and appended entries must be signed (in both the packed
+    # and the expanded form) before the next lookup
     w = wl.WORKLOADS["serve-2m"].scaled(n=30_000, batch=batch, clusters=300)
-    R = wl.hyperplanes(256, w.d, device="cuda")
+    R = wl.hyperplanes(bits, w.d, device="cuda")
     with new_cache(w, L.LACACHE_STAGE1_TENSOR, capacity=w.n + 4 * w.batch) as exact_cache, \
             new_cache(w, L.LACACHE_STAGE1_LSH, capacity=w.n + 4 * w.batch) as lsh_cache:
         fill(exact_cache, w)
         fill(lsh_cache, w)
-        L.lacache_enable_lsh(lsh_cache.h, 256, 256, R)        # radius = bits: nothing is pruned
+        L.lacache_enable_lsh(lsh_cache.h, bits, bits, R)      # radius = bits: nothing is pruned
         for step in range(3):
             q = wl.batch(w, step, device="cuda")
             a = exact_cache.lookup(q["emb"], q["prefix"], q["ids"])
@@ -153,7 +155,7 @@ def test_full_radius_equals_the_exact_scan_and_appends_are_signed(batch):
             assert torch.allclose(a["cand_score"], b["cand_score"], atol=2e-3, equal_nan=True)
             exact_cache.append_misses(q["emb"], q["prefix"], q["ids"], a["status"])
             first, m = lsh_cache.append_misses(q["emb"], q["prefix"], q["ids"], b["status"])
-        sig = torch.empty((m, 8), dtype=torch.int32, device="cuda")
+        sig = torch.empty((m, bits // 32), dtype=torch.int32, device="cuda")
         L.lacache_read_signatures(lsh_cache.h, first, m, sig)
         torch.cuda.synchronize()
         # the appended entries are the last batch's non-HIT queries, in query order
@@ -161,7 +163,7 @@ def test_full_radius_equals_the_exact_scan_and_appends_are_signed(batch):
         assert len(miss) == m
         rows = wl.bf16_bits(q["emb"][miss])
     want, amb = oracle.signatures(rows, wl.bf16_bits(R))
-    assert not np.any((_unpack(sig.cpu().numpy().view(np.uint32), 256) != want) & ~amb)
+    assert not np.any((_unpack(sig.cpu().numpy().view(np.uint32), bits) != want) & ~amb)
 
 
 def test_lookup_before_the_index_is_enabled_is_refused():
