@@ -166,6 +166,30 @@ def test_full_radius_equals_the_exact_scan_and_appends_are_signed(batch, bits):
     assert not np.any((_unpack(sig.cpu().numpy().view(np.uint32), bits) != want) & ~amb)
 
 
+@pytest.mark.parametrize("batch", [8, 64], ids=["popcount", "tensor"])
+def test_host_buffer_lookups_through_the_index_match_device_lookups(batch):
+    # inputs from mapped pinned host memory: the gather kernel writes them, the query-signature kernel waits for
+    # it before reading, and three lookups are in flight on one stream (each gather runs under the stage 2 before)
+    w = wl.WORKLOADS["mid-1m"].scaled(n=40_000, batch=batch)
+    R = wl.hyperplanes(256, w.d, device="cuda")
+    with new_cache(w, L.LACACHE_STAGE1_LSH) as cache:
+        fill(cache, w)
+        L.lacache_enable_lsh(cache.h, 256, wl.lsh_radius(w.tau_c, 256), R)
+        qs = [wl.batch(w, i, device="cuda") for i in range(3)]
+        want = [gpu_lookup(cache, q) for q in qs]
+        hq = [{k: q[k].cpu().pin_memory() for k in ("emb", "prefix", "ids")} for q in qs]
+        outs = [L.alloc_result(w.batch, w.top_c, "cpu", pinned=True) for _ in qs]
+        stream = torch.cuda.current_stream()
+        for q, o in zip(hq, outs):
+            L.lacache_lookup_host_async(cache.h, q["emb"], q["prefix"], q["ids"], o, stream)
+        stream.synchronize()
+        cache.sync()
+        assert cache.last_launch()[1] == _expected_lsh_kernel(batch)
+        for o, g in zip(outs, want):
+            for k, v in o.items():
+                assert np.array_equal(v.numpy(), g[k], equal_nan=True), k
+
+
 def test_lookup_before_the_index_is_enabled_is_refused():
     w = wl.WORKLOADS["mid-1m"].scaled(n=5_000, batch=8)
     q = wl.batch(w, 0, device="cuda")
