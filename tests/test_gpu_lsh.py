@@ -83,10 +83,10 @@ def test_single_query_lookups_on_a_large_store_match_the_oracle(bits):
 
 
 @pytest.mark.slow
-@pytest.mark.parametrize("bits", [256, 512])
+@pytest.mark.parametrize("bits", [128, 256, 512])
 def test_lsh_lookup_at_full_size_matches_the_oracle(bits):
     # mid-1m at full size (1,048,576 entries, B = 32), as the benchmark's SimHash line times it: the popcount scan
-    # with its prefix test, in its register form at 256 bits and its shared-memory ring form at 512
+    # with its prefix test, in its register form at 128 and 256 bits and its shared-memory ring form at 512
     _check_lsh_lookup(wl.WORKLOADS["mid-1m"], bits)
 
 

@@ -93,6 +93,20 @@ def test_radius_at_least_b_is_the_exact_lookup():
         assert np.array_equal(getattr(exact, f), getattr(lsh, f), equal_nan=True), f
 
 
+def test_block_wise_check_is_the_whole_store_check():
+    # the store through the SimHash key check in blocks of 7 rows (the last one ragged) gives the result of one
+    # block: A_q is a union over blocks, and each block's ids are offset by its first row
+    st, qs = _small_case()
+    R = wl.bf16_bits(wl.hyperplanes(64, 32))
+    p = Params(0.9, 0.5, 8)
+    whole, amb1 = oracle.lookup_lsh(st, qs, p, R, radius=20)
+    blocks, amb2 = oracle.lookup_lsh(st, qs, p, R, radius=20, block_rows=7)
+    assert np.array_equal(amb1, amb2)
+    for f in ("status", "entry_id", "cand_id", "cand_score", "n_cand", "n_above", "margin"):
+        assert np.array_equal(getattr(whole, f), getattr(blocks, f), equal_nan=True), f
+    assert np.any(whole.n_cand > 0)
+
+
 def test_radius_zero_keeps_only_identical_signatures():
     st, qs = _small_case()
     R = wl.bf16_bits(wl.hyperplanes(64, 32))

@@ -83,6 +83,7 @@ MUTATIONS = [
     ("signature-sign-strict", "lsh.py", "return p >= 0.0, np.abs(p) < amb", "return p > 0.0, np.abs(p) < amb", LSH),
     ("hamming-drops-factor-two", "lsh.py", "- 2 * (a @ b.T)", "- (a @ b.T)", LSH),
     ("radius-exclusive", "lsh.py", "admitted=hd <= self.radius", "admitted=hd < self.radius", LSH),
+    ("lsh-block-offset-dropped", "lsh.py", "self.kc.add_scores(s, j0,", "self.kc.add_scores(s, 0,", LSH),
     ("nearest-rank-floor", "calibrate.py", "math.ceil(percentile / 100.0 * v.size)",
      "math.floor(percentile / 100.0 * v.size)", CAL),
     ("cap-is-max", "calibrate.py", "return min(cap, p), p", "return max(cap, p), p", CAL),
