@@ -71,7 +71,8 @@ typedef enum {
                                      scan on two-CTA clusters (one M=256 MMA per pair of SMs), chosen for batches
                                      of more than 128 queries */
   LACACHE_STAGE1_LSH_TENSOR = 5   /* reported by lacache_last_launch only: the SimHash form with the Hamming test on
-                                     the tensor cores, chosen for batches of at least 40 queries */
+                                     the tensor cores, chosen for batches of at least 48 queries at 256 bits
+                                     and of at least 40 at 128 and 512 bits */
 } lacache_stage1;
 
 /* Ensemble of m lookahead checks (section 3.4, "Analysis"; Figure 6): every entry and query carries one k-token
@@ -194,10 +195,11 @@ lacache_status lacache_append_misses(lacache_t* h, int32_t B, const void* q_emb_
  * hyperplanes_dev ([bits x d] bf16, copied into the handle; random normal rows give random-hyperplane LSH). With
  * cfg->stage1 == LACACHE_STAGE1_LSH a lookup applies the exact key check only to the entries whose signature
  * differs from the query's in at most `radius` bits; stage 2 is unchanged. Existing entries are signed now and
- * later inserts and appends are signed as they arrive. Batches of fewer than 40 queries compare the packed
- * signatures by population counts; larger ones run the Hamming test on the tensor cores, over a copy of the
- * signatures expanded to one byte per bit. Allocates (capacity + max_batch) * bits / 8 bytes for the signatures and,
- * when max_batch >= 40, capacity * bits bytes (whole 128-entry blocks) for the expanded copy.
+ * later inserts and appends are signed as they arrive. Batches of fewer than T queries (T = 48 at 256 bits, 40 at
+ * 128 and 512) compare the packed signatures by population counts; larger ones run the Hamming test on the tensor
+ * cores, over a copy of the signatures expanded to one byte per bit. Allocates (capacity + max_batch) * bits / 8
+ * bytes for the signatures and, when max_batch >= T, capacity * bits bytes (whole 128-entry blocks) for the
+ * expanded copy.
  * Asynchronous on cuda_stream; calling it again replaces the index. A lookup on a handle whose cfg->stage1 is
  * LACACHE_STAGE1_LSH returns LACACHE_ERR_INVALID_ARG, and runs nothing, until this call has been made. */
 lacache_status lacache_enable_lsh(lacache_t* h, int32_t bits, int32_t radius, const void* hyperplanes_dev,

@@ -371,7 +371,7 @@ lacache_status run_lookup(lacache* h, int32_t B, const void* q_emb, const void* 
               : lc::launch_sign_queries(a.q, B, c.d, h->hyper, h->lsh_bits, h->qsig, st, gathered);
       if (e == cudaSuccess) {
         lc::LshArgs l{h->sig, h->qsig, h->lsh_bits / 32, h->lsh_radius, h->sig_index};
-        if (B >= lc::kLshTensorMinBatch && h->sig_index) {
+        if (B >= lc::lsh_tensor_min_batch(h->lsh_bits) && h->sig_index) {
           e = lc::launch_stage1_lsh_tc(a, l, h->num_sms, h->max_splits, st, &splits);
           kernel = LACACHE_STAGE1_LSH_TENSOR;
         } else {
@@ -723,7 +723,8 @@ lacache_status lacache_enable_lsh(lacache_t* h, int32_t bits, int32_t radius, co
   const int words = bits / 32;
   const lacache_config& c = h->cfg;
   // the expanded copy only where batches can be large enough to use it
-  const size_t index_bytes = c.max_batch >= lc::kLshTensorMinBatch ? lc::lsh_index_bytes(c.capacity, bits) : 0;
+  const size_t index_bytes =
+      c.max_batch >= lc::lsh_tensor_min_batch(bits) ? lc::lsh_index_bytes(c.capacity, bits) : 0;
   if (cudaMalloc(&h->sig, (size_t)c.capacity * words * 4) != cudaSuccess ||
       cudaMalloc(&h->qsig, (size_t)c.max_batch * words * 4) != cudaSuccess ||
       cudaMalloc(&h->hyper, (size_t)bits * c.d * 2) != cudaSuccess ||

@@ -155,14 +155,18 @@ struct LshArgs {
   const uint8_t* index;    // the same signatures as e4m3 +-1 bytes in swizzled 128-entry blocks (lsh_tc.cu)
 };
 // Popcount scan (small batches) and the tensor-core scan over the expanded index (batches of at least
-// kLshTensorMinBatch queries).
+// lsh_tensor_min_batch(bits) queries).
 // *ring: the launch runs the scan's shared-memory ring form (the only form with bounded waits, so the only one a
 // stall injection, a.inject_stall, acts on).
 cudaError_t launch_stage1_lsh(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits, cudaStream_t st,
                               int* splits, bool* ring);
 cudaError_t launch_stage1_lsh_tc(const Stage1Args& a, const LshArgs& l, int num_sms, int max_splits,
                                  cudaStream_t st, int* splits);
-constexpr int kLshTensorMinBatch = 40;
+// The switch between them, measured per lookup step on mid-1m with both scans forced (popcount scan with its prefix
+// test / tensor-core scan, us): 128 bits, B = 32 48.1 / 56.7, B = 40 61.0 / 57.4; 256 bits, B = 40 74.0 / 80.8,
+// B = 48 81.6 / 81.6, B = 64 97.5 / 82.4; 512 bits, B = 32 77.5 / 97.6, B = 40 104.2 / 98.9. Past 32 queries the
+// popcount scan makes a second pass over the index.
+inline int lsh_tensor_min_batch(int bits) { return bits == 256 ? 48 : 40; }
 // Bytes of the expanded index for `capacity` entries (whole 128-entry blocks of `bits` bytes each), and its update
 // from the packed signatures of entries [first, first + n).
 size_t lsh_index_bytes(int64_t capacity, int bits);

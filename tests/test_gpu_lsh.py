@@ -51,11 +51,14 @@ def test_signatures_match_the_oracle(bits):
     assert amb.mean() < 1e-3
 
 
-def _expected_lsh_kernel(batch):
-    return L.LACACHE_STAGE1_LSH_TENSOR if batch >= 40 else L.LACACHE_STAGE1_LSH
+def _expected_lsh_kernel(batch, bits):
+    # the tensor-core scan from 48 queries at 256 bits and from 40 at 128 and 512 bits
+    return L.LACACHE_STAGE1_LSH_TENSOR if batch >= (48 if bits == 256 else 40) else L.LACACHE_STAGE1_LSH
 
 
 # popcount-1 / -2: a pass of fewer queries than one group of 8 (only their distances are computed);
+# tensor-40: the tensor-core scan at 128 and 512 bits, two passes of the popcount scan at 256 bits (its switch is at
+# 48);
 # popcount-36: two passes of 32 queries (the handle's max_batch is below the tensor scan's minimum, so it keeps no
 # expanded index); tensor-200: two passes of 128 queries at 128 and 256 bits, four of 64 at 512, ragged last pass
 @pytest.mark.parametrize("batch", [1, 2, 5, 32, 36, 40, 64, 200],
@@ -114,7 +117,7 @@ def _check_lsh_lookup(w, bits, one_at_a_time=False):
             g = {k: np.concatenate([r[k] for r in parts]) for k in parts[0]}
         else:
             g = gpu_lookup(cache, q)
-            assert cache.last_launch()[1] == _expected_lsh_kernel(batch)
+            assert cache.last_launch()[1] == _expected_lsh_kernel(batch, bits)
     oq = oracle_queries(q)
     p = params(w)
     res, amb = oracle.lookup_lsh(st, oq, p, wl.bf16_bits(R), radius)
@@ -149,7 +152,7 @@ def test_full_radius_equals_the_exact_scan_and_appends_are_signed(batch, bits):
             q = wl.batch(w, step, device="cuda")
             a = exact_cache.lookup(q["emb"], q["prefix"], q["ids"])
             b = lsh_cache.lookup(q["emb"], q["prefix"], q["ids"])
-            assert lsh_cache.last_launch()[1] == _expected_lsh_kernel(batch)
+            assert lsh_cache.last_launch()[1] == _expected_lsh_kernel(batch, bits)
             assert torch.equal(a["status"], b["status"]) and torch.equal(a["entry_id"], b["entry_id"])
             assert torch.equal(a["cand_id"], b["cand_id"])
             assert torch.allclose(a["cand_score"], b["cand_score"], atol=2e-3, equal_nan=True)
@@ -171,10 +174,11 @@ def test_host_buffer_lookups_through_the_index_match_device_lookups(batch):
     # inputs from mapped pinned host memory: the gather kernel writes them, the query-signature kernel waits for
     # it before reading, and three lookups are in flight on one stream (each gather runs under the stage 2 before)
     w = wl.WORKLOADS["mid-1m"].scaled(n=40_000, batch=batch)
-    R = wl.hyperplanes(256, w.d, device="cuda")
+    bits = 256
+    R = wl.hyperplanes(bits, w.d, device="cuda")
     with new_cache(w, L.LACACHE_STAGE1_LSH) as cache:
         fill(cache, w)
-        L.lacache_enable_lsh(cache.h, 256, wl.lsh_radius(w.tau_c, 256), R)
+        L.lacache_enable_lsh(cache.h, bits, wl.lsh_radius(w.tau_c, bits), R)
         qs = [wl.batch(w, i, device="cuda") for i in range(3)]
         want = [gpu_lookup(cache, q) for q in qs]
         hq = [{k: q[k].cpu().pin_memory() for k in ("emb", "prefix", "ids")} for q in qs]
@@ -184,7 +188,7 @@ def test_host_buffer_lookups_through_the_index_match_device_lookups(batch):
             L.lacache_lookup_host_async(cache.h, q["emb"], q["prefix"], q["ids"], o, stream)
         stream.synchronize()
         cache.sync()
-        assert cache.last_launch()[1] == _expected_lsh_kernel(batch)
+        assert cache.last_launch()[1] == _expected_lsh_kernel(batch, bits)
         for o, g in zip(outs, want):
             for k, v in o.items():
                 assert np.array_equal(v.numpy(), g[k], equal_nan=True), k
