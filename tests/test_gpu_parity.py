@@ -15,7 +15,7 @@ from paper_2608_01718_gb300 import build
 from paper_2608_01718_gb300 import lacache as L
 from paper_2608_01718_gb300 import workloads as wl
 
-from parity import (TOL, Report, compare, fill, gpu_lookup, log_report, new_cache, oracle_queries, oracle_store,
+from parity import (Report, compare, fill, gpu_lookup, log_report, new_cache, oracle_queries, oracle_store,
                     pair_scores_fn, params)
 
 pytestmark = pytest.mark.gpu
