@@ -1,0 +1,56 @@
+"""Parity of the ensemble of lookahead checks (section 3.4: a hit needs every model's prefix similarity to clear
+its threshold) on seeded random configurations: each case draws the number of models (2-8), each model's prefix
+dimension and threshold, the noise on near-duplicates' prefixes, a mix with prefix-mimicking collisions, the store
+size, d, the batch, top_c and the stage-1 kernel, and compares the lookup through the C ABI with the oracle under
+the usual rules (exact outside the 2e-3 decision margin; an in-band HIT must still pass every check)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_01718_gb300 import build
+from paper_2608_01718_gb300 import lacache as L
+from paper_2608_01718_gb300 import workloads as wl
+
+from parity import compare, fill, gpu_lookup, log_report, new_cache, oracle_queries, oracle_store, pair_scores_fn, params
+
+pytestmark = pytest.mark.gpu
+
+KERNELS = [L.LACACHE_STAGE1_AUTO, L.LACACHE_STAGE1_TENSOR, L.LACACHE_STAGE1_STREAM]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def library():
+    if not torch.cuda.is_available():
+        pytest.fail("GPU tests need a CUDA device")
+    build.build()
+    L.load()
+
+
+def _draw(seed):
+    rng = np.random.default_rng(20261204 + seed)
+    m = int(rng.integers(2, 9))
+    dims = tuple(int(rng.choice([8, 64, 384, 768, 1024])) for _ in range(m))
+    taus = tuple(float(rng.choice([0.5, 0.7, 0.9])) for _ in range(m))
+    w = wl.WORKLOADS["ensemble-1m"].scaled(
+        n=int(rng.choice([300, 7000, 40_000])), d=int(rng.choice([256, 768])), batch=int(rng.choice([1, 8, 48, 200])),
+        top_c=int(rng.choice([1, 8, 16])), clusters=int(rng.choice([8, 64, 500])), prefix_dims=dims,
+        tau_a_models=taus, near_prefix_sigma=float(rng.choice([0.0, 0.3, 0.6])))
+    return w, KERNELS[int(rng.integers(0, len(KERNELS)))]
+
+
+@pytest.mark.parametrize("seed", range(16))
+def test_random_ensemble_configuration_matches_the_oracle(seed):
+    w, stage1 = _draw(seed)
+    st = oracle_store(w)
+    with new_cache(w, stage1) as cache:
+        fill(cache, w)
+        q = wl.batch(w, 0, device="cuda")
+        g = gpu_lookup(cache, q)
+    assert g["prefix_scores"].shape == (w.batch, len(w.prefix_dims))
+    p = params(w)
+    oq = oracle_queries(q)
+    rep = compare(g, oracle.lookup(st, oq, p), p, pair_scores=pair_scores_fn(st, oq))
+    log_report(f"random ensemble seed={seed} n={w.n} d={w.d} B={w.batch} c={w.top_c} dims={w.prefix_dims} "
+               f"tau_a={w.tau_a_models} sigma={w.near_prefix_sigma} stage1={stage1}", rep)
+    assert rep.exact + rep.band == w.batch
