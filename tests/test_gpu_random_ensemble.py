@@ -54,3 +54,27 @@ def test_random_ensemble_configuration_matches_the_oracle(seed):
     log_report(f"random ensemble seed={seed} n={w.n} d={w.d} B={w.batch} c={w.top_c} dims={w.prefix_dims} "
                f"tau_a={w.tau_a_models} sigma={w.near_prefix_sigma} stage1={stage1}", rep)
     assert rep.exact + rep.band == w.batch
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_random_ensemble_through_the_simhash_index(seed):
+    # the same ensembles, stage 1 through a SimHash index (the radius the threshold gives): stage 2's m checks
+    # are independent of how the candidates were found
+    w, _ = _draw(100 + seed)
+    bits = (128, 256, 512)[seed % 3]
+    radius = wl.lsh_radius(w.tau_c, bits)
+    R = wl.hyperplanes(bits, w.d, device="cuda")
+    st = oracle_store(w)
+    with new_cache(w, L.LACACHE_STAGE1_LSH) as cache:
+        fill(cache, w)
+        L.lacache_enable_lsh(cache.h, bits, radius, R)
+        q = wl.batch(w, 0, device="cuda")
+        g = gpu_lookup(cache, q)
+    p = params(w)
+    res, amb = oracle.lookup_lsh(st, oracle_queries(q), p, wl.bf16_bits(R), radius)
+    keep = np.nonzero(~amb)[0]
+    sub = oracle.Result(**{f: getattr(res, f)[keep] for f in res.__dataclass_fields__})
+    rep = compare(g, sub, p, rows=keep)
+    log_report(f"random ensemble simhash seed={seed} n={w.n} B={w.batch} dims={w.prefix_dims} bits={bits}", rep)
+    assert len(keep) >= w.batch - min(2, max(1, w.batch // 50))
+    assert rep.exact + rep.band == len(keep)
