@@ -78,3 +78,36 @@ def test_random_ensemble_through_the_simhash_index(seed):
     log_report(f"random ensemble simhash seed={seed} n={w.n} B={w.batch} dims={w.prefix_dims} bits={bits}", rep)
     assert len(keep) >= w.batch - min(2, max(1, w.batch // 50))
     assert rep.exact + rep.band == len(keep)
+
+
+def test_ensemble_host_lookups_and_appends():
+    # an ensemble's prefix rows are pd = sum of the models' dims wide: host lookups stage them, appends copy them
+    w = wl.WORKLOADS["ensemble-1m"].scaled(n=9000, batch=40, prefix_dims=(1024, 8, 384))
+    assert w.pd == 1416
+    with new_cache(w, L.LACACHE_STAGE1_TENSOR, capacity=w.n + 2 * w.batch) as cache:
+        fill(cache, w)
+        qs = [wl.batch(w, i, device="cuda") for i in range(2)]
+        want = [gpu_lookup(cache, q) for q in qs]
+        hq = [{k: q[k].cpu().pin_memory() for k in ("emb", "prefix", "ids")} for q in qs]
+        outs = [L.alloc_result(w.batch, w.top_c, "cpu", pinned=True, models=3) for _ in qs]
+        stream = torch.cuda.current_stream()
+        for q, o in zip(hq, outs):
+            L.lacache_lookup_host_async(cache.h, q["emb"], q["prefix"], q["ids"], o, stream)
+        stream.synchronize()
+        cache.sync()
+        for o, g in zip(outs, want):
+            for k, v in o.items():
+                assert np.array_equal(v.numpy(), g[k], equal_nan=True), k
+        q = qs[0]
+        status = torch.as_tensor(want[0]["status"], device="cuda")
+        first, m = cache.append_misses(q["emb"], q["prefix"], q["ids"], status)
+        miss = torch.nonzero(status != L.LACACHE_HIT).flatten()
+        assert m == len(miss) and m > 0
+        key = torch.empty((m, w.d), dtype=torch.bfloat16, device="cuda")
+        pre = torch.empty((m, w.pd), dtype=torch.bfloat16, device="cuda")
+        ids = torch.empty((m, w.k), dtype=torch.int32, device="cuda")
+        L.lacache_read_rows(cache.h, first, m, key=key, prefix=pre, ids=ids)
+        torch.cuda.synchronize()
+        assert torch.equal(key.view(torch.int16), q["emb"][miss].view(torch.int16))
+        assert torch.equal(pre.view(torch.int16), q["prefix"][miss].view(torch.int16))
+        assert torch.equal(ids, q["ids"][miss])
