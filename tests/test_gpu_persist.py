@@ -47,3 +47,42 @@ def test_saved_cache_loads_and_looks_up_identically(name, tmp_path):
         assert first == w.n and m == int((after["status"] != L.LACACHE_HIT).sum())
     finally:
         loaded.close()
+
+
+def test_saved_simhash_cache_takes_its_index_again(tmp_path):
+    # the index is not saved: the loaded handle (still configured for the SimHash stage) refuses lookups until
+    # lacache_enable_lsh signs its entries again, then looks up as the saved one did, appends included
+    w = wl.WORKLOADS["mid-1m"].scaled(n=20_000, batch=16)
+    bits = 256
+    radius = wl.lsh_radius(w.tau_c, bits)
+    R = wl.hyperplanes(bits, w.d, device="cuda")
+    path = str(tmp_path / "cache.lacache")
+    q = wl.batch(w, 0, device="cuda")
+    with new_cache(w, L.LACACHE_STAGE1_LSH) as cache:
+        fill(cache, w)
+        L.lacache_enable_lsh(cache.h, bits, radius, R)
+        before = {k: v.clone() for k, v in cache.lookup(q["emb"], q["prefix"], q["ids"]).items()}
+        cache.sync()
+        cache.save(path)
+    loaded = L.LaCache.load(path, capacity=w.n + w.batch)
+    try:
+        with pytest.raises(L.LacacheError) as e:
+            loaded.lookup(q["emb"], q["prefix"], q["ids"])
+        assert e.value.status == L.LACACHE_ERR_INVALID_ARG
+        L.lacache_enable_lsh(loaded.h, bits, radius, R)
+        after = loaded.lookup(q["emb"], q["prefix"], q["ids"])
+        loaded.sync()
+        assert loaded.last_launch()[1] == L.LACACHE_STAGE1_LSH
+        for k in before:
+            assert torch.equal(before[k].view(torch.uint8), after[k].view(torch.uint8)), k
+        first, m = loaded.append_misses(q["emb"], q["prefix"], q["ids"], after["status"])
+        again = loaded.lookup(q["emb"], q["prefix"], q["ids"])
+        loaded.sync()
+        # every appended query now finds its own row (an exact copy) through the index
+        miss = torch.nonzero(after["status"] != L.LACACHE_HIT).flatten()
+        assert m == len(miss)
+        got = again["cand_id"][miss]
+        want = torch.arange(first, first + m, device="cuda", dtype=got.dtype)
+        assert torch.all((got == want[:, None]).any(dim=1))
+    finally:
+        loaded.close()
