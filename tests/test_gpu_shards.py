@@ -136,3 +136,45 @@ def test_merged_key_score_when_a_shard_hit_falls_past_the_cut():
     assert int(merged["status"][0]) == L.LACACHE_REJECT and float(merged["key_score"][0]) == 1.0
     assert merged["cand_id"][0].tolist() == [0, 2] and int(merged["entry_id"][0]) == -1
     assert float(merged["prefix_score"][0]) == 0.0
+
+
+def test_merged_simhash_shards_equal_the_whole_store_lookup():
+    # every shard signs its own rows with the same hyperplanes, so each admits exactly its part of the whole
+    # store's admitted pairs: the merge equals the whole-store lookup through the index
+    w = wl.WORKLOADS["mid-1m"].scaled(n=30_000, batch=16)
+    cuts = (0, 11_111, 30_000)
+    bits = 256
+    radius = wl.lsh_radius(w.tau_c, bits)
+    R = wl.hyperplanes(bits, w.d, device="cuda")
+    B, c = w.batch, w.top_c
+    q = wl.batch(w, 0, device="cuda")
+    with new_cache(w, L.LACACHE_STAGE1_LSH) as whole:
+        fill(whole, w)
+        L.lacache_enable_lsh(whole.h, bits, radius, R)
+        ref = L.alloc_result(B, c, "cuda", candidates=True)
+        whole.lookup(q["emb"], q["prefix"], q["ids"], out=ref)
+        torch.cuda.synchronize()
+        whole.sync()
+    gathered = torch.zeros((len(cuts) - 1, sharded.record_bytes(B, c, 1)), dtype=torch.uint8, device="cuda")
+    shards = []
+    for g, (a, b) in enumerate(zip(cuts, cuts[1:])):
+        with new_cache(w, L.LACACHE_STAGE1_LSH, capacity=b - a) as part:
+            fill_range(part, w, a, b)
+            L.lacache_enable_lsh(part.h, bits, radius, R)
+            rec = sharded.views(gathered[g], B, c, 1)
+            part.lookup(q["emb"], q["prefix"], q["ids"], out={**L.alloc_result(B, c, "cuda", candidates=False), **rec})
+            torch.cuda.synchronize()
+            part.sync()
+        shards.append((rec, a))
+    merged = L.alloc_result(B, c, "cuda", candidates=True)
+    L.lacache_merge_shards(shards, c, 1, merged)
+    torch.cuda.synchronize()
+    got = {k: v.cpu().numpy() for k, v in merged.items()}
+    for k, v in ref.items():
+        assert np.array_equal(got[k], v.cpu().numpy(), equal_nan=True), k
+    p = params(w)
+    res, amb = oracle.lookup_lsh(oracle_store(w), oracle_queries(q), p, wl.bf16_bits(R), radius)
+    keep = np.nonzero(~amb)[0]
+    rep = compare(got, oracle.Result(**{f: getattr(res, f)[keep] for f in res.__dataclass_fields__}), p, rows=keep)
+    log_report(f"simhash: {len(cuts) - 1} shards merged, n={w.n} B={B}", rep)
+    assert rep.exact + rep.band == len(keep) and len(keep) >= B - 1
