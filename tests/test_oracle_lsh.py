@@ -107,6 +107,30 @@ def test_block_wise_check_is_the_whole_store_check():
     assert np.any(whole.n_cand > 0)
 
 
+def test_an_ambiguous_bit_at_the_radius_marks_the_query():
+    # query 0's projection on hyperplane 0 is exactly zero (an ambiguous bit); entry 0 clears the key threshold and
+    # differs from it in that bit only, so at radius 0 the entry's admission hangs on that bit and the query is
+    # marked. Query 1 has no zero projection and an identical entry: not marked.
+    d = 8
+    R = np.zeros((4, d), np.float32)
+    R[np.arange(4), np.arange(4)] = 1.0
+    q = np.zeros((2, d), np.float32)
+    q[0, 1:5] = 0.5
+    q[1, 0:4] = 0.5
+    k = np.zeros((2, d), np.float32)
+    k[0, 0], k[0, 1:5] = -0.25, 0.5        # <q0, k0> = 1, sign differs on hyperplane 0 only
+    k[1] = q[1]
+    kb, qb, rb = oracle.round_to_bf16(k), oracle.round_to_bf16(q), oracle.round_to_bf16(R)
+    P = oracle.round_to_bf16(np.eye(2, d, dtype=np.float32))
+    T = np.arange(6, dtype=np.int32).reshape(2, 3)
+    st = Store.of(kb, P, T)
+    qsig, qamb = oracle.signatures(qb, rb)
+    assert qamb[0, 0] and not qamb[1].any()
+    assert oracle.hamming(qsig, oracle.signatures(kb, rb)[0])[0, 0] == 1
+    _, amb = oracle.lookup_lsh(st, {"emb": qb, "prefix": P, "ids": T}, Params(0.9, 0.5, 2), rb, radius=0)
+    assert amb.tolist() == [True, False]
+
+
 def test_radius_zero_keeps_only_identical_signatures():
     st, qs = _small_case()
     R = wl.bf16_bits(wl.hyperplanes(64, 32))

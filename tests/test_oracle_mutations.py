@@ -84,6 +84,8 @@ MUTATIONS = [
     ("hamming-drops-factor-two", "lsh.py", "- 2 * (a @ b.T)", "- (a @ b.T)", LSH),
     ("radius-exclusive", "lsh.py", "admitted=hd <= self.radius", "admitted=hd < self.radius", LSH),
     ("lsh-block-offset-dropped", "lsh.py", "self.kc.add_scores(s, j0,", "self.kc.add_scores(s, 0,", LSH),
+    ("ambiguity-ignores-query-bits", "lsh.py", "slack = self.q_amb.sum(axis=1)[:, None] +",
+     "slack = 0 * self.q_amb.sum(axis=1)[:, None] +", LSH),
     ("nearest-rank-floor", "calibrate.py", "math.ceil(percentile / 100.0 * v.size)",
      "math.floor(percentile / 100.0 * v.size)", CAL),
     ("cap-is-max", "calibrate.py", "return min(cap, p), p", "return max(cap, p), p", CAL),
