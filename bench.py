@@ -894,6 +894,53 @@ def run_calibration(args):
     return 0
 
 
+VERIFY = {"verify-256": (256, 32)}   # queries, draft tokens: the serve loop's batch (serve-2m) and its k
+
+
+def run_verify(args):
+    """Draft verification of the speculative prefix reuse (section 3.3): per query, the number of leading draft
+    tokens with P_f >= P_g, -1 for a served query. Synthetic token probabilities (uniform) and statuses (half
+    served); one call per step."""
+    import torch
+
+    from paper_2608_01718_gb300 import build
+    from paper_2608_01718_gb300 import lacache as L
+    B, k = VERIFY[args.workload]
+    build.build()
+    g = torch.Generator(device="cuda").manual_seed(20261205)
+    p_target = torch.rand((B, k), generator=g, device="cuda")
+    p_draft = torch.rand((B, k), generator=g, device="cuda")
+    status = torch.where(torch.rand(B, generator=g, device="cuda") < 0.5, L.LACACHE_HIT,
+                         L.LACACHE_REJECT).to(torch.uint8)
+    accepted = torch.empty(B, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream()
+    for _ in range(max(3, args.warmup)):
+        L.lacache_verify_draft(p_target, p_draft, status, accepted, stream)
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    ev0.record(stream)
+    for _ in range(args.steps):
+        L.lacache_verify_draft(p_target, p_draft, status, accepted, stream)
+    ev1.record(stream)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    peaks, src = load_peaks()
+    bytes_ = 2 * B * k * 4 + B + 4 * B
+    acc = accepted.cpu()
+    line = {"metric": "draft verifications/s (section 3.3 prefix reuse)", "value": B / (ms / 1e3),
+            "unit": "queries/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+            "higher_is_better": True, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": args.workload, "queries": B, "draft_tokens": k, "served_fraction": 0.5},
+            "roofline": {"bound": "hbm", "achieved": bytes_ / (ms / 1e3) / 1e9, "peak": peaks["hbm_gbs"],
+                         "unit": "GB/s", "frac": bytes_ / (ms / 1e3) / 1e9 / peaks["hbm_gbs"],
+                         "peak_source": f"{src} (copy bandwidth)",
+                         "note": f"{bytes_} bytes a call: bound by launch and memory latency, not bandwidth"},
+            "result": {"served": int((acc == -1).sum()), "mean_accepted": float(acc[acc >= 0].float().mean())},
+            "gpu_launches": args.steps}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
     if args.gpus > 1 and "WORLD_SIZE" not in os.environ:
@@ -905,6 +952,8 @@ def main():
     from paper_2608_01718_gb300 import workloads as wl
     if args.workload in CALIBRATION:
         return run_calibration(args)
+    if args.workload in VERIFY:
+        return run_verify(args)
     w = wl.WORKLOADS[args.workload]
     if args.entries:
         w = w.scaled(n=args.entries)
